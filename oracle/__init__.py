@@ -1,0 +1,220 @@
+"""Plain fp64 CPU oracle for FLARE's block-denoising attention step.
+
+TEST INFRASTRUCTURE ONLY.  Only the tests, ``__graft_entry__.smoke()`` and the
+CPU-baseline leg of ``bench.py`` may import this package.  The product library
+never links or loads it, and it shares no code with the CUDA path.
+
+The arithmetic lives in ``flare_oracle.c`` (fp64, optional OpenMP over
+(request, head) items); this module compiles it with the system C compiler and
+marshals numpy arrays into it.  What each routine computes, and which equation
+of the paper it follows, is documented in the C file:
+
+* :func:`gdr_per_token` -- gated delta rule token by token (Eq. per-step-fwd),
+  block-end readout (Eq. noisy-block-fwd), commit at the accepted length.
+* :func:`gdr_chunked` -- the same quantities through the chunkwise WY/UT form
+  (Eq. chunk-state, Eq. f-blk); used only to pin :func:`gdr_per_token`.
+* :func:`gather_prefix` -- dense copy of a request's paged prefix.
+* :func:`block_softmax` -- softmax retrieval (Eq. softmax-retrieval) under the
+  Diffusion-Trust block mask over the paged prefix plus the block.
+
+Inputs may be bf16 (passed as raw ``uint16`` bit patterns), fp32 or fp64.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import sysconfig
+from pathlib import Path
+
+import numpy as np
+
+_HERE = Path(__file__).resolve().parent
+_SRC = _HERE / "flare_oracle.c"
+_LIB = _HERE / "_flare_oracle.so"
+_lib = None
+
+BF16, F32, F64 = 0, 1, 2
+
+
+def build(force: bool = False) -> Path:
+    """Compile the oracle into ``oracle/_flare_oracle.so`` (gcc, -O2, OpenMP if available)."""
+    if _LIB.exists() and not force and _LIB.stat().st_mtime >= _SRC.stat().st_mtime:
+        return _LIB
+    cc = os.environ.get("CC", "gcc")
+    tmp = _LIB.with_suffix(f".{os.getpid()}.tmp")
+    base = [cc, "-O2", "-std=c11", "-shared", "-fPIC", str(_SRC), "-o", str(tmp), "-lm"]
+    try:
+        subprocess.run(base[:1] + ["-fopenmp"] + base[1:], check=True, capture_output=True)
+    except subprocess.CalledProcessError:
+        subprocess.run(base, check=True, capture_output=True)
+    os.replace(tmp, _LIB)
+    return _LIB
+
+
+def _load():
+    global _lib
+    if _lib is None:
+        build()
+        lib = ctypes.CDLL(str(_LIB))
+        P, I, D = ctypes.c_void_p, ctypes.c_int, ctypes.c_double
+        lib.oracle_gdr_per_token.argtypes = [I] * 6 + [D, I, P, P, P, I, P, P, I, P, I, P, P, P, P, P, I]
+        lib.oracle_gdr_per_token.restype = I
+        lib.oracle_gdr_chunked.argtypes = [I] * 6 + [D, I, P, P, P, I, P, P, I, P, I, P, P, P, P, I]
+        lib.oracle_gdr_chunked.restype = I
+        lib.oracle_gather_prefix.argtypes = [I] * 7 + [P, P, P, P]
+        lib.oracle_gather_prefix.restype = I
+        lib.oracle_block_softmax.argtypes = [I] * 8 + [D, I, I, P, P, P, P, P, P, P, P, P, I]
+        lib.oracle_block_softmax.restype = I
+        lib.oracle_max_threads.argtypes = []
+        lib.oracle_max_threads.restype = I
+        _lib = lib
+    return _lib
+
+
+def max_threads() -> int:
+    return int(_load().oracle_max_threads())
+
+
+def _arr(x):
+    """Return (contiguous numpy array, dtype code) for bf16/fp32/fp64 inputs.
+
+    Accepts numpy arrays or CPU torch tensors; bf16 torch tensors are passed as
+    their raw 16-bit patterns (the C side widens them exactly)."""
+    if x is None:
+        return None, F64
+    if hasattr(x, "detach"):  # torch tensor
+        import torch
+
+        x = x.detach().cpu().contiguous()
+        if x.dtype == torch.bfloat16:
+            return x.view(torch.int16).numpy().view(np.uint16), BF16
+        x = x.numpy()
+    x = np.ascontiguousarray(x)
+    if x.dtype == np.uint16:
+        return x, BF16
+    if x.dtype == np.float32:
+        return x, F32
+    if x.dtype == np.float64:
+        return x, F64
+    raise TypeError(f"unsupported oracle input dtype {x.dtype}")
+
+
+def _i32(x):
+    if hasattr(x, "detach"):
+        x = x.detach().cpu().numpy()
+    return np.ascontiguousarray(np.asarray(x, dtype=np.int32))
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _gdr_args(q, k, v, log_decay, beta, state_pool, state_slot, accept_len):
+    qa, qdt = _arr(q)
+    ka, kdt = _arr(k)
+    va, vdt = _arr(v)
+    if q is not None and qdt != kdt:
+        raise TypeError("q and k must share an element type")
+    if kdt != vdt:
+        raise TypeError("k and v must share an element type")
+    ga, gdt = _arr(log_decay)
+    ba, bdt = _arr(beta)
+    if gdt != bdt:
+        raise TypeError("log_decay and beta must share an element type")
+    sa, sdt = _arr(state_pool)
+    slot = _i32(state_slot)
+    acc = None if accept_len is None else _i32(accept_len)
+    R, B, Hk, dk = ka.shape
+    Hv, dv = va.shape[2], va.shape[3]
+    return dict(qa=qa, ka=ka, va=va, ga=ga, ba=ba, sa=sa, slot=slot, acc=acc, dt=kdt, gdt=gdt,
+                sdt=sdt, R=R, B=B, Hk=Hk, Hv=Hv, dk=dk, dv=dv, nslots=sa.shape[0])
+
+
+def gdr_per_token(q, k, v, log_decay, beta, state_pool, state_slot, accept_len=None, *,
+                  scale=None, blockend=True, causal=False, state=True, nthreads=0):
+    """Gated delta rule over one block, token by token (Eq. per-step-fwd).
+
+    Shapes: q, k [R,B,Hk,dk]; v [R,B,Hv,dv]; log_decay, beta [R,B,Hv];
+    state_pool [slots,Hv,dk,dv]; state_slot [R]; accept_len [R] or None (= B).
+    Returns a dict with fp64 arrays ``blockend`` [R,B,Hv,dv] (s S_B^T q_l),
+    ``causal`` [R,B,Hv,dv] (s S_t^T q_t) and ``state`` [R,Hv,dk,dv]
+    (S at the accepted length), each present when asked for.
+    """
+    a = _gdr_args(q, k, v, log_decay, beta, state_pool, state_slot, accept_len)
+    R, B, Hv, dk, dv = a["R"], a["B"], a["Hv"], a["dk"], a["dv"]
+    s = 1.0 / np.sqrt(dk) if scale is None else float(scale)
+    ob = np.zeros((R, B, Hv, dv)) if blockend else None
+    oc = np.zeros((R, B, Hv, dv)) if causal else None
+    st = np.zeros((R, Hv, dk, dv)) if state else None
+    if (blockend or causal) and q is None:
+        raise ValueError("q is required for a readout")
+    rc = _load().oracle_gdr_per_token(
+        R, B, a["Hk"], Hv, dk, dv, s, a["dt"], _ptr(a["qa"]), _ptr(a["ka"]), _ptr(a["va"]),
+        a["gdt"], _ptr(a["ga"]), _ptr(a["ba"]), a["sdt"], _ptr(a["sa"]), a["nslots"],
+        _ptr(a["slot"]), _ptr(a["acc"]), _ptr(ob), _ptr(oc), _ptr(st), int(nthreads))
+    if rc != 0:
+        raise ValueError("oracle_gdr_per_token: invalid state slot or accepted length")
+    return {k_: v_ for k_, v_ in (("blockend", ob), ("causal", oc), ("state", st)) if v_ is not None}
+
+
+def gdr_chunked(q, k, v, log_decay, beta, state_pool, state_slot, accept_len=None, *,
+                scale=None, nthreads=0):
+    """Chunkwise WY/UT form of the same block (Eq. chunk-state, Eq. f-blk).
+
+    Returns ``blockend`` and ``state`` like :func:`gdr_per_token`."""
+    a = _gdr_args(q, k, v, log_decay, beta, state_pool, state_slot, accept_len)
+    R, B, Hv, dk, dv = a["R"], a["B"], a["Hv"], a["dk"], a["dv"]
+    s = 1.0 / np.sqrt(dk) if scale is None else float(scale)
+    ob = np.zeros((R, B, Hv, dv))
+    st = np.zeros((R, Hv, dk, dv))
+    rc = _load().oracle_gdr_chunked(
+        R, B, a["Hk"], Hv, dk, dv, s, a["dt"], _ptr(a["qa"]), _ptr(a["ka"]), _ptr(a["va"]),
+        a["gdt"], _ptr(a["ga"]), _ptr(a["ba"]), a["sdt"], _ptr(a["sa"]), a["nslots"],
+        _ptr(a["slot"]), _ptr(a["acc"]), _ptr(ob), _ptr(st), int(nthreads))
+    if rc != 0:
+        raise ValueError("oracle_gdr_chunked: invalid state slot or accepted length")
+    return {"blockend": ob, "state": st}
+
+
+def gather_prefix(r, pool, page_table, prefix_len, page_size):
+    """Dense fp64 copy [P_r, Hkv, D] of request r's paged prefix from one pool."""
+    pa, pdt = _arr(pool)
+    tab = _i32(page_table)
+    lens = _i32(prefix_len)
+    num_pages, Hkv, p, D = pa.shape
+    assert p == page_size
+    out = np.zeros((int(lens[r]), Hkv, D))
+    rc = _load().oracle_gather_prefix(int(r), Hkv, D, page_size, num_pages, tab.shape[1], pdt,
+                                      _ptr(pa), _ptr(tab), _ptr(lens), _ptr(out))
+    if rc != 0:
+        raise ValueError("oracle_gather_prefix: invalid page id or prefix length")
+    return out
+
+
+def block_softmax(q, k_blk, v_blk, k_pool, v_pool, page_table, prefix_len, *, scale=None,
+                  mask_mode=0, nthreads=0):
+    """Block-query softmax attention over paged prefix + block (Eq. softmax-retrieval).
+
+    mask_mode 0: every block row sees every block token (denoise pass);
+    mask_mode 1: block row t sees block tokens 0..t (state-update pass).
+    Returns (out [R,B,Hq,D], lse [R,B,Hq]) in fp64."""
+    qa, dt = _arr(q)
+    kb, _ = _arr(k_blk)
+    vb, _ = _arr(v_blk)
+    kp, _ = _arr(k_pool)
+    vp, _ = _arr(v_pool)
+    tab = _i32(page_table)
+    lens = _i32(prefix_len)
+    R, B, Hq, D = qa.shape
+    Hkv = kb.shape[2]
+    num_pages, _, p, _ = kp.shape
+    sc = 1.0 / np.sqrt(D) if scale is None else float(scale)
+    out = np.zeros((R, B, Hq, D))
+    lse = np.zeros((R, B, Hq))
+    rc = _load().oracle_block_softmax(
+        R, B, Hq, Hkv, D, p, num_pages, tab.shape[1], sc, int(mask_mode), dt, _ptr(qa), _ptr(kb),
+        _ptr(vb), _ptr(kp), _ptr(vp), _ptr(tab), _ptr(lens), _ptr(out), _ptr(lse), int(nthreads))
+    if rc != 0:
+        raise ValueError("oracle_block_softmax: invalid page id or prefix length")
+    return out, lse

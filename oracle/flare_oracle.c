@@ -1,0 +1,363 @@
+/*
+ * FLARE block-denoising attention step: plain fp64 CPU oracle.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Nothing on the product path may call, link or
+ * load this file; only the tests, the smoke check and the CPU-baseline leg of
+ * the benchmark do.  It shares no code, header, constant or helper with the
+ * CUDA library: the two meet only through the seeded inputs.
+ *
+ * Every routine is the paper's definition written out, slowly and in double
+ * precision, in the paper's order and notation:
+ *
+ *   gated delta rule, per step (Appendix "Single-stream chunkwise training",
+ *   Eq. per-step-fwd):
+ *       S_pre_t = exp(g_t) S_{t-1}
+ *       u_t     = v_t - S_pre_t^T k_t
+ *       delta_t = beta_t u_t
+ *       S_t     = S_pre_t + k_t delta_t^T
+ *       o_t     = s S_t^T q_t                       (token-causal readout)
+ *   noisy block forward (Eq. noisy-block-fwd): the block starts from the
+ *   committed state and every block position reads the block-end state,
+ *       o~_l = s S_B^T q~_l   for all l in the block.
+ *   commit at accepted length r (serving appendix, "Recovering the recurrent
+ *   state at the accept boundary"): the pool slot becomes S^(r) = S_r, and
+ *   r = 0 leaves it unchanged.
+ *   chunkwise form (Eq. chunk-state / Eq. f-blk with WY-corrected values):
+ *   an independent second implementation used only to pin the first.
+ *   softmax retrieval over a visible set (Eq. softmax-retrieval) with the
+ *   Diffusion-Trust block mask: every block row sees the whole paged prefix
+ *   and (bidirectional mode) every block token, or (token-causal mode) the
+ *   block tokens up to and including itself.
+ *
+ * Element types of the inputs: 0 = bf16 (raw 16-bit patterns), 1 = fp32,
+ * 2 = fp64.  Converting a bf16 or fp32 value to double is exact, so the
+ * oracle computes on exactly the values the GPU sees.
+ */
+#include <math.h>
+#include <stddef.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+enum { ORC_BF16 = 0, ORC_F32 = 1, ORC_F64 = 2 };
+
+static double ld(const void* p, int dt, size_t i) {
+  if (dt == ORC_F64) return ((const double*)p)[i];
+  if (dt == ORC_F32) return (double)((const float*)p)[i];
+  uint32_t bits = ((uint32_t)((const uint16_t*)p)[i]) << 16;
+  float f;
+  memcpy(&f, &bits, sizeof f);
+  return (double)f;
+}
+
+static void set_threads(int nthreads) {
+#ifdef _OPENMP
+  if (nthreads > 0) omp_set_num_threads(nthreads);
+#else
+  (void)nthreads;
+#endif
+}
+
+int oracle_max_threads(void) {
+#ifdef _OPENMP
+  return omp_get_max_threads();
+#else
+  return 1;
+#endif
+}
+
+/*
+ * Gated delta rule over one block for every (request r, value head j),
+ * following Eq. per-step-fwd token by token.
+ *
+ * Shapes (row-major):
+ *   q, k        [R, B, Hk, dk]       (q may be NULL when no readout is asked)
+ *   v           [R, B, Hv, dv]
+ *   log_decay   [R, B, Hv]   g_t, the log-gate; alpha_t = exp(g_t)
+ *   beta        [R, B, Hv]
+ *   state_pool  [num_slots, Hv, dk, dv], S[i][j] at i*dv + j, so o = S^T q
+ *   state_slot  [R]          pool slot holding request r's committed state
+ *   accept_len  [R] or NULL  length r at which to take the committed state
+ *                            (NULL means the full block, r = B)
+ * Outputs (each may be NULL):
+ *   out_blockend [R, B, Hv, dv]  o~_l = s S_B^T q_l   (Eq. noisy-block-fwd)
+ *   out_causal   [R, B, Hv, dv]  o_t  = s S_t^T q_t   (Eq. per-step-fwd)
+ *   state_out    [R, Hv, dk, dv] S_{accept_len[r]}
+ * Value head j reads q/k head floor(j * Hk / Hv).
+ * Returns 0, or -1 for an invalid slot or accepted length.
+ */
+int oracle_gdr_per_token(int R, int B, int Hk, int Hv, int dk, int dv, double s,
+                         int act_dt, const void* q, const void* k, const void* v,
+                         int gate_dt, const void* log_decay, const void* beta,
+                         int state_dt, const void* state_pool, int num_slots,
+                         const int32_t* state_slot, const int32_t* accept_len,
+                         double* out_blockend, double* out_causal, double* state_out,
+                         int nthreads) {
+  for (int r = 0; r < R; ++r) {
+    if (state_slot[r] < 0 || state_slot[r] >= num_slots) return -1;
+    if (accept_len && (accept_len[r] < 0 || accept_len[r] > B)) return -1;
+  }
+  set_threads(nthreads);
+#pragma omp parallel for schedule(dynamic, 1)
+  for (long item = 0; item < (long)R * Hv; ++item) {
+    const int r = (int)(item / Hv), j = (int)(item % Hv);
+    const int h = (int)(((long)j * Hk) / Hv);
+    const int r_acc = accept_len ? accept_len[r] : B;
+    double* S = (double*)malloc(sizeof(double) * dk * dv);
+    double* u = (double*)malloc(sizeof(double) * dv);
+    const size_t s0 = ((size_t)state_slot[r] * Hv + j) * dk * dv;
+    for (int e = 0; e < dk * dv; ++e) S[e] = ld(state_pool, state_dt, s0 + e);
+    if (state_out && r_acc == 0)
+      for (int e = 0; e < dk * dv; ++e) state_out[(size_t)item * dk * dv + e] = S[e];
+    for (int t = 0; t < B; ++t) {
+      const size_t kq = (((size_t)r * B + t) * Hk + h) * dk;
+      const size_t vo = (((size_t)r * B + t) * Hv + j) * dv;
+      const size_t gb = ((size_t)r * B + t) * Hv + j;
+      const double alpha = exp(ld(log_decay, gate_dt, gb));
+      const double bt = ld(beta, gate_dt, gb);
+      /* gating decay: S_pre = exp(g_t) S_{t-1} */
+      for (int e = 0; e < dk * dv; ++e) S[e] *= alpha;
+      /* prediction error u_t = v_t - S_pre^T k_t, delta update delta_t = beta_t u_t */
+      for (int c = 0; c < dv; ++c) {
+        double acc = 0.0;
+        for (int i = 0; i < dk; ++i) acc += S[i * dv + c] * ld(k, act_dt, kq + i);
+        u[c] = bt * (ld(v, act_dt, vo + c) - acc);
+      }
+      /* outer-product write S_t = S_pre + k_t delta_t^T */
+      for (int i = 0; i < dk; ++i) {
+        const double ki = ld(k, act_dt, kq + i);
+        for (int c = 0; c < dv; ++c) S[i * dv + c] += ki * u[c];
+      }
+      /* token-causal output o_t = s S_t^T q_t */
+      if (out_causal)
+        for (int c = 0; c < dv; ++c) {
+          double acc = 0.0;
+          for (int i = 0; i < dk; ++i) acc += S[i * dv + c] * ld(q, act_dt, kq + i);
+          out_causal[vo + c] = s * acc;
+        }
+      if (state_out && t + 1 == r_acc)
+        for (int e = 0; e < dk * dv; ++e) state_out[(size_t)item * dk * dv + e] = S[e];
+    }
+    /* block-end readout: every block row reads S_B (Eq. noisy-block-fwd) */
+    if (out_blockend)
+      for (int l = 0; l < B; ++l) {
+        const size_t ql = (((size_t)r * B + l) * Hk + h) * dk;
+        const size_t ol = (((size_t)r * B + l) * Hv + j) * dv;
+        for (int c = 0; c < dv; ++c) {
+          double acc = 0.0;
+          for (int i = 0; i < dk; ++i) acc += S[i * dv + c] * ld(q, act_dt, ql + i);
+          out_blockend[ol + c] = s * acc;
+        }
+      }
+    free(u);
+    free(S);
+  }
+  return 0;
+}
+
+/*
+ * The same quantities computed a second, independent way: the chunkwise
+ * (WY / UT) form of the appendix, "Chunkwise-parallel form",
+ * "Chunk-corrected values" and Eq. chunk-state, applied to one block.
+ *
+ *   gamma_t = sum_{i<=t} g_i                          (cumulative log-gate G_t)
+ *   A[t][i] = beta_t exp(gamma_t - gamma_i) (k_t . k_i)        for i < t
+ *   (I + A) delta = diag(beta) (V - diag(exp(gamma)) K S0)     (forward substitution)
+ *   S_r = exp(gamma_r) S0 + sum_{i<=r} exp(gamma_r - gamma_i) k_i delta_i^T
+ *   o~_l = s (exp(gamma_B) S0^T q_l + sum_{i<=B} exp(gamma_B - gamma_i) (q_l . k_i) delta_i)
+ *
+ * delta here is the per-step delta update (the WY-corrected value scaled by
+ * beta); Eq. chunk-state with r = B is Eq. f-blk.  Same arguments and outputs
+ * as oracle_gdr_per_token except that token-causal outputs are not formed.
+ */
+int oracle_gdr_chunked(int R, int B, int Hk, int Hv, int dk, int dv, double s,
+                       int act_dt, const void* q, const void* k, const void* v,
+                       int gate_dt, const void* log_decay, const void* beta,
+                       int state_dt, const void* state_pool, int num_slots,
+                       const int32_t* state_slot, const int32_t* accept_len,
+                       double* out_blockend, double* state_out, int nthreads) {
+  for (int r = 0; r < R; ++r) {
+    if (state_slot[r] < 0 || state_slot[r] >= num_slots) return -1;
+    if (accept_len && (accept_len[r] < 0 || accept_len[r] > B)) return -1;
+  }
+  set_threads(nthreads);
+#pragma omp parallel for schedule(dynamic, 1)
+  for (long item = 0; item < (long)R * Hv; ++item) {
+    const int r = (int)(item / Hv), j = (int)(item % Hv);
+    const int h = (int)(((long)j * Hk) / Hv);
+    const int r_acc = accept_len ? accept_len[r] : B;
+    double* S0 = (double*)malloc(sizeof(double) * dk * dv);
+    double* gam = (double*)malloc(sizeof(double) * (B + 1));
+    double* A = (double*)calloc((size_t)B * B, sizeof(double));
+    double* delta = (double*)malloc(sizeof(double) * B * dv);
+    const size_t s0 = ((size_t)state_slot[r] * Hv + j) * dk * dv;
+    for (int e = 0; e < dk * dv; ++e) S0[e] = ld(state_pool, state_dt, s0 + e);
+#define KEL(t, i) ld(k, act_dt, (((size_t)r * B + (t)) * Hk + h) * dk + (i))
+#define QEL(t, i) ld(q, act_dt, (((size_t)r * B + (t)) * Hk + h) * dk + (i))
+#define VEL(t, c) ld(v, act_dt, (((size_t)r * B + (t)) * Hv + j) * dv + (c))
+#define GB(t) (((size_t)r * B + (t)) * Hv + j)
+    /* gam[t+1] = gamma after token t (1-based cumulative), gam[0] = 0 */
+    gam[0] = 0.0;
+    for (int t = 0; t < B; ++t) gam[t + 1] = gam[t] + ld(log_decay, gate_dt, GB(t));
+    for (int t = 0; t < B; ++t)
+      for (int i = 0; i < t; ++i) {
+        double kk = 0.0;
+        for (int e = 0; e < dk; ++e) kk += KEL(t, e) * KEL(i, e);
+        A[t * B + i] = ld(beta, gate_dt, GB(t)) * exp(gam[t + 1] - gam[i + 1]) * kk;
+      }
+    /* right-hand side, then forward substitution through the unit lower-triangular I + A */
+    for (int t = 0; t < B; ++t) {
+      const double bt = ld(beta, gate_dt, GB(t));
+      const double G = exp(gam[t + 1]);
+      for (int c = 0; c < dv; ++c) {
+        double ks = 0.0;
+        for (int i = 0; i < dk; ++i) ks += KEL(t, i) * S0[i * dv + c];
+        double x = bt * (VEL(t, c) - G * ks);
+        for (int i = 0; i < t; ++i) x -= A[t * B + i] * delta[i * dv + c];
+        delta[t * dv + c] = x;
+      }
+    }
+    if (state_out) {
+      double* So = state_out + (size_t)item * dk * dv;
+      const double Gr = exp(gam[r_acc]);
+      for (int i = 0; i < dk; ++i)
+        for (int c = 0; c < dv; ++c) {
+          double acc = Gr * S0[i * dv + c];
+          for (int t = 0; t < r_acc; ++t)
+            acc += exp(gam[r_acc] - gam[t + 1]) * KEL(t, i) * delta[t * dv + c];
+          So[i * dv + c] = acc;
+        }
+    }
+    if (out_blockend) {
+      const double GB_ = exp(gam[B]);
+      for (int l = 0; l < B; ++l)
+        for (int c = 0; c < dv; ++c) {
+          double acc = 0.0;
+          for (int i = 0; i < dk; ++i) acc += QEL(l, i) * S0[i * dv + c];
+          acc *= GB_;
+          for (int t = 0; t < B; ++t) {
+            double qk = 0.0;
+            for (int e = 0; e < dk; ++e) qk += QEL(l, e) * KEL(t, e);
+            acc += exp(gam[B] - gam[t + 1]) * qk * delta[t * dv + c];
+          }
+          out_blockend[(((size_t)r * B + l) * Hv + j) * dv + c] = s * acc;
+        }
+    }
+#undef KEL
+#undef QEL
+#undef VEL
+#undef GB
+    free(delta);
+    free(A);
+    free(gam);
+    free(S0);
+  }
+  return 0;
+}
+
+/*
+ * Dense copy of request r's paged prefix for one pool (K or V):
+ * token j < prefix_len[r] lives in page page_table[r * max_pages + j / page_size],
+ * row j % page_size, of the pool laid out [num_pages, Hkv, page_size, D].
+ * out is [prefix_len[r], Hkv, D] in fp64.  Returns -1 on an invalid page id or
+ * a prefix longer than max_pages * page_size.
+ */
+int oracle_gather_prefix(int r, int Hkv, int D, int page_size, int num_pages, int max_pages,
+                         int act_dt, const void* pool, const int32_t* page_table,
+                         const int32_t* prefix_len, double* out) {
+  const int P = prefix_len[r];
+  if (P < 0 || P > max_pages * page_size) return -1;
+  for (int jt = 0; jt < P; ++jt) {
+    const int page = page_table[(size_t)r * max_pages + jt / page_size];
+    if (page < 0 || page >= num_pages) return -1;
+    for (int hk = 0; hk < Hkv; ++hk)
+      for (int d = 0; d < D; ++d)
+        out[((size_t)jt * Hkv + hk) * D + d] =
+            ld(pool, act_dt, (((size_t)page * Hkv + hk) * page_size + jt % page_size) * D + d);
+  }
+  return 0;
+}
+
+/*
+ * Block-query softmax attention (Eq. softmax-retrieval) with the
+ * Diffusion-Trust block mask.  For request r, query head h (kv head
+ * h / (Hq / Hkv)) and block row t the visible set is every prefix token
+ * j < prefix_len[r] (read through the page table) plus the block tokens i
+ * with i < B (mask_mode 0, bidirectional denoise pass) or i <= t
+ * (mask_mode 1, token-causal state-update pass).  Two passes in fp64:
+ *   z_i = scale (q . k_i),  m = max_i z_i,  w_i = exp(z_i - m),
+ *   o = sum_i w_i v_i / sum_i w_i,  lse = m + log(sum_i w_i).
+ * Shapes: q [R,B,Hq,D]; k_blk, v_blk [R,B,Hkv,D]; pools
+ * [num_pages,Hkv,page_size,D]; page_table [R,max_pages]; prefix_len [R];
+ * out [R,B,Hq,D]; lse [R,B,Hq] (may be NULL).
+ */
+int oracle_block_softmax(int R, int B, int Hq, int Hkv, int D, int page_size, int num_pages,
+                         int max_pages, double scale, int mask_mode, int act_dt,
+                         const void* q, const void* k_blk, const void* v_blk,
+                         const void* k_pool, const void* v_pool,
+                         const int32_t* page_table, const int32_t* prefix_len,
+                         double* out, double* lse, int nthreads) {
+  if (Hkv <= 0 || Hq % Hkv != 0) return -1;
+  for (int r = 0; r < R; ++r) {
+    const int P = prefix_len[r];
+    if (P < 0 || P > max_pages * page_size) return -1;
+    for (int pg = 0; pg < (P + page_size - 1) / page_size; ++pg) {
+      const int page = page_table[(size_t)r * max_pages + pg];
+      if (page < 0 || page >= num_pages) return -1;
+    }
+  }
+  const int G = Hq / Hkv;
+  set_threads(nthreads);
+#pragma omp parallel for schedule(dynamic, 1)
+  for (long item = 0; item < (long)R * Hq * B; ++item) {
+    const int r = (int)(item / ((long)Hq * B));
+    const int h = (int)((item / B) % Hq);
+    const int t = (int)(item % B);
+    const int kvh = h / G;
+    const int P = prefix_len[r];
+    const int nblk = (mask_mode == 0) ? B : t + 1;
+    const int n = P + nblk;
+    double* z = (double*)malloc(sizeof(double) * (n > 0 ? n : 1));
+    const size_t qo = (((size_t)r * B + t) * Hq + h) * D;
+    /* visible keys: prefix first, then the block */
+    for (int jt = 0; jt < n; ++jt) {
+      double acc = 0.0;
+      if (jt < P) {
+        const int page = page_table[(size_t)r * max_pages + jt / page_size];
+        const size_t ko = (((size_t)page * Hkv + kvh) * page_size + jt % page_size) * D;
+        for (int d = 0; d < D; ++d) acc += ld(q, act_dt, qo + d) * ld(k_pool, act_dt, ko + d);
+      } else {
+        const size_t ko = (((size_t)r * B + (jt - P)) * Hkv + kvh) * D;
+        for (int d = 0; d < D; ++d) acc += ld(q, act_dt, qo + d) * ld(k_blk, act_dt, ko + d);
+      }
+      z[jt] = scale * acc;
+    }
+    double m = -INFINITY;
+    for (int jt = 0; jt < n; ++jt) m = z[jt] > m ? z[jt] : m;
+    double Z = 0.0;
+    for (int jt = 0; jt < n; ++jt) {
+      z[jt] = exp(z[jt] - m);
+      Z += z[jt];
+    }
+    for (int d = 0; d < D; ++d) {
+      double acc = 0.0;
+      for (int jt = 0; jt < n; ++jt) {
+        double vv;
+        if (jt < P) {
+          const int page = page_table[(size_t)r * max_pages + jt / page_size];
+          vv = ld(v_pool, act_dt, (((size_t)page * Hkv + kvh) * page_size + jt % page_size) * D + d);
+        } else {
+          vv = ld(v_blk, act_dt, (((size_t)r * B + (jt - P)) * Hkv + kvh) * D + d);
+        }
+        acc += z[jt] * vv;
+      }
+      out[qo + d] = acc / Z;
+    }
+    if (lse) lse[((size_t)r * B + t) * Hq + h] = m + log(Z);
+    free(z);
+  }
+  return 0;
+}
