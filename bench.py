@@ -1,0 +1,516 @@
+#!/usr/bin/env python3
+"""Benchmark of the FLARE block-denoising attention step on GB300.
+
+One step = one pass of the whole hot path over one batch: for each of the
+workload's denoise steps, one gated-delta-rule layer call
+(flare_block_linear_attn) and one softmax layer call (flare_block_softmax_attn)
+over fresh block inputs, then one commit of every request's state at its
+accepted length (flare_commit_state).  Metric: block-tokens/s =
+requests x block_len x denoise_steps / step time.
+
+Default workload: multistep_batch128 (128 requests, GDN 16 qk / 32 v heads,
+d=128, softmax 16 q / 2 kv heads, D=256, block 64, 8 denoise steps over paged
+prefixes ~U[1024,16384], commit at accepted lengths ~U[1,64]).  Each step
+streams ~2.7 GB of KV and state (> 129 MB L2), so no L2 flush is needed.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+                  [--impl flare|reference]
+
+Under torchrun (N > 1) every rank runs its own batch (requests are
+independent: weak scaling, no collective on the data path); the timed region
+is bracketed by barriers and the max over ranks is reported.
+``--impl reference`` times the fp64 CPU oracle on a bounded sample of the same
+workload on the host cores (rank 0 only).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import shutil
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2606_01774_gb300 import workloads  # noqa: E402
+
+METRIC = "denoise-step attention block-tokens/s"
+UNIT = "block-tokens/s"
+DEFAULT_WORKLOAD = "multistep_batch128"
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            pk = json.load(f)
+        return {"hbm_gbs": pk["hbm_gbs"], "bf16_tflops": pk["bf16_tflops"],
+                "bf16_tflops_sustained": pk.get("bf16_tflops_sustained", pk["bf16_tflops"]),
+                "source": "measured"}
+    except (OSError, KeyError, ValueError):
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                "source": "fallback"}
+
+
+# ---------------------------------------------------------------- algorithmic counts
+
+
+def linear_bytes(spec):
+    R, B, Hk, Hv, dk, dv = (spec.num_requests, spec.block_len, spec.num_qk_heads,
+                            spec.num_v_heads, spec.head_dim_k, spec.head_dim_v)
+    e = 2 if spec.act_dtype == "bf16" else 4
+    return (R * Hv * dk * dv * 4 + 2 * R * B * Hk * dk * e + R * B * Hv * dv * e
+            + 2 * R * B * Hv * 4 + R * B * Hv * dv * e)
+
+
+def linear_flops(spec):
+    B, dk, dv = spec.block_len, spec.head_dim_k, spec.head_dim_v
+    per_head = 4 * B * B * dk + 4 * B * dk * dv + 2 * B * B * dv + (2 / 3) * B ** 3
+    return spec.num_requests * spec.num_v_heads * per_head
+
+
+def softmax_bytes(spec, prefix_sum):
+    R, B, Hq, Hkv, D = (spec.num_requests, spec.block_len, spec.num_q_heads, spec.num_kv_heads,
+                        spec.head_dim)
+    e = 2 if spec.act_dtype == "bf16" else 4
+    return (2 * prefix_sum * Hkv * D * e + R * B * Hq * D * e + 2 * R * B * Hkv * D * e
+            + R * B * Hq * D * e)
+
+
+def softmax_flops(spec, prefix_sum):
+    return 4.0 * spec.block_len * spec.num_q_heads * spec.head_dim * (
+        prefix_sum + spec.num_requests * spec.block_len)
+
+
+def commit_bytes(spec, accept):
+    n = int((accept > 0).sum())
+    B, Hk, Hv, dk, dv = (spec.block_len, spec.num_qk_heads, spec.num_v_heads, spec.head_dim_k,
+                         spec.head_dim_v)
+    e = 2 if spec.act_dtype == "bf16" else 4
+    R = spec.num_requests
+    return (2 * n * Hv * dk * dv * 4 + R * B * Hk * dk * e + R * B * Hv * dv * e
+            + 2 * R * B * Hv * 4)
+
+
+# ---------------------------------------------------------------- clocks
+
+
+class ClockSampler:
+    """nvidia-smi samples every 200 ms while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index):
+        self.proc = None
+        self.path = None
+        exe = shutil.which("nvidia-smi")
+        if exe is None:
+            return
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        self.out = open(self.path, "w")
+        self.proc = subprocess.Popen(
+            [exe, f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200",
+             "-i", str(device_index)], stdout=self.out, stderr=subprocess.DEVNULL)
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.out.close()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if "Active" in r[5 + i]
+                          and "Not" not in r[5 + i]})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(rows)}
+
+
+# ---------------------------------------------------------------- GPU arm
+
+
+class FlareRunner:
+    """Holds one workload on the device and issues the step's C-ABI calls."""
+
+    def __init__(self, spec, device, seed_offset=0):
+        from paper_2606_01774_gb300 import flare
+
+        self.flare = flare
+        self.spec = spec.replace(seed=spec.seed + seed_offset)
+        self.device = device
+        self.w = workloads.generate(self.spec, device)
+        s = self.spec
+        self.act = flare.FLARE_DT_BF16 if s.act_dtype == "bf16" else flare.FLARE_DT_F32
+        nslots = self.w.state_pool.shape[0]
+        self.ldesc = flare.linear_desc(s.num_requests, s.block_len, s.num_qk_heads,
+                                       s.num_v_heads, s.head_dim_k, s.head_dim_v, nslots,
+                                       self.act, 1.0 / math.sqrt(s.head_dim_k))
+        self.sdesc = flare.softmax_desc(s.num_requests, s.block_len, s.num_q_heads,
+                                        s.num_kv_heads, s.head_dim, s.page_size,
+                                        self.w.k_pool.shape[0], self.w.page_table.shape[1],
+                                        self.act, 1.0 / math.sqrt(s.head_dim))
+        self.ws_bytes = flare.flare_softmax_workspace_size(self.sdesc)
+        self.ws = torch.empty(max(self.ws_bytes, 256), dtype=torch.uint8, device=device)
+        self.status = torch.zeros(1, dtype=torch.int32, device=device)
+        self.lin_out = [torch.empty_like(b.v) for b in self.w.denoise]
+        self.sm_out = [torch.empty_like(b.q) for b in self.w.softmax]
+        self.prefill_states()
+
+    def prefill_states(self):
+        """Committed state S0 of every request: the gated delta rule over its
+        random prefix tokens from the zero state, run through the library's own
+        commit in blocks of up to 64 tokens (what a serving prefill does)."""
+        fl, s, w = self.flare, self.spec, self.w
+        w.state_pool.zero_()
+        sp = w.state_prefix
+        n = sp.k.shape[1]
+        for lo in range(0, n, 64):
+            hi = min(lo + 64, n)
+            d = fl.linear_desc(s.num_requests, hi - lo, s.num_qk_heads, s.num_v_heads,
+                               s.head_dim_k, s.head_dim_v, w.state_pool.shape[0], self.act,
+                               1.0 / math.sqrt(s.head_dim_k))
+            acc = torch.full((s.num_requests,), hi - lo, dtype=torch.int32, device=self.device)
+            fl.check(fl.flare_commit_state(
+                d, None, sp.k[:, lo:hi].contiguous(), sp.v[:, lo:hi].contiguous(),
+                sp.log_decay[:, lo:hi].contiguous(), sp.beta[:, lo:hi].contiguous(),
+                w.state_pool, w.state_slot, acc, None, self.status), "prefill")
+        torch.cuda.synchronize()
+
+    def linear(self, i, ev=None):
+        fl, w, b = self.flare, self.w, self.w.denoise[i]
+        rc = fl.flare_block_linear_attn(self.ldesc, b.q, b.k, b.v, b.log_decay, b.beta,
+                                        w.state_pool, w.state_slot, self.lin_out[i], self.status)
+        if rc:
+            fl.check(rc, "flare_block_linear_attn")
+
+    def softmax(self, i):
+        fl, w, b = self.flare, self.w, self.w.softmax[i]
+        rc = fl.flare_block_softmax_attn(self.sdesc, b.q, b.k_blk, b.v_blk, w.k_pool, w.v_pool,
+                                         w.page_table, w.prefix_len, self.sm_out[i], None,
+                                         self.ws, self.ws_bytes, self.status)
+        if rc:
+            fl.check(rc, "flare_block_softmax_attn")
+
+    def commit(self):
+        fl, w, b = self.flare, self.w, self.w.commit
+        rc = fl.flare_commit_state(self.ldesc, None, b.k, b.v, b.log_decay, b.beta,
+                                   w.state_pool, w.state_slot, w.accept_len, None, self.status)
+        if rc:
+            fl.check(rc, "flare_commit_state")
+
+    def step(self, events=None):
+        """One pass of the hot path; events (if given) bracket each call."""
+        for i in range(self.spec.denoise_steps):
+            if events is not None:
+                events["linear"].append(torch.cuda.Event(enable_timing=True))
+                events["linear"][-1].record()
+            self.linear(i)
+            if events is not None:
+                events["linear"].append(torch.cuda.Event(enable_timing=True))
+                events["linear"][-1].record()
+                events["softmax"].append(torch.cuda.Event(enable_timing=True))
+                events["softmax"][-1].record()
+            self.softmax(i)
+            if events is not None:
+                events["softmax"].append(torch.cuda.Event(enable_timing=True))
+                events["softmax"][-1].record()
+        if events is not None:
+            events["commit"].append(torch.cuda.Event(enable_timing=True))
+            events["commit"][-1].record()
+        self.commit()
+        if events is not None:
+            events["commit"].append(torch.cuda.Event(enable_timing=True))
+            events["commit"][-1].record()
+
+
+class E2ERunner:
+    """The same step through the C ABI with the step's inputs in pinned host
+    memory: host->device copies of every per-step input and device->host
+    copies of every output happen inside the timed region.  The paged KV pool
+    and the recurrent-state pool are the serving caches and stay resident."""
+
+    def __init__(self, fr: FlareRunner):
+        self.fr = fr
+        w = fr.w
+        self.h2d = []  # (pinned host, device) pairs
+        self.d2h = []
+        for b in w.denoise:
+            for t in (b.q, b.k, b.v, b.log_decay, b.beta):
+                self.h2d.append((t.cpu().pin_memory(), t))
+        for t in (w.commit.k, w.commit.v, w.commit.log_decay, w.commit.beta):
+            self.h2d.append((t.cpu().pin_memory(), t))
+        for b in w.softmax:
+            for t in (b.q, b.k_blk, b.v_blk):
+                self.h2d.append((t.cpu().pin_memory(), t))
+        for t in (w.page_table, w.prefix_len, w.accept_len, w.state_slot):
+            self.h2d.append((t.cpu().pin_memory(), t))
+        for t in fr.lin_out + fr.sm_out:
+            self.d2h.append((t, torch.empty(t.shape, dtype=t.dtype, pin_memory=True)))
+        self.h2d_bytes = sum(h.numel() * h.element_size() for h, _ in self.h2d)
+        self.d2h_bytes = sum(h.numel() * h.element_size() for _, h in self.d2h)
+
+    def step(self):
+        for h, d in self.h2d:
+            d.copy_(h, non_blocking=True)
+        self.fr.step()
+        for d, h in self.d2h:
+            h.copy_(d, non_blocking=True)
+        torch.cuda.current_stream().synchronize()
+
+
+def _elapsed_pairs(evs):
+    return [evs[i].elapsed_time(evs[i + 1]) for i in range(0, len(evs), 2)]
+
+
+def run_flare(args, spec, rank, world, local_rank):
+    device = torch.device("cuda", local_rank)
+    torch.cuda.set_device(device)
+    from paper_2606_01774_gb300 import flare
+
+    flare.load()
+    fr = FlareRunner(spec, device, seed_offset=1000 * rank)
+    dist = world > 1
+    if dist:
+        import torch.distributed as tdist
+
+    for _ in range(args.warmup):
+        fr.step()
+    torch.cuda.synchronize()
+    st, bits = flare.flare_read_status(fr.status)
+    if st != flare.FLARE_OK:
+        raise RuntimeError(f"device status {bits:#x} after warm-up")
+
+    events = {"linear": [], "softmax": [], "commit": []}
+    clocks = ClockSampler(torch.cuda.current_device()) if rank == 0 else None
+    if dist:
+        tdist.barrier()
+    torch.cuda.synchronize()
+    launches0 = flare.flare_launch_count()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for _ in range(args.steps):
+        fr.step(events)
+    t1.record()
+    torch.cuda.synchronize()
+    launches = flare.flare_launch_count() - launches0
+    if dist:
+        tdist.barrier()
+    clk = clocks.stop() if clocks else None
+    ms = t0.elapsed_time(t1)
+    if dist:
+        tt = torch.tensor([ms], dtype=torch.float64, device=device)
+        tdist.all_reduce(tt, op=tdist.ReduceOp.MAX)
+        ms = float(tt.item())
+    ms_step = ms / args.steps
+
+    # end-to-end through host buffers
+    e2e = E2ERunner(fr)
+    for _ in range(max(1, min(args.warmup, 2))):
+        e2e.step()
+    if dist:
+        tdist.barrier()
+    t_e = time.perf_counter()
+    for _ in range(args.steps):
+        e2e.step()
+    e2e_ms = (time.perf_counter() - t_e) * 1e3 / args.steps
+    if dist:
+        tt = torch.tensor([e2e_ms], dtype=torch.float64, device=device)
+        tdist.all_reduce(tt, op=tdist.ReduceOp.MAX)
+        e2e_ms = float(tt.item())
+    st, bits = flare.flare_read_status(fr.status)
+    if st != flare.FLARE_OK:
+        raise RuntimeError(f"device status {bits:#x} after timing")
+
+    if rank != 0:
+        return None
+    s = fr.spec
+    tokens = s.num_requests * s.block_len * s.denoise_steps
+    value = world * tokens / (ms_step / 1e3)
+    per = {k: float(np.mean(_elapsed_pairs(v))) for k, v in events.items()}
+    prefix_sum = int(fr.w.prefix_len.sum().item())
+    acc = fr.w.accept_len.cpu().numpy()
+    peaks = load_peaks()
+    kern = {
+        "linear": dict(bytes=linear_bytes(s), flops=linear_flops(s), kernel="flare_block_linear_attn"),
+        "softmax": dict(bytes=softmax_bytes(s, prefix_sum), flops=softmax_flops(s, prefix_sum),
+                        kernel="flare_block_softmax_attn"),
+        "commit": dict(bytes=commit_bytes(s, acc), flops=0.0, kernel="flare_commit_state"),
+    }
+    share = {k: per[k] * (s.denoise_steps if k != "commit" else 1) for k in per}
+    dom = max(share, key=share.get)
+    kd = kern[dom]
+    dur_s = per[dom] / 1e3
+    t_hbm = kd["bytes"] / (peaks["hbm_gbs"] * 1e9)
+    t_tc = kd["flops"] / (peaks["bf16_tflops_sustained"] * 1e12)
+    if t_tc > t_hbm:
+        roof = {"bound": "tensor", "achieved": kd["flops"] / dur_s / 1e12,
+                "peak": peaks["bf16_tflops_sustained"], "unit": "TFLOP/s"}
+    else:
+        roof = {"bound": "hbm", "achieved": kd["bytes"] / dur_s / 1e9,
+                "peak": peaks["hbm_gbs"], "unit": "GB/s"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["traffic"] = None
+    roof["kernel"] = kd["kernel"]
+    roof["peak_source"] = f"{peaks['source']} ({'bf16_tflops_sustained' if roof['unit'] == 'TFLOP/s' else 'hbm_gbs'})"
+    roof["algorithmic_per_launch"] = kd["flops"] if roof["bound"] == "tensor" else kd["bytes"]
+    step_bytes = s.denoise_steps * (kern["linear"]["bytes"] + kern["softmax"]["bytes"]) + \
+        kern["commit"]["bytes"]
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": s.act_dtype, "data": "synthetic",
+        "config": {"workload": s.name, "requests": s.num_requests, "block_len": s.block_len,
+                   "denoise_steps": s.denoise_steps, "gdn_heads": [s.num_qk_heads, s.num_v_heads],
+                   "head_dim_k": s.head_dim_k, "softmax_heads": [s.num_q_heads, s.num_kv_heads],
+                   "head_dim": s.head_dim, "page_size": s.page_size,
+                   "prefix": [s.prefix_lo, s.prefix_hi], "parallelism": f"replicas{world}",
+                   "l2": f"no flush: each step streams {step_bytes / 1e9:.2f} GB > 129 MB L2"},
+        "achieved_hbm_gbs": step_bytes / (ms_step / 1e3) / 1e9,
+        "per_call_ms": per,
+        "roofline": roof,
+        "e2e": {"value": world * tokens / (e2e_ms / 1e3), "unit": UNIT, "ms_per_step": e2e_ms,
+                "h2d_bytes_per_step": e2e.h2d_bytes, "d2h_bytes_per_step": e2e.d2h_bytes},
+        "gpu_launches": int(launches),
+        "clocks": clk,
+    }
+    return line
+
+
+# ---------------------------------------------------------------- oracle (CPU) arm
+
+
+def oracle_sample_rate(spec, n_requests, seed_offset=0, one_head=False):
+    """Times the fp64 oracle on a bounded sample of the workload (drawn on the
+    host with the same recipe): the first n_requests, one denoise step (linear
+    + softmax) and the commit.  With one_head, only q head 0 (and its kv head)
+    and v head 0 (and its q/k head) are computed and the time is scaled by the
+    head counts, heads being independent.  Returns (block-tokens/s, seconds
+    per bench step, threads, sample description)."""
+    import oracle
+
+    oracle.build()
+    sub = spec.replace(num_requests=n_requests, denoise_steps=1, seed=spec.seed + seed_offset)
+    w = workloads.generate(sub, "cpu")
+    R, Hv, dk, dv = sub.num_requests, sub.num_v_heads, sub.head_dim_k, sub.head_dim_v
+    b, c, sb, sp = w.denoise[0], w.commit, w.softmax[0], w.state_prefix
+    hv = slice(0, 1) if one_head else slice(0, Hv)
+    hk = slice(0, 1) if one_head else slice(0, sub.num_qk_heads)
+    hq = slice(0, 1) if one_head else slice(0, sub.num_q_heads)
+    hkv = slice(0, 1) if one_head else slice(0, sub.num_kv_heads)
+    nv = hv.stop - hv.start
+    S0 = oracle.gdr_per_token(None, sp.k[:, :, hk], sp.v[:, :, hv], sp.log_decay[:, :, hv],
+                              sp.beta[:, :, hv], np.zeros((1, nv, dk, dv), np.float32),
+                              np.zeros(R, np.int32), None, blockend=False)["state"]
+    pool = S0.astype(np.float32)
+    slots = np.arange(R, dtype=np.int32)
+    kp, vp = w.k_pool[:, hkv], w.v_pool[:, hkv]
+    t0 = time.perf_counter()
+    oracle.gdr_per_token(b.q[:, :, hk], b.k[:, :, hk], b.v[:, :, hv], b.log_decay[:, :, hv],
+                         b.beta[:, :, hv], pool, slots, None, state=False)
+    t1 = time.perf_counter()
+    oracle.block_softmax(sb.q[:, :, hq], sb.k_blk[:, :, hkv], sb.v_blk[:, :, hkv], kp, vp,
+                         w.page_table, w.prefix_len, scale=1.0 / math.sqrt(sub.head_dim))
+    t2 = time.perf_counter()
+    oracle.gdr_per_token(None, c.k[:, :, hk], c.v[:, :, hv], c.log_decay[:, :, hv],
+                         c.beta[:, :, hv], pool, slots, w.accept_len, blockend=False)
+    t3 = time.perf_counter()
+    f_v = sub.num_v_heads if one_head else 1
+    f_q = sub.num_q_heads if one_head else 1
+    step_s = spec.denoise_steps * ((t1 - t0) * f_v + (t2 - t1) * f_q) + (t3 - t2) * f_v
+    tokens = R * spec.block_len * spec.denoise_steps
+    heads = ("q head 0 and v head 0 timed, scaled by the head counts "
+             f"({sub.num_q_heads} q, {sub.num_v_heads} v)" if one_head else "all heads")
+    desc = (f"{R} request(s) of {spec.name} drawn on the host with the same recipe "
+            f"(prefix {int(w.prefix_len.sum())} tokens), {heads}: one denoise step "
+            f"(linear + softmax) timed and counted {spec.denoise_steps}x, plus the commit")
+    return tokens / step_s, step_s, oracle.max_threads(), desc
+
+
+def run_reference(args, spec):
+    secs = []
+    threads, desc = None, None
+    for i in range(args.warmup + args.steps):
+        _, s, threads, desc = oracle_sample_rate(spec, 1, seed_offset=i, one_head=True)
+        if i >= args.warmup:
+            secs.append(s)
+    value = len(secs) * spec.block_len * spec.denoise_steps / sum(secs)
+    return {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * float(np.mean(secs)),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": spec.name, "requests_per_step": 1, "parallelism": "host cores"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
+                         "sample": "each step: " + desc},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(workloads.WORKLOADS))
+    ap.add_argument("--impl", default="flare", choices=["flare", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-sample-requests", type=int, default=2)
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "flare":
+        ap.error("--warmup must be >= 3")
+    spec = workloads.WORKLOADS[args.workload]
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        if rank != 0:
+            return 0
+        print(json.dumps(run_reference(args, spec)), flush=True)
+        return 0
+
+    if world > 1:
+        import torch.distributed as tdist
+
+        torch.cuda.set_device(local_rank)
+        tdist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    line = run_flare(args, spec, rank, world, local_rank)
+    if rank == 0:
+        if world == 1 and not args.no_cpu_baseline:
+            rate, secs, threads, desc = oracle_sample_rate(spec, args.cpu_sample_requests)
+            line["cpu_baseline"] = {"value": rate, "unit": UNIT, "cores": threads,
+                                    "kind": "oracle", "sample": desc, "seconds": secs}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        tdist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

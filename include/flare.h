@@ -1,0 +1,224 @@
+/*
+ * flare.h -- C ABI of the FLARE block-denoising attention step on GB300 (sm_103a).
+ *
+ * FLARE serves a hybrid backbone (gated-delta-rule linear attention layers
+ * interleaved with softmax attention layers) by denoising a block of B tokens
+ * per request.  Each block is processed by two kinds of forward pass (serving
+ * appendix, "Differences between the denoise pass and the state-update pass"):
+ *   - denoise passes read the committed recurrent state and the paged KV
+ *     prefix but write neither;
+ *   - one state-update pass writes the recurrent state at the accepted length.
+ * This library exposes exactly the per-layer attention work of those passes:
+ *
+ *   flare_block_linear_attn   gated-delta-rule block pass, block-end readout
+ *   flare_commit_state        write S^(r) into the state pool
+ *   flare_block_softmax_attn  block queries over paged prefix + block
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ *  - All tensor arguments are DEVICE pointers to contiguous row-major arrays
+ *    in the shapes stated per call.  Integer arrays are int32.
+ *  - Ownership: the caller allocates and frees every buffer (inputs, outputs,
+ *    pools, workspace, status word).  The library allocates no device memory,
+ *    frees nothing and never synchronizes inside a compute call.  Work is
+ *    enqueued on `stream` (a cudaStream_t passed as void*, NULL = legacy
+ *    default stream); a call returns once its kernels are enqueued.
+ *  - Errors a host can see (null pointer, unsupported size, bad dtype, too
+ *    small workspace) are returned immediately and nothing is launched.
+ *  - Errors only the device can see (a page id, state slot, prefix length or
+ *    accepted length out of range) set bits in *dev_status with an atomic OR
+ *    (FLARE_DEV_* below); the offending (request, head) item is skipped and its
+ *    outputs are left untouched.  Nothing traps.  The caller clears
+ *    *dev_status (4 bytes, device memory) and reads it back, e.g. with
+ *    flare_read_status.
+ *  - Kernels are launched on the current CUDA device; all pointers must live
+ *    on that device.
+ */
+#ifndef FLARE_H_
+#define FLARE_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum flare_status {
+  FLARE_OK = 0,
+  FLARE_ERR_INVALID_ARGUMENT = 1, /* null pointer, inconsistent sizes */
+  FLARE_ERR_UNSUPPORTED = 2,      /* sizes or dtypes this build does not implement */
+  FLARE_ERR_CUDA = 3,             /* a CUDA runtime call failed (launch, attribute) */
+  FLARE_ERR_DEVICE_STATUS = 4     /* flare_read_status found device error bits */
+} flare_status;
+
+typedef enum flare_dtype { FLARE_DT_BF16 = 0, FLARE_DT_F32 = 1 } flare_dtype;
+
+/* Softmax block mask (decoding appendix, attention patterns): every block row
+ * sees the whole prefix; in the denoise pass (BIDIR) it also sees every block
+ * token, in the state-update pass (CAUSAL) the block tokens up to itself. */
+typedef enum flare_mask_mode {
+  FLARE_MASK_BLOCK_BIDIR = 0,
+  FLARE_MASK_BLOCK_CAUSAL = 1
+} flare_mask_mode;
+
+/* Device status bits (OR-ed into *dev_status). */
+#define FLARE_DEV_BAD_SLOT 0x1       /* state_slot[r] outside [0, num_state_slots) */
+#define FLARE_DEV_BAD_PAGE 0x2       /* page id outside [0, num_pages) */
+#define FLARE_DEV_BAD_PREFIX_LEN 0x4 /* prefix_len[r] < 0 or > max_pages_per_req * page_size */
+#define FLARE_DEV_BAD_ACCEPT_LEN 0x8 /* accept_len[r] outside [0, block_len] */
+#define FLARE_DEV_WAIT_TIMEOUT 0x10  /* an in-kernel pipeline wait gave up (bounded spin) */
+
+/* Gated-delta-rule layer shape.
+ *   num_requests R, block_len B (1..64), num_qk_heads Hk, num_v_heads Hv
+ *   (Hv a multiple of Hk; value head j reads q/k head j / (Hv / Hk)),
+ *   head_dim_k dk and head_dim_v dv (each 64 or 128), num_state_slots in the
+ *   pool, act_dtype of q/k/v/out, scale s of the readout (the paper's
+ *   s = 1/sqrt(dk); pass it explicitly). */
+typedef struct flare_linear_desc {
+  int32_t num_requests;
+  int32_t block_len;
+  int32_t num_qk_heads;
+  int32_t num_v_heads;
+  int32_t head_dim_k;
+  int32_t head_dim_v;
+  int32_t num_state_slots;
+  flare_dtype act_dtype;
+  float scale;
+} flare_linear_desc;
+
+/* Softmax layer shape.
+ *   num_requests R, block_len B (1..64), num_q_heads Hq, num_kv_heads Hkv
+ *   (Hq a multiple of Hkv; q head h reads kv head h / (Hq / Hkv)), head_dim D
+ *   (64, 128 or 256), page_size p (16 or 64 tokens), num_pages in each pool,
+ *   max_pages_per_req (columns of the page table), act_dtype of every
+ *   activation and pool, scale of the logits (the paper's 1/sqrt(D)),
+ *   mask_mode as above. */
+typedef struct flare_softmax_desc {
+  int32_t num_requests;
+  int32_t block_len;
+  int32_t num_q_heads;
+  int32_t num_kv_heads;
+  int32_t head_dim;
+  int32_t page_size;
+  int32_t num_pages;
+  int32_t max_pages_per_req;
+  flare_dtype act_dtype;
+  float scale;
+  flare_mask_mode mask_mode;
+} flare_softmax_desc;
+
+/*
+ * Denoise pass of a gated-delta-rule layer (Eq. flare-gdn-schedule, noisy
+ * branch; Eq. noisy-block-fwd).  For each request r and value head j the block
+ * recurrence starts from S0 = state_pool[state_slot[r]][j] and runs the B
+ * block tokens through the gated delta rule (Eq. per-step-fwd); every block
+ * position then reads the block-end state:
+ *     out[r][l][j] = scale * S_B^T q[r][l][h],   h = j / (Hv / Hk),  all l.
+ * The state pool is read and NEVER written.
+ *   q, k        [R, B, Hk, dk]   act_dtype
+ *   v           [R, B, Hv, dv]   act_dtype
+ *   log_decay   [R, B, Hv]       fp32, g_t (the gate is exp(g_t))
+ *   beta        [R, B, Hv]       fp32
+ *   state_pool  [num_state_slots, Hv, dk, dv] fp32, S[i][c] at i*dv + c
+ *   state_slot  [R]              int32
+ *   out         [R, B, Hv, dv]   act_dtype
+ *   dev_status  int32 (device)   FLARE_DEV_BAD_SLOT
+ */
+flare_status flare_block_linear_attn(const flare_linear_desc* desc, const void* q,
+                                     const void* k, const void* v, const float* log_decay,
+                                     const float* beta, const float* state_pool,
+                                     const int32_t* state_slot, void* out, int32_t* dev_status,
+                                     void* stream);
+
+/*
+ * State commit at the accepted length (serving appendix, "Recovering the
+ * recurrent state at the accept boundary"; Eq. chunk-state / Eq. f-blk for a
+ * full block).  With the state-update pass's own block inputs, for each
+ * request r with n = accept_len[r] in [0, B]:
+ *     state_pool[state_slot[r]][j] <- S_n,
+ * the state after the first n block tokens of the gated delta rule started
+ * from the committed state.  n = 0 leaves the slot untouched (bit-identical);
+ * n = B applies the full clean-transition map.  Written in place.
+ * If causal_out is non-NULL the token-causal outputs of the state-update pass
+ * are written for every block position t (Eq. per-step-fwd, o_t line):
+ *     causal_out[r][t][j] = scale * S_t^T q[r][t][h]   (q must then be non-NULL).
+ * Precondition: the state_slot entries are distinct within one call.
+ *   q (nullable), k, v, log_decay, beta, state_pool, state_slot: as above
+ *   accept_len  [R]             int32
+ *   causal_out  [R, B, Hv, dv]  act_dtype, nullable
+ *   dev_status  FLARE_DEV_BAD_SLOT | FLARE_DEV_BAD_ACCEPT_LEN
+ */
+flare_status flare_commit_state(const flare_linear_desc* desc, const void* q, const void* k,
+                                const void* v, const float* log_decay, const float* beta,
+                                float* state_pool, const int32_t* state_slot,
+                                const int32_t* accept_len, void* causal_out,
+                                int32_t* dev_status, void* stream);
+
+/*
+ * Bytes of device workspace flare_block_softmax_attn needs for `desc`
+ * (partial outputs of split prefixes).  May be 0.  Host-only, no GPU work.
+ */
+flare_status flare_softmax_workspace_size(const flare_softmax_desc* desc, size_t* bytes);
+
+/*
+ * Block-query softmax attention over a paged KV prefix (Eq. softmax-retrieval
+ * with the Diffusion-Trust block mask; native dLLM mask modes of the serving
+ * appendix).  For request r, query head h (kv head h / (Hq / Hkv)) and block
+ * row t the visible keys are the prefix tokens j < prefix_len[r], read from
+ * page page_table[r][j / p], row j % p of the pools, followed by the block's
+ * own keys (all B of them in BIDIR mode, 0..t in CAUSAL mode):
+ *     out[r][t][h] = sum_i softmax_i(scale * q . k_i) v_i
+ *     lse[r][t][h] = log sum_i exp(scale * q . k_i)          (natural log)
+ * The block's keys/values are not in the pools (they are appended only by the
+ * state-update pass).  Pool rows past a request's prefix end are never used,
+ * whatever they hold.
+ *   q              [R, B, Hq, D]                 act_dtype
+ *   k_blk, v_blk   [R, B, Hkv, D]                act_dtype
+ *   k_pool, v_pool [num_pages, Hkv, p, D]        act_dtype
+ *   page_table     [R, max_pages_per_req]        int32
+ *   prefix_len     [R]                           int32
+ *   out            [R, B, Hq, D]                 act_dtype
+ *   lse            [R, B, Hq]                    fp32, nullable
+ *   workspace      >= flare_softmax_workspace_size bytes, 256-byte aligned
+ *                  (may be NULL when that size is 0)
+ *   dev_status     FLARE_DEV_BAD_PAGE | FLARE_DEV_BAD_PREFIX_LEN | FLARE_DEV_WAIT_TIMEOUT
+ */
+flare_status flare_block_softmax_attn(const flare_softmax_desc* desc, const void* q,
+                                      const void* k_blk, const void* v_blk, const void* k_pool,
+                                      const void* v_pool, const int32_t* page_table,
+                                      const int32_t* prefix_len, void* out, float* lse,
+                                      void* workspace, size_t workspace_bytes,
+                                      int32_t* dev_status, void* stream);
+
+/*
+ * Test/debug helper: dense copy of request `request`'s paged prefix,
+ * k_out/v_out [prefix_len[request], Hkv, D] act_dtype (the caller sizes them
+ * from the prefix length it wrote).  Same page arithmetic as the attention
+ * kernels; bit-exact copy.  dev_status: FLARE_DEV_BAD_PAGE | FLARE_DEV_BAD_PREFIX_LEN.
+ */
+flare_status flare_debug_gather_prefix(const flare_softmax_desc* desc, const void* k_pool,
+                                       const void* v_pool, const int32_t* page_table,
+                                       const int32_t* prefix_len, int32_t request, void* k_out,
+                                       void* v_out, int32_t* dev_status, void* stream);
+
+/*
+ * Waits for `stream`, copies the status word to *bits_out (nullable) and
+ * returns FLARE_ERR_DEVICE_STATUS if any bit is set, FLARE_ERR_CUDA if the
+ * stream reported an error, else FLARE_OK.  This is the one call that
+ * synchronizes.
+ */
+flare_status flare_read_status(const int32_t* dev_status, void* stream, int32_t* bits_out);
+
+/* Static string naming a status code. */
+const char* flare_status_string(flare_status status);
+
+/* Number of kernels this library has enqueued since it was loaded, over all
+ * devices and threads (diagnostic; a relaxed atomic counter). */
+uint64_t flare_launch_count(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FLARE_H_ */

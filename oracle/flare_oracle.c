@@ -108,6 +108,8 @@ int oracle_gdr_per_token(int R, int B, int Hk, int Hv, int dk, int dv, double s,
     const int r_acc = accept_len ? accept_len[r] : B;
     double* S = (double*)malloc(sizeof(double) * dk * dv);
     double* u = (double*)malloc(sizeof(double) * dv);
+    double* kt = (double*)malloc(sizeof(double) * dk);
+    double* qt = (double*)malloc(sizeof(double) * dk);
     const size_t s0 = ((size_t)state_slot[r] * Hv + j) * dk * dv;
     for (int e = 0; e < dk * dv; ++e) S[e] = ld(state_pool, state_dt, s0 + e);
     if (state_out && r_acc == 0)
@@ -118,26 +120,26 @@ int oracle_gdr_per_token(int R, int B, int Hk, int Hv, int dk, int dv, double s,
       const size_t gb = ((size_t)r * B + t) * Hv + j;
       const double alpha = exp(ld(log_decay, gate_dt, gb));
       const double bt = ld(beta, gate_dt, gb);
+      for (int i = 0; i < dk; ++i) kt[i] = ld(k, act_dt, kq + i);
       /* gating decay: S_pre = exp(g_t) S_{t-1} */
       for (int e = 0; e < dk * dv; ++e) S[e] *= alpha;
       /* prediction error u_t = v_t - S_pre^T k_t, delta update delta_t = beta_t u_t */
-      for (int c = 0; c < dv; ++c) {
-        double acc = 0.0;
-        for (int i = 0; i < dk; ++i) acc += S[i * dv + c] * ld(k, act_dt, kq + i);
-        u[c] = bt * (ld(v, act_dt, vo + c) - acc);
-      }
+      for (int c = 0; c < dv; ++c) u[c] = 0.0;
+      for (int i = 0; i < dk; ++i)
+        for (int c = 0; c < dv; ++c) u[c] += S[i * dv + c] * kt[i];
+      for (int c = 0; c < dv; ++c) u[c] = bt * (ld(v, act_dt, vo + c) - u[c]);
       /* outer-product write S_t = S_pre + k_t delta_t^T */
-      for (int i = 0; i < dk; ++i) {
-        const double ki = ld(k, act_dt, kq + i);
-        for (int c = 0; c < dv; ++c) S[i * dv + c] += ki * u[c];
-      }
+      for (int i = 0; i < dk; ++i)
+        for (int c = 0; c < dv; ++c) S[i * dv + c] += kt[i] * u[c];
       /* token-causal output o_t = s S_t^T q_t */
-      if (out_causal)
+      if (out_causal) {
+        for (int i = 0; i < dk; ++i) qt[i] = ld(q, act_dt, kq + i);
         for (int c = 0; c < dv; ++c) {
           double acc = 0.0;
-          for (int i = 0; i < dk; ++i) acc += S[i * dv + c] * ld(q, act_dt, kq + i);
+          for (int i = 0; i < dk; ++i) acc += S[i * dv + c] * qt[i];
           out_causal[vo + c] = s * acc;
         }
+      }
       if (state_out && t + 1 == r_acc)
         for (int e = 0; e < dk * dv; ++e) state_out[(size_t)item * dk * dv + e] = S[e];
     }
@@ -146,12 +148,15 @@ int oracle_gdr_per_token(int R, int B, int Hk, int Hv, int dk, int dv, double s,
       for (int l = 0; l < B; ++l) {
         const size_t ql = (((size_t)r * B + l) * Hk + h) * dk;
         const size_t ol = (((size_t)r * B + l) * Hv + j) * dv;
+        for (int i = 0; i < dk; ++i) qt[i] = ld(q, act_dt, ql + i);
         for (int c = 0; c < dv; ++c) {
           double acc = 0.0;
-          for (int i = 0; i < dk; ++i) acc += S[i * dv + c] * ld(q, act_dt, ql + i);
+          for (int i = 0; i < dk; ++i) acc += S[i * dv + c] * qt[i];
           out_blockend[ol + c] = s * acc;
         }
       }
+    free(qt);
+    free(kt);
     free(u);
     free(S);
   }
@@ -321,17 +326,19 @@ int oracle_block_softmax(int R, int B, int Hq, int Hkv, int D, int page_size, in
     const int nblk = (mask_mode == 0) ? B : t + 1;
     const int n = P + nblk;
     double* z = (double*)malloc(sizeof(double) * (n > 0 ? n : 1));
+    double* qv = (double*)malloc(sizeof(double) * D);
     const size_t qo = (((size_t)r * B + t) * Hq + h) * D;
+    for (int d = 0; d < D; ++d) qv[d] = ld(q, act_dt, qo + d);
     /* visible keys: prefix first, then the block */
     for (int jt = 0; jt < n; ++jt) {
       double acc = 0.0;
       if (jt < P) {
         const int page = page_table[(size_t)r * max_pages + jt / page_size];
         const size_t ko = (((size_t)page * Hkv + kvh) * page_size + jt % page_size) * D;
-        for (int d = 0; d < D; ++d) acc += ld(q, act_dt, qo + d) * ld(k_pool, act_dt, ko + d);
+        for (int d = 0; d < D; ++d) acc += qv[d] * ld(k_pool, act_dt, ko + d);
       } else {
         const size_t ko = (((size_t)r * B + (jt - P)) * Hkv + kvh) * D;
-        for (int d = 0; d < D; ++d) acc += ld(q, act_dt, qo + d) * ld(k_blk, act_dt, ko + d);
+        for (int d = 0; d < D; ++d) acc += qv[d] * ld(k_blk, act_dt, ko + d);
       }
       z[jt] = scale * acc;
     }
@@ -357,6 +364,7 @@ int oracle_block_softmax(int R, int B, int Hq, int Hkv, int D, int page_size, in
       out[qo + d] = acc / Z;
     }
     if (lse) lse[((size_t)r * B + t) * Hq + h] = m + log(Z);
+    free(qv);
     free(z);
   }
   return 0;

@@ -1,0 +1,302 @@
+// C ABI of the FLARE attention step: argument checks, work planning, launch.
+// The declarations and the contract of every entry point are in flare.h.
+#include <cuda_runtime.h>
+#include <stdint.h>
+#include <string.h>
+
+#include <atomic>
+
+#include "flare.h"
+#include "kernels.h"
+
+namespace flare {
+cudaError_t launch_softmax_simt(const SoftmaxParams& p, const SoftmaxPlan& plan, bool bf16,
+                                cudaStream_t stream);
+}
+
+using namespace flare;
+
+namespace {
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+bool valid_dtype(flare_dtype d) { return d == FLARE_DT_BF16 || d == FLARE_DT_F32; }
+
+flare_status check_linear(const flare_linear_desc* d) {
+  if (!d) return FLARE_ERR_INVALID_ARGUMENT;
+  if (d->num_requests < 0 || d->block_len < 1 || d->num_qk_heads < 1 || d->num_v_heads < 1 ||
+      d->num_state_slots < 1 || !valid_dtype(d->act_dtype))
+    return FLARE_ERR_INVALID_ARGUMENT;
+  if (d->num_v_heads % d->num_qk_heads != 0) return FLARE_ERR_INVALID_ARGUMENT;
+  if (d->block_len > 64) return FLARE_ERR_UNSUPPORTED;
+  if ((d->head_dim_k != 64 && d->head_dim_k != 128) ||
+      (d->head_dim_v != 64 && d->head_dim_v != 128))
+    return FLARE_ERR_UNSUPPORTED;
+  return FLARE_OK;
+}
+
+flare_status check_softmax(const flare_softmax_desc* d) {
+  if (!d) return FLARE_ERR_INVALID_ARGUMENT;
+  if (d->num_requests < 0 || d->block_len < 1 || d->num_q_heads < 1 || d->num_kv_heads < 1 ||
+      d->page_size < 1 || d->num_pages < 0 || d->max_pages_per_req < 0 ||
+      !valid_dtype(d->act_dtype))
+    return FLARE_ERR_INVALID_ARGUMENT;
+  if (d->mask_mode != FLARE_MASK_BLOCK_BIDIR && d->mask_mode != FLARE_MASK_BLOCK_CAUSAL)
+    return FLARE_ERR_INVALID_ARGUMENT;
+  if (d->num_q_heads % d->num_kv_heads != 0) return FLARE_ERR_INVALID_ARGUMENT;
+  if (d->block_len > 64) return FLARE_ERR_UNSUPPORTED;
+  if (d->head_dim != 64 && d->head_dim != 128 && d->head_dim != 256) return FLARE_ERR_UNSUPPORTED;
+  if (d->page_size != 16 && d->page_size != 32 && d->page_size != 64 && d->page_size != 128)
+    return FLARE_ERR_UNSUPPORTED;
+  if ((int64_t)d->max_pages_per_req * d->page_size > (1 << 24)) return FLARE_ERR_UNSUPPORTED;
+  return FLARE_OK;
+}
+
+int device_sms() {
+  int dev = 0, n = kNumSMs;
+  if (cudaGetDevice(&dev) == cudaSuccess)
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+  return n > 0 ? n : kNumSMs;
+}
+
+SoftmaxParams softmax_params(const flare_softmax_desc* d) {
+  SoftmaxParams p;
+  memset(&p, 0, sizeof p);
+  p.R = d->num_requests;
+  p.B = d->block_len;
+  p.Hq = d->num_q_heads;
+  p.Hkv = d->num_kv_heads;
+  p.G = d->num_q_heads / d->num_kv_heads;
+  p.D = d->head_dim;
+  p.page_size = d->page_size;
+  p.num_pages = d->num_pages;
+  p.max_pages = d->max_pages_per_req;
+  p.scale_log2 = d->scale * 1.4426950408889634f;
+  p.causal = d->mask_mode == FLARE_MASK_BLOCK_CAUSAL;
+  return p;
+}
+
+SoftmaxPlan plan_for(const flare_softmax_desc* d) {
+  return plan_softmax(d->num_requests, d->block_len, d->num_q_heads, d->num_kv_heads,
+                      d->head_dim, d->page_size, d->max_pages_per_req,
+                      d->act_dtype == FLARE_DT_BF16, device_sms());
+}
+
+}  // namespace
+
+namespace flare {
+
+static std::atomic<uint64_t> g_launches{0};
+void note_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
+
+SoftmaxPlan plan_softmax(int R, int B, int Hq, int Hkv, int D, int page_size, int max_pages,
+                         bool bf16, int num_sms) {
+  (void)bf16;
+  SoftmaxPlan pl;
+  memset(&pl, 0, sizeof pl);
+  pl.kernel = 0;
+  pl.rows_per_cta = 16;
+  const int G = Hq / Hkv, M = B * G;
+  const long total_max = (long)max_pages * page_size + B;
+  const long base = (long)R * Hkv * ((M + pl.rows_per_cta - 1) / pl.rows_per_cta);
+  const long target = 4L * num_sms;
+  long ns = base > 0 ? (target + base - 1) / base : 1;
+  const long max_split = (total_max + 255) / 256;
+  if (ns > max_split) ns = max_split;
+  if (ns < 1) ns = 1;
+  long len = (total_max + ns - 1) / ns;
+  len = (len + 63) / 64 * 64;
+  ns = (total_max + len - 1) / len;
+  pl.n_split = (int)ns;
+  pl.split_len = (int)len;
+  if (pl.n_split > 1) {
+    const size_t rows = (size_t)R * Hkv * pl.n_split * M;
+    pl.ws_o_bytes = (rows * D * sizeof(float) + 255) / 256 * 256;
+    pl.ws_lse_bytes = (rows * sizeof(float) + 255) / 256 * 256;
+  }
+  pl.workspace_bytes = pl.ws_o_bytes + pl.ws_lse_bytes;
+  return pl;
+}
+
+cudaError_t launch_softmax(const SoftmaxParams& p, const SoftmaxPlan& plan, bool bf16,
+                           cudaStream_t stream) {
+  return launch_softmax_simt(p, plan, bf16, stream);
+}
+
+}  // namespace flare
+
+extern "C" {
+
+const char* flare_status_string(flare_status s) {
+  switch (s) {
+    case FLARE_OK: return "FLARE_OK";
+    case FLARE_ERR_INVALID_ARGUMENT: return "FLARE_ERR_INVALID_ARGUMENT";
+    case FLARE_ERR_UNSUPPORTED: return "FLARE_ERR_UNSUPPORTED";
+    case FLARE_ERR_CUDA: return "FLARE_ERR_CUDA";
+    case FLARE_ERR_DEVICE_STATUS: return "FLARE_ERR_DEVICE_STATUS";
+  }
+  return "FLARE_ERR_UNKNOWN";
+}
+
+flare_status flare_block_linear_attn(const flare_linear_desc* d, const void* q, const void* k,
+                                     const void* v, const float* log_decay, const float* beta,
+                                     const float* state_pool, const int32_t* state_slot,
+                                     void* out, int32_t* dev_status, void* stream) {
+  flare_status st = check_linear(d);
+  if (st != FLARE_OK) return st;
+  if (!q || !k || !v || !log_decay || !beta || !state_pool || !state_slot || !out || !dev_status)
+    return FLARE_ERR_INVALID_ARGUMENT;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(state_pool) ||
+      !aligned16(out))
+    return FLARE_ERR_INVALID_ARGUMENT;
+  if (d->num_requests == 0) return FLARE_OK;
+  GdrParams p;
+  memset(&p, 0, sizeof p);
+  p.R = d->num_requests;
+  p.B = d->block_len;
+  p.Hk = d->num_qk_heads;
+  p.Hv = d->num_v_heads;
+  p.dk = d->head_dim_k;
+  p.dv = d->head_dim_v;
+  p.nslots = d->num_state_slots;
+  p.scale = d->scale;
+  p.q = q;
+  p.k = k;
+  p.v = v;
+  p.log_decay = log_decay;
+  p.beta = beta;
+  p.state_pool = const_cast<float*>(state_pool);  // read only: write_state = 0
+  p.state_slot = state_slot;
+  p.out_blockend = out;
+  p.write_state = 0;
+  p.dev_status = dev_status;
+  const cudaError_t e = launch_gdr_recurrent(p, d->act_dtype == FLARE_DT_BF16,
+                                             static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? FLARE_OK : FLARE_ERR_CUDA;
+}
+
+flare_status flare_commit_state(const flare_linear_desc* d, const void* q, const void* k,
+                                const void* v, const float* log_decay, const float* beta,
+                                float* state_pool, const int32_t* state_slot,
+                                const int32_t* accept_len, void* causal_out,
+                                int32_t* dev_status, void* stream) {
+  flare_status st = check_linear(d);
+  if (st != FLARE_OK) return st;
+  if (!k || !v || !log_decay || !beta || !state_pool || !state_slot || !accept_len ||
+      !dev_status || (causal_out && !q))
+    return FLARE_ERR_INVALID_ARGUMENT;
+  if ((q && !aligned16(q)) || !aligned16(k) || !aligned16(v) || !aligned16(state_pool) ||
+      (causal_out && !aligned16(causal_out)))
+    return FLARE_ERR_INVALID_ARGUMENT;
+  if (d->num_requests == 0) return FLARE_OK;
+  GdrParams p;
+  memset(&p, 0, sizeof p);
+  p.R = d->num_requests;
+  p.B = d->block_len;
+  p.Hk = d->num_qk_heads;
+  p.Hv = d->num_v_heads;
+  p.dk = d->head_dim_k;
+  p.dv = d->head_dim_v;
+  p.nslots = d->num_state_slots;
+  p.scale = d->scale;
+  p.q = causal_out ? q : nullptr;
+  p.k = k;
+  p.v = v;
+  p.log_decay = log_decay;
+  p.beta = beta;
+  p.state_pool = state_pool;
+  p.state_slot = state_slot;
+  p.accept_len = accept_len;
+  p.out_causal = causal_out;
+  p.write_state = 1;
+  p.dev_status = dev_status;
+  const cudaError_t e = launch_gdr_recurrent(p, d->act_dtype == FLARE_DT_BF16,
+                                             static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? FLARE_OK : FLARE_ERR_CUDA;
+}
+
+flare_status flare_softmax_workspace_size(const flare_softmax_desc* d, size_t* bytes) {
+  flare_status st = check_softmax(d);
+  if (st != FLARE_OK) return st;
+  if (!bytes) return FLARE_ERR_INVALID_ARGUMENT;
+  *bytes = d->num_requests == 0 ? 0 : plan_for(d).workspace_bytes;
+  return FLARE_OK;
+}
+
+flare_status flare_block_softmax_attn(const flare_softmax_desc* d, const void* q,
+                                      const void* k_blk, const void* v_blk, const void* k_pool,
+                                      const void* v_pool, const int32_t* page_table,
+                                      const int32_t* prefix_len, void* out, float* lse,
+                                      void* workspace, size_t workspace_bytes,
+                                      int32_t* dev_status, void* stream) {
+  flare_status st = check_softmax(d);
+  if (st != FLARE_OK) return st;
+  if (!q || !k_blk || !v_blk || !prefix_len || !out || !dev_status)
+    return FLARE_ERR_INVALID_ARGUMENT;
+  if (d->max_pages_per_req > 0 && (!k_pool || !v_pool || !page_table))
+    return FLARE_ERR_INVALID_ARGUMENT;
+  if (!aligned16(q) || !aligned16(k_blk) || !aligned16(v_blk) || !aligned16(k_pool) ||
+      !aligned16(v_pool) || !aligned16(out))
+    return FLARE_ERR_INVALID_ARGUMENT;
+  if (d->num_requests == 0) return FLARE_OK;
+  const SoftmaxPlan plan = plan_for(d);
+  if (workspace_bytes < plan.workspace_bytes) return FLARE_ERR_INVALID_ARGUMENT;
+  if (plan.workspace_bytes && (!workspace || ((uintptr_t)workspace & 255u)))
+    return FLARE_ERR_INVALID_ARGUMENT;
+  SoftmaxParams p = softmax_params(d);
+  p.q = q;
+  p.k_blk = k_blk;
+  p.v_blk = v_blk;
+  p.k_pool = k_pool;
+  p.v_pool = v_pool;
+  p.page_table = page_table;
+  p.prefix_len = prefix_len;
+  p.out = out;
+  p.lse = lse;
+  p.n_split = plan.n_split;
+  p.split_len = plan.split_len;
+  if (plan.workspace_bytes) {
+    p.ws_o = static_cast<float*>(workspace);
+    p.ws_lse = reinterpret_cast<float*>(static_cast<char*>(workspace) + plan.ws_o_bytes);
+  }
+  p.dev_status = dev_status;
+  const cudaError_t e = launch_softmax(p, plan, d->act_dtype == FLARE_DT_BF16,
+                                       static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? FLARE_OK : FLARE_ERR_CUDA;
+}
+
+flare_status flare_debug_gather_prefix(const flare_softmax_desc* d, const void* k_pool,
+                                       const void* v_pool, const int32_t* page_table,
+                                       const int32_t* prefix_len, int32_t request, void* k_out,
+                                       void* v_out, int32_t* dev_status, void* stream) {
+  flare_status st = check_softmax(d);
+  if (st != FLARE_OK) return st;
+  if (!k_pool || !v_pool || !page_table || !prefix_len || !k_out || !v_out || !dev_status)
+    return FLARE_ERR_INVALID_ARGUMENT;
+  if (request < 0 || request >= d->num_requests) return FLARE_ERR_INVALID_ARGUMENT;
+  SoftmaxParams p = softmax_params(d);
+  p.k_pool = k_pool;
+  p.v_pool = v_pool;
+  p.page_table = page_table;
+  p.prefix_len = prefix_len;
+  p.dev_status = dev_status;
+  const cudaError_t e = launch_gather_prefix(p, request, k_out, v_out,
+                                             d->act_dtype == FLARE_DT_BF16,
+                                             static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? FLARE_OK : FLARE_ERR_CUDA;
+}
+
+uint64_t flare_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+flare_status flare_read_status(const int32_t* dev_status, void* stream, int32_t* bits_out) {
+  if (!dev_status) return FLARE_ERR_INVALID_ARGUMENT;
+  int32_t bits = 0;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaMemcpyAsync(&bits, dev_status, sizeof bits, cudaMemcpyDeviceToHost, s) != cudaSuccess)
+    return FLARE_ERR_CUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return FLARE_ERR_CUDA;
+  if (bits_out) *bits_out = bits;
+  return bits ? FLARE_ERR_DEVICE_STATUS : FLARE_OK;
+}
+
+}  // extern "C"

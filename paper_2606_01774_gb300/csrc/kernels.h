@@ -1,0 +1,72 @@
+// Internal launch interface between the C ABI layer and the kernels.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace flare {
+
+constexpr int kNumSMs = 152;  // GB300: 2 dies x 76 SMs (re-read at run time)
+
+// Counts kernel launches for flare_launch_count().
+void note_launches(int n);
+
+struct GdrParams {
+  int R, B, Hk, Hv, dk, dv, nslots;
+  float scale;
+  const void* q;  // [R,B,Hk,dk], nullable when no readout is asked
+  const void* k;  // [R,B,Hk,dk]
+  const void* v;  // [R,B,Hv,dv]
+  const float* log_decay;  // [R,B,Hv]
+  const float* beta;       // [R,B,Hv]
+  float* state_pool;       // [nslots,Hv,dk,dv]; written only when write_state
+  const int32_t* state_slot;  // [R]
+  const int32_t* accept_len;  // [R] or nullptr (= B)
+  void* out_blockend;         // [R,B,Hv,dv] or nullptr
+  void* out_causal;           // [R,B,Hv,dv] or nullptr
+  int write_state;
+  int32_t* dev_status;
+};
+
+struct SoftmaxParams {
+  int R, B, Hq, Hkv, G, D, page_size, num_pages, max_pages;
+  float scale_log2;  // logit scale * log2(e)
+  int causal;
+  const void* q;      // [R,B,Hq,D]
+  const void* k_blk;  // [R,B,Hkv,D]
+  const void* v_blk;
+  const void* k_pool;  // [num_pages,Hkv,page_size,D]
+  const void* v_pool;
+  const int32_t* page_table;  // [R,max_pages]
+  const int32_t* prefix_len;  // [R]
+  void* out;                  // [R,B,Hq,D]
+  float* lse;                 // [R,B,Hq] or nullptr
+  float* ws_o;                // split partial outputs [R*Hkv][n_split][B*G][D]
+  float* ws_lse;              // split partial lse     [R*Hkv][n_split][B*G]
+  int n_split, split_len;
+  int32_t* dev_status;
+};
+
+// Work decomposition of the softmax call; identical for the workspace query
+// and the launch.
+struct SoftmaxPlan {
+  int kernel;  // 0 = CUDA-core kernel, 1 = tensor-core kernel
+  int rows_per_cta;
+  int n_split;
+  int split_len;
+  size_t ws_o_bytes, ws_lse_bytes;
+  size_t workspace_bytes;
+};
+
+size_t gdr_recurrent_smem_bytes(int dk, int dv, int threads);
+cudaError_t launch_gdr_recurrent(const GdrParams& p, bool bf16, cudaStream_t stream);
+
+SoftmaxPlan plan_softmax(int R, int B, int Hq, int Hkv, int D, int page_size, int max_pages,
+                         bool bf16, int num_sms);
+cudaError_t launch_softmax(const SoftmaxParams& p, const SoftmaxPlan& plan, bool bf16,
+                           cudaStream_t stream);
+cudaError_t launch_gather_prefix(const SoftmaxParams& p, int request, void* k_out, void* v_out,
+                                 bool bf16, cudaStream_t stream);
+
+}  // namespace flare

@@ -1,0 +1,63 @@
+"""CPU checks of the C-ABI library: it builds, loads, exports every entry point
+include/flare.h declares, and rejects bad arguments on the host before any
+CUDA work (no compute call is made here)."""
+import ctypes
+
+import pytest
+
+from paper_2606_01774_gb300 import build, flare
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return flare.load()
+
+
+def test_header_declares_the_boundary():
+    names = flare.declared_functions()
+    for n in ("flare_block_linear_attn", "flare_commit_state", "flare_block_softmax_attn",
+              "flare_softmax_workspace_size", "flare_debug_gather_prefix", "flare_read_status",
+              "flare_status_string"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for n in flare.declared_functions():
+        assert hasattr(lib, n), n
+
+
+def test_status_strings(lib):
+    assert flare.flare_status_string(0) == "FLARE_OK"
+    assert flare.flare_status_string(4) == "FLARE_ERR_DEVICE_STATUS"
+
+
+def test_host_argument_checks_need_no_gpu(lib):
+    d = flare.linear_desc(2, 32, 16, 32, 128, 128, 6, flare.FLARE_DT_BF16, 0.088)
+    null = [None] * 10
+    assert lib.flare_block_linear_attn(ctypes.byref(d), *null) == flare.FLARE_ERR_INVALID_ARGUMENT
+    d.head_dim_k = 96
+    assert lib.flare_block_linear_attn(ctypes.byref(d), *null) == flare.FLARE_ERR_UNSUPPORTED
+    d.head_dim_k = 128
+    d.num_v_heads = 24
+    d.num_qk_heads = 16
+    assert lib.flare_block_linear_attn(ctypes.byref(d), *null) == flare.FLARE_ERR_INVALID_ARGUMENT
+    assert lib.flare_block_linear_attn(None, *null) == flare.FLARE_ERR_INVALID_ARGUMENT
+    s = flare.softmax_desc(2, 32, 16, 2, 256, 64, 100, 64, flare.FLARE_DT_BF16, 0.0625)
+    s.mask_mode = 7
+    n = ctypes.c_size_t(0)
+    assert lib.flare_softmax_workspace_size(ctypes.byref(s), ctypes.byref(n)) == \
+        flare.FLARE_ERR_INVALID_ARGUMENT
+    s.mask_mode = 0
+    s.page_size = 48
+    assert lib.flare_softmax_workspace_size(ctypes.byref(s), ctypes.byref(n)) == \
+        flare.FLARE_ERR_UNSUPPORTED
+    assert lib.flare_read_status(None, None, None) == flare.FLARE_ERR_INVALID_ARGUMENT
+
+
+def test_workspace_query_is_host_only(lib):
+    s = flare.softmax_desc(1, 32, 16, 2, 256, 64, 100, 64, flare.FLARE_DT_BF16, 0.0625)
+    n = flare.flare_softmax_workspace_size(s)
+    assert n >= 0 and n % 256 == 0
+    s.num_requests = 0
+    assert flare.flare_softmax_workspace_size(s) == 0
