@@ -9,11 +9,6 @@
 #include "flare.h"
 #include "kernels.h"
 
-namespace flare {
-cudaError_t launch_softmax_simt(const SoftmaxParams& p, const SoftmaxPlan& plan, bool bf16,
-                                cudaStream_t stream);
-}
-
 using namespace flare;
 
 namespace {
@@ -91,24 +86,42 @@ void note_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_
 
 SoftmaxPlan plan_softmax(int R, int B, int Hq, int Hkv, int D, int page_size, int max_pages,
                          bool bf16, int num_sms) {
-  (void)bf16;
   SoftmaxPlan pl;
   memset(&pl, 0, sizeof pl);
-  pl.kernel = 0;
-  pl.rows_per_cta = 16;
   const int G = Hq / Hkv, M = B * G;
-  const long total_max = (long)max_pages * page_size + B;
-  const long base = (long)R * Hkv * ((M + pl.rows_per_cta - 1) / pl.rows_per_cta);
-  const long target = 4L * num_sms;
-  long ns = base > 0 ? (target + base - 1) / base : 1;
-  const long max_split = (total_max + 255) / 256;
-  if (ns > max_split) ns = max_split;
-  if (ns < 1) ns = 1;
-  long len = (total_max + ns - 1) / ns;
-  len = (len + 63) / 64 * 64;
-  ns = (total_max + len - 1) / len;
-  pl.n_split = (int)ns;
-  pl.split_len = (int)len;
+  const long prefix_max = (long)max_pages * page_size;
+  if (bf16 && softmax_tc_supported(B, Hq, Hkv, D, page_size)) {
+    // tensor-core kernel: 128 query rows per CTA, one CTA per SM; split the
+    // prefix only when the batch gives fewer than two CTAs per SM, and keep
+    // at least 16 tiles (1024 keys) per split so partials stay small.
+    pl.kernel = 1;
+    pl.rows_per_cta = 128;
+    const long items = (long)R * Hkv * ((M + 127) / 128);
+    const long tiles = (prefix_max + 63) / 64;
+    long ns = 1;
+    if (items > 0 && items < 2L * num_sms) ns = (2L * num_sms + items - 1) / items;
+    const long cap = tiles / 16 > 1 ? tiles / 16 : 1;
+    if (ns > cap) ns = cap;
+    const long tps = ns > 0 ? (tiles + ns - 1) / ns : 1;
+    pl.split_len = (int)((tps > 0 ? tps : 1) * 64);
+    pl.n_split = tiles > 0 ? (int)((tiles + tps - 1) / tps) : 1;
+    if (pl.n_split < 1) pl.n_split = 1;
+  } else {
+    pl.kernel = 0;
+    pl.rows_per_cta = 16;
+    const long total_max = prefix_max + B;
+    const long base = (long)R * Hkv * ((M + pl.rows_per_cta - 1) / pl.rows_per_cta);
+    const long target = 4L * num_sms;
+    long ns = base > 0 ? (target + base - 1) / base : 1;
+    const long max_split = (total_max + 255) / 256;
+    if (ns > max_split) ns = max_split;
+    if (ns < 1) ns = 1;
+    long len = (total_max + ns - 1) / ns;
+    len = (len + 63) / 64 * 64;
+    ns = (total_max + len - 1) / len;
+    pl.n_split = (int)ns;
+    pl.split_len = (int)len;
+  }
   if (pl.n_split > 1) {
     const size_t rows = (size_t)R * Hkv * pl.n_split * M;
     pl.ws_o_bytes = (rows * D * sizeof(float) + 255) / 256 * 256;
@@ -120,6 +133,7 @@ SoftmaxPlan plan_softmax(int R, int B, int Hq, int Hkv, int D, int page_size, in
 
 cudaError_t launch_softmax(const SoftmaxParams& p, const SoftmaxPlan& plan, bool bf16,
                            cudaStream_t stream) {
+  if (plan.kernel == 1) return launch_softmax_tc(p, plan, stream);
   return launch_softmax_simt(p, plan, bf16, stream);
 }
 

@@ -66,6 +66,12 @@ SoftmaxPlan plan_softmax(int R, int B, int Hq, int Hkv, int D, int page_size, in
                          bool bf16, int num_sms);
 cudaError_t launch_softmax(const SoftmaxParams& p, const SoftmaxPlan& plan, bool bf16,
                            cudaStream_t stream);
+cudaError_t launch_softmax_simt(const SoftmaxParams& p, const SoftmaxPlan& plan, bool bf16,
+                                cudaStream_t stream);
+cudaError_t launch_softmax_tc(const SoftmaxParams& p, const SoftmaxPlan& plan,
+                              cudaStream_t stream);
+cudaError_t launch_softmax_combine(const SoftmaxParams& p, bool bf16, cudaStream_t stream);
+bool softmax_tc_supported(int B, int Hq, int Hkv, int D, int page_size);
 cudaError_t launch_gather_prefix(const SoftmaxParams& p, int request, void* k_out, void* v_out,
                                  bool bf16, cudaStream_t stream);
 

@@ -212,9 +212,7 @@ cudaError_t launch_simt_d(const SoftmaxParams& p, const SoftmaxPlan& plan, cudaS
   note_launches(1);
   e = cudaGetLastError();
   if (e != cudaSuccess || plan.n_split == 1) return e;
-  softmax_combine_kernel<T><<<dim3(p.R * p.Hkv, M), 256, 0, stream>>>(p);
-  note_launches(1);
-  return cudaGetLastError();
+  return launch_softmax_combine(p, sizeof(T) == 2, stream);
 }
 
 template <typename T>
@@ -227,6 +225,16 @@ cudaError_t launch_simt(const SoftmaxParams& p, const SoftmaxPlan& plan, cudaStr
   }
 }
 }  // namespace
+
+cudaError_t launch_softmax_combine(const SoftmaxParams& p, bool bf16, cudaStream_t stream) {
+  const dim3 grid(p.R * p.Hkv, p.B * p.G);
+  if (bf16)
+    softmax_combine_kernel<__nv_bfloat16><<<grid, 256, 0, stream>>>(p);
+  else
+    softmax_combine_kernel<float><<<grid, 256, 0, stream>>>(p);
+  note_launches(1);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_softmax_simt(const SoftmaxParams& p, const SoftmaxPlan& plan, bool bf16,
                                 cudaStream_t stream) {
