@@ -184,8 +184,11 @@ flare_status flare_block_linear_attn(const flare_linear_desc* d, const void* q, 
   p.out_blockend = out;
   p.write_state = 0;
   p.dev_status = dev_status;
-  const cudaError_t e = launch_gdr_recurrent(p, d->act_dtype == FLARE_DT_BF16,
-                                             static_cast<cudaStream_t>(stream));
+  const bool bf16 = d->act_dtype == FLARE_DT_BF16;
+  const cudaError_t e =
+      (bf16 && gdr_denoise_tc_supported(p.B, p.dk, p.dv))
+          ? launch_gdr_denoise_tc(p, static_cast<cudaStream_t>(stream))
+          : launch_gdr_recurrent(p, bf16, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? FLARE_OK : FLARE_ERR_CUDA;
 }
 

@@ -1,0 +1,419 @@
+// Denoise pass of a gated-delta-rule layer on tcgen05 tensor cores.
+//
+// For one (request r, value head j) with q/k head h, block length B <= 64 and
+// frozen state S0 (dk x dv, fp32), the block-end readout (Eq. noisy-block-fwd)
+// is evaluated through the chunkwise WY/UT form of the block (appendix,
+// "Chunk-corrected values", Eq. chunk-state) instead of B sequential steps:
+//
+//   gamma_t = sum_{i<=t} g_i,  Gam_t = exp(gamma_t)             (cumulative log-gate)
+//   A[t][i] = beta_t exp(gamma_t - gamma_i) (k_t . k_i),  i < t
+//   T       = (I + A)^{-1}                                     (unit lower triangular)
+//   X       = diag(beta) (V - diag(Gam) K S0)
+//   delta   = T X                                              (per-step delta updates)
+//   out[l]  = s (Gam_B S0^T q_l + sum_i exp(gamma_B - gamma_i) (q_l . k_i) delta_i)
+//
+// Every product with S0 or delta is computed transposed, with the value
+// dimension c on the 128 TMEM lanes: column c of the state evolves
+// independently of the others (the update acts on S from the left), so thread
+// c owns everything about column c from the first MMA to its output.
+//
+//   MMA 1   G   = [K;Q] K^T          M=128 (64 k rows, 64 q rows), N=Bp, K=dk
+//   MMA 2   W^T = S0^T [K;Q]^T       M=128 (c),  N=128, K=dk   (S0^T is MN-major)
+//   solve   T   = (I + A)^{-1}       64 threads, one column each, in registers
+//   MMA 3   delta^T = X^T T^T        M=128 (c),  N=Bp,  K=Bp
+//   MMA 4   O2^T = delta^T M2^T      M=128 (c),  N=Bp,  K=Bp, M2[l][i] = exp(gamma_B-gamma_i) q_l.k_i
+//   out[l][c] = s (Gam_B W^T[c][64+l] + O2^T[c][l])
+//
+// Inputs bf16, state fp32 read once and rounded to bf16 for the MMA, all
+// accumulation fp32.  One CTA per (request, value head); 128 threads; 97 KiB
+// shared memory and 256 TMEM columns, so two CTAs share an SM.
+#include <cudaTypedefs.h>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "tc.cuh"
+
+namespace flare {
+
+namespace {
+
+constexpr int kLinThreads = 128;
+constexpr int kBmax = 64;
+
+template <int DK, int DV>
+struct LinCfg {
+  static constexpr int kKQ = (DK / 64) * 128 * 128;  // [K;Q]: DK/64 chunks of 128 rows x 128 B
+  static constexpr int kS0 = 2 * DK * 128;           // S0^T, MN-major: 2 chunks of DK rows x 128 B
+  static constexpr int kM2 = kBmax * 128;             // [l][i] K-major
+  static constexpr int kT = kBmax * 128;              // [t][i] K-major
+  static constexpr int kX = 128 * 128;                // X^T / delta^T [c][t] K-major; also A (fp32 64x64)
+  static constexpr int kSmem = kKQ + kS0 + kM2 + kT + kX;
+};
+
+struct LinShared {
+  uint64_t bar_kq, bar_mma;
+  uint32_t tmem_base;
+  int abort_flag;
+  float gam[kBmax];   // gamma_t
+  float Gam[kBmax];   // exp(gamma_t)
+  float beta[kBmax];
+};
+
+struct LinMaps {
+  CUtensorMap k;  // (dk, Hk, B, R)  box (64, 1, 64, 1), 128-byte swizzle
+  CUtensorMap q;
+};
+
+__device__ __forceinline__ bool lin_wait(uint64_t* bar, uint32_t parity, LinShared& sh,
+                                         int32_t* status) {
+  const bool ok = tc::mbar_wait(bar, parity, &sh.abort_flag);
+  const bool all = __syncthreads_and(ok);
+  if (!all && threadIdx.x == 0 && !sh.abort_flag) {
+    sh.abort_flag = 1;
+    flag(status, FLARE_DEV_WAIT_TIMEOUT);
+  }
+  return all;
+}
+
+__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float (&v)[64]) {
+  uint32_t r[64];
+#pragma unroll
+  for (int c = 0; c < 64; c += 16) tc::tmem_ld16(taddr + c, *reinterpret_cast<uint32_t(*)[16]>(&r[c]));
+  tc::tmem_ld_wait();
+#pragma unroll
+  for (int i = 0; i < 64; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// 64 bf16 values as one 128-byte row of a K-major SW128 tile.
+__device__ __forceinline__ void store_row_sw128(uint8_t* tile, int row, const float (&v)[64]) {
+  uint8_t* p = tile + row * 128;
+#pragma unroll
+  for (int c16 = 0; c16 < 8; ++c16) {
+    uint32_t w[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      __nv_bfloat162 h = __floats2bfloat162_rn(v[c16 * 8 + 2 * e], v[c16 * 8 + 2 * e + 1]);
+      w[e] = *reinterpret_cast<uint32_t*>(&h);
+    }
+    *reinterpret_cast<uint4*>(p + ((c16 ^ (row & 7)) * 16)) = make_uint4(w[0], w[1], w[2], w[3]);
+  }
+}
+
+}  // namespace
+
+template <int DK, int DV>
+__global__ void __launch_bounds__(kLinThreads, 2)
+    gdr_denoise_tc_kernel(const __grid_constant__ LinMaps maps, GdrParams p) {
+  using C = LinCfg<DK, DV>;
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ LinShared sh;
+  uint8_t* base = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint8_t* KQs = base;
+  uint8_t* S0s = KQs + C::kKQ;
+  uint8_t* M2s = S0s + C::kS0;
+  uint8_t* Ts = M2s + C::kM2;
+  uint8_t* Xs = Ts + C::kT;
+  float* A32 = reinterpret_cast<float*>(Xs);  // aliases X^T (A is dead before X is written)
+
+  const int item = blockIdx.x;
+  const int r = item / p.Hv, j = item % p.Hv;
+  const int h = j / (p.Hv / p.Hk);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int B = p.B;
+  const int Bp = (B + 15) & ~15;
+
+  const int slot = p.state_slot[r];
+  if (slot < 0 || slot >= p.nslots) {
+    if (tid == 0) flag(p.dev_status, FLARE_DEV_BAD_SLOT);
+    return;
+  }
+
+  if (tid == 0) {
+    sh.abort_flag = 0;
+    tc::mbar_init(&sh.bar_kq, 1);
+    tc::mbar_init(&sh.bar_mma, 1);
+    tc::fence_mbar_init();
+  }
+  if (warp == 0) tc::tmem_alloc(&sh.tmem_base, 256);
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = sh.tmem_base;
+  const uint32_t tmA = tmem;        // G, then delta^T, then O2^T   (64 columns)
+  const uint32_t tmW = tmem + 128;  // W^T = S0^T [K;Q]^T           (128 columns)
+  const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
+
+  if (tid == 0) {
+    tc::mbar_expect_tx(&sh.bar_kq, 2 * (DK / 64) * kBmax * 128);
+    for (int c = 0; c < DK / 64; ++c) {
+      tc::tma_load_4d(KQs + c * 16384, &maps.k, &sh.bar_kq, c * 64, h, 0, r);
+      tc::tma_load_4d(KQs + c * 16384 + 8192, &maps.q, &sh.bar_kq, c * 64, h, 0, r);
+    }
+  }
+
+  // S0 (fp32, global) -> bf16 S0^T operand, MN-major 128-byte swizzle:
+  // element (c, i) in chunk c/64 at row i, 16-byte group ((c%64)/8) ^ (i%8).
+  {
+    const float4* S0g =
+        reinterpret_cast<const float4*>(p.state_pool + ((size_t)slot * p.Hv + j) * DK * DV);
+    constexpr int kPer = DK * DV / 4 / kLinThreads;
+    float4 buf[kPer];
+#pragma unroll
+    for (int n = 0; n < kPer; ++n) buf[n] = __ldg(S0g + tid + n * kLinThreads);
+#pragma unroll
+    for (int n = 0; n < kPer; ++n) {
+      const int f = tid + n * kLinThreads;
+      const int i = f / (DV / 4), c = (f % (DV / 4)) * 4;
+      __nv_bfloat162 lo = __floats2bfloat162_rn(buf[n].x, buf[n].y);
+      __nv_bfloat162 hi = __floats2bfloat162_rn(buf[n].z, buf[n].w);
+      uint2 w = make_uint2(*reinterpret_cast<uint32_t*>(&lo), *reinterpret_cast<uint32_t*>(&hi));
+      const int cc = c & 63;
+      uint8_t* dst = S0s + (c >> 6) * (DK * 128) + i * 128 + (((cc >> 3) ^ (i & 7)) << 4) +
+                     ((cc & 7) << 1);
+      *reinterpret_cast<uint2*>(dst) = w;
+    }
+  }
+  // gates: gamma = inclusive prefix sum of the log-gates over the block
+  if (warp == 0) {
+    const size_t gb = (size_t)r * B * p.Hv + j;
+    float g0 = lane < B ? p.log_decay[gb + (size_t)lane * p.Hv] : 0.f;
+    float g1 = lane + 32 < B ? p.log_decay[gb + (size_t)(lane + 32) * p.Hv] : 0.f;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float a = __shfl_up_sync(0xffffffffu, g0, o);
+      const float b = __shfl_up_sync(0xffffffffu, g1, o);
+      if (lane >= o) {
+        g0 += a;
+        g1 += b;
+      }
+    }
+    g1 += __shfl_sync(0xffffffffu, g0, 31);
+    sh.gam[lane] = g0;
+    sh.gam[lane + 32] = g1;
+    sh.Gam[lane] = expf(g0);
+    sh.Gam[lane + 32] = expf(g1);
+    sh.beta[lane] = lane < B ? p.beta[gb + (size_t)lane * p.Hv] : 0.f;
+    sh.beta[lane + 32] = lane + 32 < B ? p.beta[gb + (size_t)(lane + 32) * p.Hv] : 0.f;
+  }
+  tc::fence_async_smem();
+  if (!lin_wait(&sh.bar_kq, 0, sh, p.dev_status)) goto done;
+
+  // ---- MMA 1 (Gram) and MMA 2 (state products)
+  if (tid == 0) {
+    tc::fence_after_sync();
+    const uint32_t idG = tc::idesc_bf16(128, Bp, false, false);
+    const uint32_t idW = tc::idesc_bf16(128, 128, true, false);
+#pragma unroll
+    for (int kk = 0; kk < DK / 16; ++kk) {
+      const int c = kk >> 2, off = (kk & 3) * 32;
+      const uint64_t kq = tc::sdesc_sw128(tc::smem_u32(KQs + c * 16384 + off), 16, 1024);
+      tc::mma_bf16_ss(tmA, kq, kq, idG, kk > 0);
+      const uint64_t s0 = tc::sdesc_sw128(tc::smem_u32(S0s + kk * 2048), DK * 128, 1024);
+      tc::mma_bf16_ss(tmW, s0, kq, idW, kk > 0);
+    }
+    tc::mma_commit(&sh.bar_mma);
+  }
+  if (!lin_wait(&sh.bar_mma, 0, sh, p.dev_status)) goto done;
+  tc::fence_after_sync();
+
+  // ---- A (rows 0..63 of G) and M2 (rows 64..127)
+  {
+    float gr[64];
+    tmem_ld64(tmA + lane_off, gr);
+    const int row = tid & 63;
+    const float gB = sh.gam[B - 1];
+    if (tid < 64) {
+      const float bt = sh.beta[row], gt = sh.gam[row];
+      float4* arow = reinterpret_cast<float4*>(A32 + row * 64);
+#pragma unroll
+      for (int i = 0; i < 64; i += 4) {
+        float a[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int ii = i + e;
+          a[e] = (ii < row && row < B) ? bt * expf(gt - sh.gam[ii]) * gr[ii] : 0.f;
+        }
+        arow[i / 4] = make_float4(a[0], a[1], a[2], a[3]);
+      }
+    } else {
+      float m2[64];
+#pragma unroll
+      for (int i = 0; i < 64; ++i)
+        m2[i] = (i < B && row < B) ? expf(gB - sh.gam[i]) * gr[i] : 0.f;
+      store_row_sw128(M2s, row, m2);
+    }
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+
+  // ---- T = (I + A)^{-1}: thread `col` solves (I + A) x = e_col by forward substitution
+  if (tid < 64) {
+    const int col = tid;
+    float x[64];
+#pragma unroll
+    for (int t = 0; t < 64; ++t) {
+      const float4* arow = reinterpret_cast<const float4*>(A32 + t * 64);
+      float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+#pragma unroll
+      for (int i4 = 0; i4 < t / 4; ++i4) {
+        const float4 a = arow[i4];
+        a0 = fmaf(a.x, x[4 * i4], a0);
+        a1 = fmaf(a.y, x[4 * i4 + 1], a1);
+        a2 = fmaf(a.z, x[4 * i4 + 2], a2);
+        a3 = fmaf(a.w, x[4 * i4 + 3], a3);
+      }
+#pragma unroll
+      for (int i = (t / 4) * 4; i < t; ++i) a0 = fmaf(A32[t * 64 + i], x[i], a0);
+      x[t] = (t == col ? 1.f : 0.f) - ((a0 + a1) + (a2 + a3));
+    }
+    // T[t][col] into the K-major tile (row t, column col)
+#pragma unroll
+    for (int t = 0; t < 64; ++t)
+      *reinterpret_cast<__nv_bfloat16*>(Ts + t * 128 + ((((col >> 3) ^ (t & 7))) << 4) +
+                                        ((col & 7) << 1)) = __float2bfloat16_rn(x[t]);
+  }
+  __syncthreads();  // A is dead from here on; its buffer becomes X^T
+
+  // ---- X^T[c][t] = beta_t (V[t][c] - Gam_t (K S0)[t][c])
+  {
+    const int c = tid;
+    float w[64];
+    tmem_ld64(tmW + lane_off, w);  // columns 0..63: (K S0)^T[c][t]
+    float xv[64];
+    const __nv_bfloat16* vcol =
+        static_cast<const __nv_bfloat16*>(p.v) + ((size_t)r * B * p.Hv + j) * DV + c;
+#pragma unroll
+    for (int t = 0; t < 64; ++t) {
+      const float vt = (c < DV && t < B) ? __bfloat162float(vcol[(size_t)t * p.Hv * DV]) : 0.f;
+      xv[t] = t < B ? sh.beta[t] * (vt - sh.Gam[t] * w[t]) : 0.f;
+    }
+    store_row_sw128(Xs, c, xv);
+  }
+  tc::fence_async_smem();
+  tc::fence_before_sync();
+  __syncthreads();
+
+  // ---- MMA 3: delta^T = X^T T^T
+  if (tid == 0) {
+    tc::fence_after_sync();
+    const uint32_t id = tc::idesc_bf16(128, Bp, false, false);
+    for (int kk = 0; kk < Bp / 16; ++kk) {
+      const uint64_t a = tc::sdesc_sw128(tc::smem_u32(Xs + kk * 32), 16, 1024);
+      const uint64_t b = tc::sdesc_sw128(tc::smem_u32(Ts + kk * 32), 16, 1024);
+      tc::mma_bf16_ss(tmA, a, b, id, kk > 0);
+    }
+    tc::mma_commit(&sh.bar_mma);
+  }
+  if (!lin_wait(&sh.bar_mma, 1, sh, p.dev_status)) goto done;
+  tc::fence_after_sync();
+  {
+    float d[64];
+    tmem_ld64(tmA + lane_off, d);
+#pragma unroll
+    for (int t = 0; t < 64; ++t) d[t] = t < B ? d[t] : 0.f;
+    store_row_sw128(Xs, tid, d);  // delta^T replaces X^T (MMA 3 has completed)
+  }
+  tc::fence_async_smem();
+  tc::fence_before_sync();
+  __syncthreads();
+
+  // ---- MMA 4: O2^T = delta^T M2^T
+  if (tid == 0) {
+    tc::fence_after_sync();
+    const uint32_t id = tc::idesc_bf16(128, Bp, false, false);
+    for (int kk = 0; kk < Bp / 16; ++kk) {
+      const uint64_t a = tc::sdesc_sw128(tc::smem_u32(Xs + kk * 32), 16, 1024);
+      const uint64_t b = tc::sdesc_sw128(tc::smem_u32(M2s + kk * 32), 16, 1024);
+      tc::mma_bf16_ss(tmA, a, b, id, kk > 0);
+    }
+    tc::mma_commit(&sh.bar_mma);
+  }
+  if (!lin_wait(&sh.bar_mma, 0, sh, p.dev_status)) goto done;
+  tc::fence_after_sync();
+  {
+    const int c = tid;
+    float o2[64], wq[64];
+    tmem_ld64(tmA + lane_off, o2);
+    tmem_ld64(tmW + lane_off + 64, wq);  // columns 64..127: (Q S0)^T[c][l]
+    const float GB = sh.Gam[B - 1];
+    if (c < DV) {
+      __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.out_blockend);
+#pragma unroll
+      for (int l = 0; l < 64; ++l)
+        if (l < B)
+          out[(((size_t)r * B + l) * p.Hv + j) * DV + c] =
+              __float2bfloat16_rn(p.scale * (GB * wq[l] + o2[l]));
+    }
+  }
+
+done:
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == 0) {
+    tc::fence_after_sync();
+    tc::tmem_dealloc(tmem, 256);
+  }
+}
+
+// ------------------------------------------------------------------ host side
+
+namespace {
+
+PFN_cuTensorMapEncodeTiled_v12000 lin_encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+  }
+  return fn;
+}
+
+bool lin_map(CUtensorMap* m, const void* ptr, int d, int H, int B, int R, bool swizzle) {
+  auto fn = lin_encode_fn();
+  if (!fn) return false;
+  cuuint64_t gd[4] = {(cuuint64_t)d, (cuuint64_t)H, (cuuint64_t)B, (cuuint64_t)R};
+  cuuint64_t gs[3] = {(cuuint64_t)d * 2, (cuuint64_t)H * d * 2, (cuuint64_t)B * H * d * 2};
+  cuuint32_t bx[4] = {64, 1, (cuuint32_t)kBmax, 1};
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(ptr), gd, gs, bx, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE,
+            swizzle ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+         CUDA_SUCCESS;
+}
+
+template <int DK, int DV>
+cudaError_t launch_lin_tc(const GdrParams& p, cudaStream_t stream) {
+  using C = LinCfg<DK, DV>;
+  LinMaps maps;
+  if (!lin_map(&maps.k, p.k, DK, p.Hk, p.B, p.R, true) ||
+      !lin_map(&maps.q, p.q, DK, p.Hk, p.B, p.R, true))
+    return cudaErrorInvalidValue;
+  const int smem = C::kSmem + 1024;
+  cudaError_t e = cudaFuncSetAttribute(gdr_denoise_tc_kernel<DK, DV>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  gdr_denoise_tc_kernel<DK, DV><<<p.R * p.Hv, kLinThreads, smem, stream>>>(maps, p);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+bool gdr_denoise_tc_supported(int B, int dk, int dv) {
+  return B >= 1 && B <= kBmax && (dk == 64 || dk == 128) && (dv == 64 || dv == 128);
+}
+
+cudaError_t launch_gdr_denoise_tc(const GdrParams& p, cudaStream_t stream) {
+  if (p.dk == 128 && p.dv == 128) return launch_lin_tc<128, 128>(p, stream);
+  if (p.dk == 128 && p.dv == 64) return launch_lin_tc<128, 64>(p, stream);
+  if (p.dk == 64 && p.dv == 128) return launch_lin_tc<64, 128>(p, stream);
+  if (p.dk == 64 && p.dv == 64) return launch_lin_tc<64, 64>(p, stream);
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace flare
