@@ -330,19 +330,21 @@ def run_flare(args, spec, rank, world, local_rank):
     ms_step = ms / args.steps
 
     # end-to-end through host buffers
-    e2e = E2ERunner(fr)
-    for _ in range(max(1, min(args.warmup, 2))):
-        e2e.step()
-    if dist:
-        tdist.barrier()
-    t_e = time.perf_counter()
-    for _ in range(args.steps):
-        e2e.step()
-    e2e_ms = (time.perf_counter() - t_e) * 1e3 / args.steps
-    if dist:
-        tt = torch.tensor([e2e_ms], dtype=torch.float64, device=device)
-        tdist.all_reduce(tt, op=tdist.ReduceOp.MAX)
-        e2e_ms = float(tt.item())
+    e2e, e2e_ms = None, None
+    if not args.no_e2e:
+        e2e = E2ERunner(fr)
+        for _ in range(max(1, min(args.warmup, 2))):
+            e2e.step()
+        if dist:
+            tdist.barrier()
+        t_e = time.perf_counter()
+        for _ in range(args.steps):
+            e2e.step()
+        e2e_ms = (time.perf_counter() - t_e) * 1e3 / args.steps
+        if dist:
+            tt = torch.tensor([e2e_ms], dtype=torch.float64, device=device)
+            tdist.all_reduce(tt, op=tdist.ReduceOp.MAX)
+            e2e_ms = float(tt.item())
     st, bits = flare.flare_read_status(fr.status)
     if st != flare.FLARE_OK:
         raise RuntimeError(f"device status {bits:#x} after timing")
@@ -394,8 +396,9 @@ def run_flare(args, spec, rank, world, local_rank):
         "achieved_hbm_gbs": step_bytes / (ms_step / 1e3) / 1e9,
         "per_call_ms": per,
         "roofline": roof,
-        "e2e": {"value": world * tokens / (e2e_ms / 1e3), "unit": UNIT, "ms_per_step": e2e_ms,
-                "h2d_bytes_per_step": e2e.h2d_bytes, "d2h_bytes_per_step": e2e.d2h_bytes},
+        "e2e": None if e2e is None else {
+            "value": world * tokens / (e2e_ms / 1e3), "unit": UNIT, "ms_per_step": e2e_ms,
+            "h2d_bytes_per_step": e2e.h2d_bytes, "d2h_bytes_per_step": e2e.d2h_bytes},
         "gpu_launches": int(launches),
         "clocks": clk,
     }
@@ -480,6 +483,8 @@ def main():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(workloads.WORKLOADS))
     ap.add_argument("--impl", default="flare", choices=["flare", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true",
+                    help="skip the host-buffer end-to-end measurement (profiling runs)")
     ap.add_argument("--cpu-sample-requests", type=int, default=2)
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "flare":

@@ -51,7 +51,7 @@ struct LinCfg {
 };
 
 struct LinShared {
-  uint64_t bar_kq, bar_mma;
+  uint64_t bar_kq, bar_v, bar_mma;
   uint32_t tmem_base;
   int abort_flag;
   float gam[kBmax];   // gamma_t
@@ -62,6 +62,7 @@ struct LinShared {
 struct LinMaps {
   CUtensorMap k;  // (dk, Hk, B, R)  box (64, 1, 64, 1), 128-byte swizzle
   CUtensorMap q;
+  CUtensorMap v;  // (dv, Hv, B, R)  box (64, 1, 64, 1), no swizzle
 };
 
 __device__ __forceinline__ bool lin_wait(uint64_t* bar, uint32_t parity, LinShared& sh,
@@ -131,6 +132,7 @@ __global__ void __launch_bounds__(kLinThreads, 2)
   if (tid == 0) {
     sh.abort_flag = 0;
     tc::mbar_init(&sh.bar_kq, 1);
+    tc::mbar_init(&sh.bar_v, 1);
     tc::mbar_init(&sh.bar_mma, 1);
     tc::fence_mbar_init();
   }
@@ -215,6 +217,12 @@ __global__ void __launch_bounds__(kLinThreads, 2)
   }
   if (!lin_wait(&sh.bar_mma, 0, sh, p.dev_status)) goto done;
   tc::fence_after_sync();
+  // the S0^T operand is dead: stage the V tile there while A, M2 and T are built
+  if (tid == 0) {
+    tc::mbar_expect_tx(&sh.bar_v, (DV / 64) * kBmax * 128);
+    for (int c = 0; c < DV / 64; ++c)
+      tc::tma_load_4d(S0s + c * (kBmax * 128), &maps.v, &sh.bar_v, c * 64, j, 0, r);
+  }
 
   // ---- A (rows 0..63 of G) and M2 (rows 64..127)
   {
@@ -279,13 +287,13 @@ __global__ void __launch_bounds__(kLinThreads, 2)
     const int c = tid;
     float w[64];
     tmem_ld64(tmW + lane_off, w);  // columns 0..63: (K S0)^T[c][t]
+    if (!lin_wait(&sh.bar_v, 0, sh, p.dev_status)) goto done;
     float xv[64];
-    const __nv_bfloat16* vcol =
-        static_cast<const __nv_bfloat16*>(p.v) + ((size_t)r * B * p.Hv + j) * DV + c;
+    const uint8_t* vcol = S0s + ((c & (DV - 1)) >> 6) * (kBmax * 128) + (c & 63) * 2;
 #pragma unroll
     for (int t = 0; t < 64; ++t) {
-      const float vt = (c < DV && t < B) ? __bfloat162float(vcol[(size_t)t * p.Hv * DV]) : 0.f;
-      xv[t] = t < B ? sh.beta[t] * (vt - sh.Gam[t] * w[t]) : 0.f;
+      const float vt = __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(vcol + t * 128));
+      xv[t] = (t < B && c < DV) ? sh.beta[t] * (vt - sh.Gam[t] * w[t]) : 0.f;
     }
     store_row_sw128(Xs, c, xv);
   }
@@ -391,7 +399,8 @@ cudaError_t launch_lin_tc(const GdrParams& p, cudaStream_t stream) {
   using C = LinCfg<DK, DV>;
   LinMaps maps;
   if (!lin_map(&maps.k, p.k, DK, p.Hk, p.B, p.R, true) ||
-      !lin_map(&maps.q, p.q, DK, p.Hk, p.B, p.R, true))
+      !lin_map(&maps.q, p.q, DK, p.Hk, p.B, p.R, true) ||
+      !lin_map(&maps.v, p.v, DV, p.Hv, p.B, p.R, false))
     return cudaErrorInvalidValue;
   const int smem = C::kSmem + 1024;
   cudaError_t e = cudaFuncSetAttribute(gdr_denoise_tc_kernel<DK, DV>,
