@@ -191,6 +191,39 @@ flare_status flare_block_softmax_attn(const flare_softmax_desc* desc, const void
                                       void* workspace, size_t workspace_bytes,
                                       int32_t* dev_status, void* stream);
 
+/* Size of the library-owned scratch array used by flare_block_softmax_attn_noalloc. */
+#define FLARE_NOALLOC_SCRATCH_BYTES (64u * 1024u * 1024u)
+
+/*
+ * flare_block_softmax_attn for callers that cannot allocate device memory.
+ * The paper has no counterpart; this is a deployment convenience.
+ * Some callers cannot supply a workspace: a serving engine whose memory
+ * manager owns all device memory and forbids cudaMalloc/cudaFree while
+ * requests are in flight (they synchronize the device and can fail under
+ * memory pressure), or a plugin host that passes only the request's own
+ * tensors.  Same arguments, layouts, outputs and status bits as
+ * flare_block_softmax_attn, minus the workspace: the split partials live in a
+ * file-scope device array of FLARE_NOALLOC_SCRATCH_BYTES that the library
+ * holds on every GPU that loads it, until the process exits.
+ *  - This call allocates nothing (no cudaMalloc, cudaFree or allocating
+ *    library routine).
+ *  - The first call on each device looks up the array's device address
+ *    (cudaGetSymbolAddress, current device); make that first call before any
+ *    stream capture.
+ *  - If the shape needs more scratch than FLARE_NOALLOC_SCRATCH_BYTES
+ *    (flare_softmax_workspace_size reports the need), the call returns
+ *    FLARE_ERR_UNSUPPORTED and launches nothing.
+ *  - Every call shares the one array: calls that overlap on the GPU (other
+ *    streams, other host threads) race on it and must be serialized by the
+ *    caller.  No part of it needs to start at zero.
+ */
+flare_status flare_block_softmax_attn_noalloc(const flare_softmax_desc* desc, const void* q,
+                                              const void* k_blk, const void* v_blk,
+                                              const void* k_pool, const void* v_pool,
+                                              const int32_t* page_table,
+                                              const int32_t* prefix_len, void* out, float* lse,
+                                              int32_t* dev_status, void* stream);
+
 /*
  * Test/debug helper: dense copy of request `request`'s paged prefix,
  * k_out/v_out [prefix_len[request], Hkv, D] act_dtype (the caller sizes them
