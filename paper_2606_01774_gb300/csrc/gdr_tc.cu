@@ -54,7 +54,7 @@ struct LinShared {
   uint64_t bar_kq, bar_v, bar_mma;
   uint32_t tmem_base;
   int abort_flag;
-  float gam[kBmax];   // gamma_t
+  float gam2[kBmax];  // gamma_t * log2(e)
   float Gam[kBmax];   // exp(gamma_t)
   float beta[kBmax];
 };
@@ -76,27 +76,19 @@ __device__ __forceinline__ bool lin_wait(uint64_t* bar, uint32_t parity, LinShar
   return all;
 }
 
-__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float (&v)[64]) {
-  uint32_t r[64];
-#pragma unroll
-  for (int c = 0; c < 64; c += 16) tc::tmem_ld16(taddr + c, *reinterpret_cast<uint32_t(*)[16]>(&r[c]));
-  tc::tmem_ld_wait();
-#pragma unroll
-  for (int i = 0; i < 64; ++i) v[i] = __uint_as_float(r[i]);
-}
-
-// 64 bf16 values as one 128-byte row of a K-major SW128 tile.
-__device__ __forceinline__ void store_row_sw128(uint8_t* tile, int row, const float (&v)[64]) {
+// 16 bf16 values (columns c0..c0+15) into row `row` of a K-major SW128 tile.
+__device__ __forceinline__ void store16_sw128(uint8_t* tile, int row, int c0, const float (&v)[16]) {
   uint8_t* p = tile + row * 128;
 #pragma unroll
-  for (int c16 = 0; c16 < 8; ++c16) {
+  for (int h = 0; h < 2; ++h) {
     uint32_t w[4];
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
-      __nv_bfloat162 h = __floats2bfloat162_rn(v[c16 * 8 + 2 * e], v[c16 * 8 + 2 * e + 1]);
-      w[e] = *reinterpret_cast<uint32_t*>(&h);
+      __nv_bfloat162 b = __floats2bfloat162_rn(v[8 * h + 2 * e], v[8 * h + 2 * e + 1]);
+      w[e] = *reinterpret_cast<uint32_t*>(&b);
     }
-    *reinterpret_cast<uint4*>(p + ((c16 ^ (row & 7)) * 16)) = make_uint4(w[0], w[1], w[2], w[3]);
+    const int g = (c0 >> 3) + h;
+    *reinterpret_cast<uint4*>(p + ((g ^ (row & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
   }
 }
 
@@ -114,7 +106,9 @@ __global__ void __launch_bounds__(kLinThreads, 2)
   uint8_t* M2s = S0s + C::kS0;
   uint8_t* Ts = M2s + C::kM2;
   uint8_t* Xs = Ts + C::kT;
-  float* A32 = reinterpret_cast<float*>(Xs);  // aliases X^T (A is dead before X is written)
+  float* A32 = reinterpret_cast<float*>(Xs);   // aliases X^T (A is dead before X is written)
+  float* T32 = reinterpret_cast<float*>(KQs);  // fp32 T, in [K;Q] once MMA 1/2 have run
+  float* Ytmp = reinterpret_cast<float*>(Ts);  // 3 x 256 floats, dead until T is converted
 
   const int item = blockIdx.x;
   const int r = item / p.Hv, j = item % p.Hv;
@@ -190,8 +184,8 @@ __global__ void __launch_bounds__(kLinThreads, 2)
       }
     }
     g1 += __shfl_sync(0xffffffffu, g0, 31);
-    sh.gam[lane] = g0;
-    sh.gam[lane + 32] = g1;
+    sh.gam2[lane] = g0 * 1.4426950408889634f;
+    sh.gam2[lane + 32] = g1 * 1.4426950408889634f;
     sh.Gam[lane] = expf(g0);
     sh.Gam[lane + 32] = expf(g1);
     sh.beta[lane] = lane < B ? p.beta[gb + (size_t)lane * p.Hv] : 0.f;
@@ -224,78 +218,124 @@ __global__ void __launch_bounds__(kLinThreads, 2)
       tc::tma_load_4d(S0s + c * (kBmax * 128), &maps.v, &sh.bar_v, c * 64, j, 0, r);
   }
 
-  // ---- A (rows 0..63 of G) and M2 (rows 64..127)
+  // ---- A (rows 0..63 of G) and M2 (rows 64..127), 16 columns at a time
   {
-    float gr[64];
-    tmem_ld64(tmA + lane_off, gr);
     const int row = tid & 63;
-    const float gB = sh.gam[B - 1];
-    if (tid < 64) {
-      const float bt = sh.beta[row], gt = sh.gam[row];
-      float4* arow = reinterpret_cast<float4*>(A32 + row * 64);
+    const float gB = sh.gam2[B - 1];
+    const float bt = sh.beta[row], gt = sh.gam2[row];
+#pragma unroll 1
+    for (int c0 = 0; c0 < 64; c0 += 16) {
+      uint32_t gr[16];
+      tc::tmem_ld16(tmA + lane_off + c0, gr);
+      tc::tmem_ld_wait();
+      float v[16];
+      if (tid < 64) {
 #pragma unroll
-      for (int i = 0; i < 64; i += 4) {
-        float a[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int ii = i + e;
-          a[e] = (ii < row && row < B) ? bt * expf(gt - sh.gam[ii]) * gr[ii] : 0.f;
+        for (int e = 0; e < 16; ++e) {
+          const int i = c0 + e;
+          v[e] = (i < row && row < B) ? bt * tc::ex2(gt - sh.gam2[i]) * __uint_as_float(gr[e]) : 0.f;
         }
-        arow[i / 4] = make_float4(a[0], a[1], a[2], a[3]);
-      }
-    } else {
-      float m2[64];
+        float4* arow = reinterpret_cast<float4*>(A32 + row * 64 + c0);
 #pragma unroll
-      for (int i = 0; i < 64; ++i)
-        m2[i] = (i < B && row < B) ? expf(gB - sh.gam[i]) * gr[i] : 0.f;
-      store_row_sw128(M2s, row, m2);
+        for (int q4 = 0; q4 < 4; ++q4)
+          arow[q4] = make_float4(v[4 * q4], v[4 * q4 + 1], v[4 * q4 + 2], v[4 * q4 + 3]);
+      } else {
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+          const int i = c0 + e;
+          v[e] = (i < B && row < B) ? tc::ex2(gB - sh.gam2[i]) * __uint_as_float(gr[e]) : 0.f;
+        }
+        store16_sw128(M2s, row, c0, v);
+      }
     }
+  }
+  // T32 (fp32 [64][64], in the dead [K;Q] operand) starts at zero
+  {
+    float4* t4 = reinterpret_cast<float4*>(T32);
+#pragma unroll
+    for (int n = 0; n < 64 * 64 / 4 / kLinThreads; ++n)
+      t4[tid + n * kLinThreads] = make_float4(0.f, 0.f, 0.f, 0.f);
   }
   tc::fence_before_sync();
   __syncthreads();
 
-  // ---- T = (I + A)^{-1}: thread `col` solves (I + A) x = e_col by forward substitution
+  // ---- T = (I + A)^{-1}, blocked by 16 (A is strictly lower triangular).
+  // Diagonal blocks: thread (blk, col) solves (I + A_kk) x = e_col in registers.
   if (tid < 64) {
-    const int col = tid;
-    float x[64];
+    const int blk = tid >> 4, col = tid & 15, o = blk * 16;
+    float x[16];
 #pragma unroll
-    for (int t = 0; t < 64; ++t) {
-      const float4* arow = reinterpret_cast<const float4*>(A32 + t * 64);
-      float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+    for (int t = 0; t < 16; ++t) {
+      float acc = (t == col) ? 1.f : 0.f;
 #pragma unroll
-      for (int i4 = 0; i4 < t / 4; ++i4) {
-        const float4 a = arow[i4];
-        a0 = fmaf(a.x, x[4 * i4], a0);
-        a1 = fmaf(a.y, x[4 * i4 + 1], a1);
-        a2 = fmaf(a.z, x[4 * i4 + 2], a2);
-        a3 = fmaf(a.w, x[4 * i4 + 3], a3);
-      }
-#pragma unroll
-      for (int i = (t / 4) * 4; i < t; ++i) a0 = fmaf(A32[t * 64 + i], x[i], a0);
-      x[t] = (t == col ? 1.f : 0.f) - ((a0 + a1) + (a2 + a3));
+      for (int i = 0; i < t; ++i) acc = fmaf(-A32[(o + t) * 64 + o + i], x[i], acc);
+      x[t] = acc;
     }
-    // T[t][col] into the K-major tile (row t, column col)
 #pragma unroll
-    for (int t = 0; t < 64; ++t)
-      *reinterpret_cast<__nv_bfloat16*>(Ts + t * 128 + ((((col >> 3) ^ (t & 7))) << 4) +
-                                        ((col & 7) << 1)) = __float2bfloat16_rn(x[t]);
+    for (int t = 0; t < 16; ++t) T32[(o + t) * 64 + o + col] = x[t];
+  }
+  __syncthreads();
+  // Off-diagonal blocks by distance d = i - j:  T_ij = -T_ii sum_{k=j}^{i-1} A_ik T_kj
+#pragma unroll 1
+  for (int d = 1; d < 4; ++d) {
+    const int nel = (4 - d) * 256;
+#pragma unroll 1
+    for (int e = tid; e < nel; e += kLinThreads) {
+      const int bj = e >> 8, rr = (e >> 4) & 15, cc = e & 15, bi = bj + d;
+      const float* arow = A32 + (16 * bi + rr) * 64;
+      const float* tcol = T32 + 16 * bj + cc;
+      float a0 = 0.f, a1 = 0.f;
+#pragma unroll 4
+      for (int k = 16 * bj; k < 16 * bi; k += 2) {
+        a0 = fmaf(arow[k], tcol[k * 64], a0);
+        a1 = fmaf(arow[k + 1], tcol[(k + 1) * 64], a1);
+      }
+      Ytmp[e] = a0 + a1;
+    }
+    __syncthreads();
+#pragma unroll 1
+    for (int e = tid; e < nel; e += kLinThreads) {
+      const int bj = e >> 8, rr = (e >> 4) & 15, cc = e & 15, bi = bj + d;
+      const float* trow = T32 + (16 * bi + rr) * 64 + 16 * bi;
+      float acc = 0.f;
+#pragma unroll 4
+      for (int u = 0; u <= rr; ++u) acc = fmaf(trow[u], Ytmp[bj * 256 + u * 16 + cc], acc);
+      T32[(16 * bi + rr) * 64 + 16 * bj + cc] = -acc;
+    }
+    __syncthreads();
+  }
+  // T (bf16) into the K-major operand tile, one row per thread
+  if (tid < 64) {
+#pragma unroll 1
+    for (int c0 = 0; c0 < 64; c0 += 16) {
+      float v[16];
+#pragma unroll
+      for (int e = 0; e < 16; ++e) v[e] = T32[tid * 64 + c0 + e];
+      store16_sw128(Ts, tid, c0, v);
+    }
   }
   __syncthreads();  // A is dead from here on; its buffer becomes X^T
 
   // ---- X^T[c][t] = beta_t (V[t][c] - Gam_t (K S0)[t][c])
   {
     const int c = tid;
-    float w[64];
-    tmem_ld64(tmW + lane_off, w);  // columns 0..63: (K S0)^T[c][t]
     if (!lin_wait(&sh.bar_v, 0, sh, p.dev_status)) goto done;
-    float xv[64];
     const uint8_t* vcol = S0s + ((c & (DV - 1)) >> 6) * (kBmax * 128) + (c & 63) * 2;
+#pragma unroll 1
+    for (int c0 = 0; c0 < 64; c0 += 16) {
+      uint32_t w[16];
+      tc::tmem_ld16(tmW + lane_off + c0, w);  // (K S0)^T[c][t]
+      tc::tmem_ld_wait();
+      float xv[16];
 #pragma unroll
-    for (int t = 0; t < 64; ++t) {
-      const float vt = __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(vcol + t * 128));
-      xv[t] = (t < B && c < DV) ? sh.beta[t] * (vt - sh.Gam[t] * w[t]) : 0.f;
+      for (int e = 0; e < 16; ++e) {
+        const int t = c0 + e;
+        const float vt =
+            __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(vcol + t * 128));
+        xv[e] = (t < B && c < DV) ? sh.beta[t] * (vt - sh.Gam[t] * __uint_as_float(w[e])) : 0.f;
+      }
+      store16_sw128(Xs, c, c0, xv);
     }
-    store_row_sw128(Xs, c, xv);
   }
   tc::fence_async_smem();
   tc::fence_before_sync();
@@ -314,12 +354,15 @@ __global__ void __launch_bounds__(kLinThreads, 2)
   }
   if (!lin_wait(&sh.bar_mma, 1, sh, p.dev_status)) goto done;
   tc::fence_after_sync();
-  {
-    float d[64];
-    tmem_ld64(tmA + lane_off, d);
+#pragma unroll 1
+  for (int c0 = 0; c0 < 64; c0 += 16) {
+    uint32_t dd[16];
+    tc::tmem_ld16(tmA + lane_off + c0, dd);
+    tc::tmem_ld_wait();
+    float v[16];
 #pragma unroll
-    for (int t = 0; t < 64; ++t) d[t] = t < B ? d[t] : 0.f;
-    store_row_sw128(Xs, tid, d);  // delta^T replaces X^T (MMA 3 has completed)
+    for (int e = 0; e < 16; ++e) v[e] = (c0 + e < B) ? __uint_as_float(dd[e]) : 0.f;
+    store16_sw128(Xs, tid, c0, v);  // delta^T replaces X^T (MMA 3 has completed)
   }
   tc::fence_async_smem();
   tc::fence_before_sync();
@@ -340,17 +383,24 @@ __global__ void __launch_bounds__(kLinThreads, 2)
   tc::fence_after_sync();
   {
     const int c = tid;
-    float o2[64], wq[64];
-    tmem_ld64(tmA + lane_off, o2);
-    tmem_ld64(tmW + lane_off + 64, wq);  // columns 64..127: (Q S0)^T[c][l]
     const float GB = sh.Gam[B - 1];
-    if (c < DV) {
-      __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.out_blockend);
+    __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.out_blockend) +
+                         ((size_t)r * B * p.Hv + j) * DV + c;
+#pragma unroll 1
+    for (int c0 = 0; c0 < 64; c0 += 16) {
+      uint32_t o2[16], wq[16];
+      tc::tmem_ld16(tmA + lane_off + c0, o2);
+      tc::tmem_ld16(tmW + lane_off + 64 + c0, wq);  // (Q S0)^T[c][l]
+      tc::tmem_ld_wait();
+      if (c < DV) {
 #pragma unroll
-      for (int l = 0; l < 64; ++l)
-        if (l < B)
-          out[(((size_t)r * B + l) * p.Hv + j) * DV + c] =
-              __float2bfloat16_rn(p.scale * (GB * wq[l] + o2[l]));
+        for (int e = 0; e < 16; ++e) {
+          const int l = c0 + e;
+          if (l < B)
+            out[(size_t)l * p.Hv * DV] = __float2bfloat16_rn(
+                p.scale * (GB * __uint_as_float(wq[e]) + __uint_as_float(o2[e])));
+        }
+      }
     }
   }
 
