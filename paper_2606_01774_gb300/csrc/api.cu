@@ -227,8 +227,8 @@ flare_status flare_commit_state(const flare_linear_desc* d, const void* q, const
   p.out_causal = causal_out;
   p.write_state = 1;
   p.dev_status = dev_status;
-  const cudaError_t e = launch_gdr_recurrent(p, d->act_dtype == FLARE_DT_BF16,
-                                             static_cast<cudaStream_t>(stream));
+  const cudaError_t e = launch_gdr_commit(p, d->act_dtype == FLARE_DT_BF16,
+                                          static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? FLARE_OK : FLARE_ERR_CUDA;
 }
 

@@ -61,6 +61,7 @@ struct SoftmaxPlan {
 
 size_t gdr_recurrent_smem_bytes(int dk, int dv, int threads);
 bool gdr_denoise_tc_supported(int B, int dk, int dv);
+cudaError_t launch_gdr_commit(const GdrParams& p, bool bf16, cudaStream_t stream);
 cudaError_t launch_gdr_denoise_tc(const GdrParams& p, cudaStream_t stream);
 cudaError_t launch_gdr_recurrent(const GdrParams& p, bool bf16, cudaStream_t stream);
 
