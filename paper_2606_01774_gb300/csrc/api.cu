@@ -38,6 +38,7 @@ flare_status check_softmax(const flare_softmax_desc* d) {
     return FLARE_ERR_INVALID_ARGUMENT;
   if (d->mask_mode != FLARE_MASK_BLOCK_BIDIR && d->mask_mode != FLARE_MASK_BLOCK_CAUSAL)
     return FLARE_ERR_INVALID_ARGUMENT;
+  if (!(d->scale >= 0.f) || !(d->scale < 3.0e38f)) return FLARE_ERR_INVALID_ARGUMENT;
   if (d->num_q_heads % d->num_kv_heads != 0) return FLARE_ERR_INVALID_ARGUMENT;
   if (d->block_len > 64) return FLARE_ERR_UNSUPPORTED;
   if (d->head_dim != 64 && d->head_dim != 128 && d->head_dim != 256) return FLARE_ERR_UNSUPPORTED;

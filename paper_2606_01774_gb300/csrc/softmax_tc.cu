@@ -11,18 +11,19 @@
 // every prefix token; the mask only touches the ragged prefix end and the
 // block tile (bidirectional, or token-causal for the state-update pass).
 //
-// Warp roles (192 threads):
+// Warp roles (320 threads):
 //   warp 0     TMA producer: Q once, then K and V tiles (one TMA box per page
 //              and 64-column chunk, 128-byte swizzle) into a ring of stages.
 //   warp 1     tensor-memory owner and MMA issuer: S = Q K^T into one of two
 //              TMEM buffers, then O += P V with P from shared memory; zeroes
 //              the V rows past the prefix end so poisoned cache rows never
 //              meet a zero probability (0 * NaN).
-//   warps 2-5  softmax: one query row per thread (its TMEM lane), online
-//              base-2 softmax with a lazily moved running max (O in TMEM is
-//              rescaled only when the max grows by more than 2^8), P written
-//              as bf16 in the swizzled layout the MMA reads; epilogue divides
-//              by the row sum and stores the output (or a split partial).
+//   warps 2-9  softmax: two warps per TMEM lane quarter, each thread one
+//              query row and half of the tile's key columns; online base-2
+//              softmax with a lazily moved running max (O in TMEM is rescaled
+//              only when the max grows by more than 2^8), P written as bf16 in
+//              the swizzled layout the MMA reads; epilogue divides by the row
+//              sum and stores the output (or a split partial).
 // Every wait is bounded (tc::mbar_wait); a timeout sets FLARE_DEV_WAIT_TIMEOUT,
 // the CTA stops issuing work, writes nothing, frees its TMEM and exits.
 #include <cudaTypedefs.h>
@@ -37,7 +38,7 @@ namespace {
 
 constexpr int kTileN = 64;     // keys per tile
 constexpr int kRowsM = 128;    // query rows per CTA (TMEM lanes)
-constexpr int kThreadsTC = 192;
+constexpr int kThreadsTC = 320;  // producer warp, MMA warp, 8 softmax warps
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 
 struct TcMaps {
@@ -65,6 +66,9 @@ struct TcShared {
   uint64_t k_full[4], v_full[4], k_empty[4], v_empty[4];
   uint64_t s_full[2], s_empty[2], p_full[2], p_empty[2];
   uint64_t o_final;
+  uint64_t xbar[4];     // row-pair exchange written, one per TMEM lane quarter (64 arrivals)
+  uint64_t xread[4];    // row-pair exchange read (64 arrivals)
+  float xch[256];       // [half][128 rows]
   uint32_t tmem_base;
   int abort_flag;
 };
@@ -141,11 +145,15 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     }
     for (int b = 0; b < 2; ++b) {
       tc::mbar_init(&sh.s_full[b], 1);
-      tc::mbar_init(&sh.s_empty[b], 128);
-      tc::mbar_init(&sh.p_full[b], 128);
+      tc::mbar_init(&sh.s_empty[b], 256);
+      tc::mbar_init(&sh.p_full[b], 256);
       tc::mbar_init(&sh.p_empty[b], 1);
     }
     tc::mbar_init(&sh.o_final, 1);
+    for (int q = 0; q < 4; ++q) {
+      tc::mbar_init(&sh.xbar[q], 64);
+      tc::mbar_init(&sh.xread[q], 64);
+    }
     tc::fence_mbar_init();
   }
   if (warp == 1) tc::tmem_alloc(&sh.tmem_base, C::kTmemCols);
@@ -184,41 +192,44 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         tc::tma_load_4d(Qs + c * (kRowsM * 128), &maps.q, &sh.q_full, c * 64, kvh * p.G,
                         mtile * Bt, r);
       const int box_rows = p.page_size < kTileN ? p.page_size : kTileN;
-      for (int j = 0; j < n_tiles && !aborted(sh); ++j) {
+      // one K or V tile into its ring slot (waits for the slot to be free)
+      auto load = [&](int j, int kv) -> bool {
         const int st = j % C::kStages;
         const uint32_t ph = (uint32_t)(j / C::kStages) & 1u;
+        uint64_t* empty = kv ? &sh.v_empty[st] : &sh.k_empty[st];
+        uint64_t* full = kv ? &sh.v_full[st] : &sh.k_full[st];
+        uint8_t* dst = (kv ? Vs : Ks) + st * C::kKVBytes;
+        if (!tc::mbar_wait(empty, ph ^ 1u, &sh.abort_flag)) return false;
         int pt;
-        const bool blk = tile_kind(j, pt);
-        for (int kv = 0; kv < 2; ++kv) {
-          uint64_t* empty = kv ? &sh.v_empty[st] : &sh.k_empty[st];
-          uint64_t* full = kv ? &sh.v_full[st] : &sh.k_full[st];
-          uint8_t* dst = (kv ? Vs : Ks) + st * C::kKVBytes;
-          if (!tc::mbar_wait(empty, ph ^ 1u, &sh.abort_flag)) {
-            set_abort(sh, p.dev_status);
-            break;
-          }
-          if (blk) {
-            tc::mbar_expect_tx(full, C::kKVBytes);
-            const CUtensorMap* m = kv ? &maps.vblk : &maps.kblk;
+        if (tile_kind(j, pt)) {
+          tc::mbar_expect_tx(full, C::kKVBytes);
+          const CUtensorMap* m = kv ? &maps.vblk : &maps.kblk;
+          for (int c = 0; c < C::kChunks; ++c)
+            tc::tma_load_4d(dst + c * (kTileN * 128), m, full, c * 64, kvh, 0, r);
+        } else {
+          const int tok0 = pt * kTileN;
+          const int valid = min(kTileN, P - tok0);
+          const int nbox = (valid + box_rows - 1) / box_rows;
+          tc::mbar_expect_tx(full, (uint32_t)(C::kChunks * nbox * box_rows * 128));
+          const CUtensorMap* m = kv ? &maps.vpool : &maps.kpool;
+          for (int b = 0; b < nbox; ++b) {
+            const int tok = tok0 + b * box_rows;
+            const int page = p.page_table[(size_t)r * p.max_pages + tok / p.page_size];
+            const int row0 = tok % p.page_size;
             for (int c = 0; c < C::kChunks; ++c)
-              tc::tma_load_4d(dst + c * (kTileN * 128), m, full, c * 64, kvh, 0, r);
-          } else {
-            const int tok0 = pt * kTileN;
-            const int valid = min(kTileN, P - tok0);
-            const int nbox = (valid + box_rows - 1) / box_rows;
-            tc::mbar_expect_tx(full, (uint32_t)(C::kChunks * nbox * box_rows * 128));
-            const CUtensorMap* m = kv ? &maps.vpool : &maps.kpool;
-            for (int b = 0; b < nbox; ++b) {
-              const int tok = tok0 + b * box_rows;
-              const int page = p.page_table[(size_t)r * p.max_pages + tok / p.page_size];
-              const int row0 = tok % p.page_size;
-              for (int c = 0; c < C::kChunks; ++c)
-                tc::tma_load_4d(dst + c * (kTileN * 128) + b * box_rows * 128, m, full, c * 64,
-                                row0, kvh, page);
-            }
+              tc::tma_load_4d(dst + c * (kTileN * 128) + b * box_rows * 128, m, full, c * 64,
+                              row0, kvh, page);
           }
         }
+        return true;
+      };
+      // consumption order of the MMA warp: K0, K1, V0, K2, V1, ...
+      bool ok = load(0, 0);
+      for (int j = 0; j < n_tiles && ok && !aborted(sh); ++j) {
+        if (j + 1 < n_tiles) ok = load(j + 1, 0);
+        if (ok) ok = load(j, 1);
       }
+      if (!ok) set_abort(sh, p.dev_status);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
@@ -287,12 +298,17 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     if (!ok && lane == 0) set_abort(sh, p.dev_status);
   } else {
     // ------------------------------------------------------------ softmax warps
-    const int quarter = warp & 3;  // TMEM lanes this warp may access
+    // Eight warps: warp w reads TMEM lanes 32*(w%4).. (its 32 rows) and key
+    // columns 32*half.. of each tile; the two warps of a row pair exchange
+    // their tile maxima through shared memory every tile.
+    const int quarter = warp & 3;
+    const int half = (warp - 2) >> 2;
     const int row = quarter * 32 + lane;
     const int m = mtile * kRowsM + row;
     const int trow = m / p.G;
     const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
-    float m_run = -INFINITY, l_run = 0.f;
+    constexpr int kDh = D / 2;  // output columns this half rescales / stores
+    float m_run = -INFINITY, l_run = 0.f;  // l_run: this half's share of the row sum
     bool ok = true;
     for (int j = 0; j < n_tiles; ++j) {
       const int sb = j & 1;
@@ -301,10 +317,11 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         break;
       }
       tc::fence_after_sync();
-      uint32_t sr[kTileN];
-#pragma unroll
-      for (int c = 0; c < kTileN; c += 16)
-        tc::tmem_ld16(tmem_s + lane_off + sb * kTileN + c, *reinterpret_cast<uint32_t(*)[16]>(&sr[c]));
+      uint32_t sr[32];
+      tc::tmem_ld16(tmem_s + lane_off + sb * kTileN + 32 * half,
+                    *reinterpret_cast<uint32_t(*)[16]>(&sr[0]));
+      tc::tmem_ld16(tmem_s + lane_off + sb * kTileN + 32 * half + 16,
+                    *reinterpret_cast<uint32_t(*)[16]>(&sr[16]));
       tc::tmem_ld_wait();
       tc::fence_before_sync();
       tc::mbar_arrive(&sh.s_empty[sb]);
@@ -312,28 +329,56 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
       int pt;
       const bool blk = tile_kind(j, pt);
       const int valid = tile_valid(j);
-      const int lim = (blk && p.causal) ? min(valid, trow + 1) : valid;
-      float x[kTileN];
+      const bool full = !blk && valid == kTileN;  // prefix tile: no mask at all
+      const int lim = full ? kTileN : ((blk && p.causal) ? min(valid, trow + 1) : valid);
+      // tile maximum of the raw scores (scale >= 0 keeps the order)
       float mt = -INFINITY;
 #pragma unroll
-      for (int c = 0; c < kTileN; ++c) {
-        x[c] = c < lim ? __uint_as_float(sr[c]) * p.scale_log2 : -INFINITY;
-        mt = fmaxf(mt, x[c]);
+      for (int c = 0; c < 32; ++c)
+        if (full || 32 * half + c < lim) mt = fmaxf(mt, __uint_as_float(sr[c]));
+      // the partner has read this slot's previous value before it is overwritten
+      if (j >= 1 && !warp_wait(&sh.xread[quarter], (uint32_t)(j - 1) & 1u, &sh.abort_flag)) {
+        ok = false;
+        break;
       }
-      const float m_new = fmaxf(m_run, mt);
+      sh.xch[half * 128 + row] = mt;
+      tc::mbar_arrive(&sh.xbar[quarter]);
+      if (!warp_wait(&sh.xbar[quarter], (uint32_t)j & 1u, &sh.abort_flag)) {
+        ok = false;
+        break;
+      }
+      mt = fmaxf(mt, sh.xch[(1 - half) * 128 + row]);
+      tc::mbar_arrive(&sh.xread[quarter]);
+      const float m_new = fmaxf(m_run, mt * p.scale_log2);
       const bool need = (j == 0) || (m_new > m_run + kRescaleThreshold);
       const bool warp_rescale = __any_sync(0xffffffffu, need);
       float m_use = m_run;
       if (warp_rescale) m_use = (j == 0 || m_new > m_run) ? m_new : m_run;
       const float corr = (j == 0) ? 0.f : tc::ex2(m_run - m_use);
+      const float neg_m = -m_use;
       float sum = 0.f;
-      uint32_t pk[kTileN / 2];
+      uint32_t pk[16];
+      if (full) {
 #pragma unroll
-      for (int c = 0; c < kTileN; c += 2) {
-        const float p0 = tc::ex2(x[c] - m_use), p1 = tc::ex2(x[c + 1] - m_use);
-        sum += p0 + p1;
-        __nv_bfloat162 h = __floats2bfloat162_rn(p0, p1);
-        pk[c / 2] = *reinterpret_cast<uint32_t*>(&h);
+        for (int c = 0; c < 32; c += 2) {
+          const float p0 = tc::ex2(fmaf(__uint_as_float(sr[c]), p.scale_log2, neg_m));
+          const float p1 = tc::ex2(fmaf(__uint_as_float(sr[c + 1]), p.scale_log2, neg_m));
+          sum += p0 + p1;
+          __nv_bfloat162 h2 = __floats2bfloat162_rn(p0, p1);
+          pk[c / 2] = *reinterpret_cast<uint32_t*>(&h2);
+        }
+      } else {
+#pragma unroll
+        for (int c = 0; c < 32; c += 2) {
+          const int col = 32 * half + c;
+          const float p0 =
+              col < lim ? tc::ex2(fmaf(__uint_as_float(sr[c]), p.scale_log2, neg_m)) : 0.f;
+          const float p1 =
+              col + 1 < lim ? tc::ex2(fmaf(__uint_as_float(sr[c + 1]), p.scale_log2, neg_m)) : 0.f;
+          sum += p0 + p1;
+          __nv_bfloat162 h2 = __floats2bfloat162_rn(p0, p1);
+          pk[c / 2] = *reinterpret_cast<uint32_t*>(&h2);
+        }
       }
       l_run = (j == 0) ? sum : l_run * corr + sum;
       // P buffer free once the P.V of tile j-2 has completed
@@ -341,7 +386,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         ok = false;
         break;
       }
-      // rescale O in TMEM when the running max moved (needs P.V of tile j-1 done)
+      // rescale this half's O columns when the running max moved (P.V of tile j-1 done)
       if (warp_rescale && j >= 1) {
         const int pb = (j - 1) & 1;
         if (!warp_wait(&sh.p_empty[pb], (uint32_t)((j - 1) >> 1) & 1u, &sh.abort_flag)) {
@@ -350,7 +395,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         }
         tc::fence_after_sync();
 #pragma unroll 1
-        for (int c = 0; c < D; c += 16) {
+        for (int c = half * kDh; c < (half + 1) * kDh; c += 16) {
           uint32_t o[16];
           tc::tmem_ld16(tmem_o + lane_off + c, o);
           tc::tmem_ld_wait();
@@ -369,14 +414,23 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
       m_run = m_use;
       uint8_t* prow = Ps + sb * C::kPBytes + row * 128;
 #pragma unroll
-      for (int c16 = 0; c16 < 8; ++c16) {
-        const int sw = c16 ^ (row & 7);
+      for (int q = 0; q < 4; ++q) {
+        const int sw = (4 * half + q) ^ (row & 7);
         *reinterpret_cast<uint4*>(prow + sw * 16) =
-            make_uint4(pk[c16 * 4], pk[c16 * 4 + 1], pk[c16 * 4 + 2], pk[c16 * 4 + 3]);
+            make_uint4(pk[q * 4], pk[q * 4 + 1], pk[q * 4 + 2], pk[q * 4 + 3]);
       }
       tc::fence_async_smem();
       tc::fence_before_sync();
       tc::mbar_arrive(&sh.p_full[sb]);
+    }
+    // row sum = the two halves' shares
+    if (ok && !warp_wait(&sh.xread[quarter], (uint32_t)(n_tiles - 1) & 1u, &sh.abort_flag))
+      ok = false;
+    if (ok) {
+      sh.xch[half * 128 + row] = l_run;
+      tc::mbar_arrive(&sh.xbar[quarter]);
+      if (!warp_wait(&sh.xbar[quarter], (uint32_t)n_tiles & 1u, &sh.abort_flag)) ok = false;
+      if (ok) l_run += sh.xch[(1 - half) * 128 + row];
     }
     if (ok && !warp_wait(&sh.o_final, 0, &sh.abort_flag)) ok = false;
     if (!ok) set_abort(sh, p.dev_status);
@@ -387,7 +441,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     const size_t orow = (((size_t)r * p.B + trow) * p.Hq + kvh * p.G + g);
     if (ok) {
 #pragma unroll 1
-      for (int c = 0; c < D; c += 16) {
+      for (int c = half * kDh; c < (half + 1) * kDh; c += 16) {
         uint32_t o[16];
         tc::tmem_ld16(tmem_o + lane_off + c, o);
         tc::tmem_ld_wait();
@@ -396,9 +450,9 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
           uint32_t pkd[8];
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
-            __nv_bfloat162 h = __floats2bfloat162_rn(__uint_as_float(o[2 * i]) * inv,
-                                                     __uint_as_float(o[2 * i + 1]) * inv);
-            pkd[i] = *reinterpret_cast<uint32_t*>(&h);
+            __nv_bfloat162 h2 = __floats2bfloat162_rn(__uint_as_float(o[2 * i]) * inv,
+                                                      __uint_as_float(o[2 * i + 1]) * inv);
+            pkd[i] = *reinterpret_cast<uint32_t*>(&h2);
           }
           uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(p.out) + orow * D + c);
           dst[0] = make_uint4(pkd[0], pkd[1], pkd[2], pkd[3]);
@@ -413,7 +467,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         }
       }
     }
-    if (write) {
+    if (write && half == 0) {
       const float lse = l_run > 0.f ? (m_run + __log2f(l_run)) * 0.6931471805599453f : -INFINITY;
       if (p.n_split == 1) {
         if (p.lse) p.lse[orow] = lse;
