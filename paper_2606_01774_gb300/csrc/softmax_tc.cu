@@ -11,19 +11,26 @@
 // every prefix token; the mask only touches the ragged prefix end and the
 // block tile (bidirectional, or token-causal for the state-update pass).
 //
+// Tensor memory holds Q (bf16, loaded once), the O accumulator and two S
+// buffers; each S buffer is overwritten in place by its bf16 probabilities P,
+// which the P.V MMA reads straight from tensor memory.  Shared memory only
+// holds a ring of K and V tiles, so per tile the SM moves each K/V byte in
+// once (TMA) and out once (MMA operand read).
+//
 // Warp roles (320 threads):
-//   warp 0     TMA producer: Q once, then K and V tiles (one TMA box per page
-//              and 64-column chunk, 128-byte swizzle) into a ring of stages.
-//   warp 1     tensor-memory owner and MMA issuer: S = Q K^T into one of two
-//              TMEM buffers, then O += P V with P from shared memory; zeroes
-//              the V rows past the prefix end so poisoned cache rows never
-//              meet a zero probability (0 * NaN).
-//   warps 2-9  softmax: two warps per TMEM lane quarter, each thread one
-//              query row and half of the tile's key columns; online base-2
-//              softmax with a lazily moved running max (O in TMEM is rescaled
-//              only when the max grows by more than 2^8), P written as bf16 in
-//              the swizzled layout the MMA reads; epilogue divides by the row
-//              sum and stores the output (or a split partial).
+//   warp 0     TMA producer: K and V tiles (one box per page and 64-column
+//              chunk, 128-byte swizzle) in the order the MMA warp consumes
+//              them (K runs one tile ahead of V).
+//   warp 1     tensor-memory owner and MMA issuer: S_j = Q K_j^T, then
+//              O += P_{j-1} V_{j-1}; zeroes V rows past the prefix end so
+//              poisoned cache rows never meet a zero probability (0 * NaN).
+//              MMAs from this one thread execute in issue order, which is what
+//              lets S_{j+2} reuse the buffer P_j lives in.
+//   warps 2-9  softmax: two warps per TMEM lane quarter, each thread one query
+//              row and half of the tile's 64 key columns; online base-2
+//              softmax with a lazily moved running max (O is rescaled only when
+//              the max grows by more than 2^8); epilogue divides by the row sum
+//              and stores the output (or a split partial).
 // Every wait is bounded (tc::mbar_wait); a timeout sets FLARE_DEV_WAIT_TIMEOUT,
 // the CTA stops issuing work, writes nothing, frees its TMEM and exits.
 #include <cudaTypedefs.h>
@@ -42,7 +49,6 @@ constexpr int kThreadsTC = 320;  // producer warp, MMA warp, 8 softmax warps
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 
 struct TcMaps {
-  CUtensorMap q;      // (D, Hq, B, R)           box (64, G, 128/G, 1)
   CUtensorMap kblk;   // (D, Hkv, B, R)          box (64, 1, 64, 1)
   CUtensorMap vblk;
   CUtensorMap kpool;  // (D, p, Hkv, num_pages)  box (64, min(p,64), 1, 1)
@@ -52,19 +58,19 @@ struct TcMaps {
 template <int D>
 struct TcCfg {
   static constexpr int kChunks = D / 64;
-  static constexpr int kStages = D == 256 ? 2 : 4;
-  static constexpr int kQBytes = kChunks * kRowsM * 128;
-  static constexpr int kKVBytes = kChunks * kTileN * 128;  // one K (or V) stage
-  static constexpr int kPBytes = kRowsM * 128;             // 128 rows x 64 bf16
-  static constexpr int kSmem = kQBytes + 2 * kStages * kKVBytes + 2 * kPBytes;
-  static constexpr int kTmemCols = D == 256 ? 512 : 256;
-  static constexpr int kSCol = D == 256 ? 256 : (D == 128 ? 128 : 64);  // first S buffer
+  static constexpr int kKVBytes = kChunks * kTileN * 128;  // one K (or V) tile
+  static constexpr int kStages = D == 256 ? 3 : (D == 128 ? 6 : 8);
+  static constexpr int kSmem = 2 * kStages * kKVBytes;
+  // tensor memory: O [0, D), S/P buffers [D, D + 128), Q (bf16 pairs) [D + 128, D + 128 + D/2)
+  static constexpr int kTmemCols = (D + 128 + D / 2) > 256 ? 512 : 256;
+  static constexpr int kSCol = D;
+  static constexpr int kQCol = D + 128;
 };
 
 struct TcShared {
-  uint64_t q_full;
-  uint64_t k_full[4], v_full[4], k_empty[4], v_empty[4];
-  uint64_t s_full[2], s_empty[2], p_full[2], p_empty[2];
+  uint64_t q_ready;
+  uint64_t k_full[8], v_full[8], k_empty[8], v_empty[8];
+  uint64_t s_full[2], p_full[2], pv_done[2];
   uint64_t o_final;
   uint64_t xbar[4];     // row-pair exchange written, one per TMEM lane quarter (64 arrivals)
   uint64_t xread[4];    // row-pair exchange read (64 arrivals)
@@ -91,6 +97,32 @@ __device__ __forceinline__ void set_abort(TcShared& sh, int32_t* status) {
   }
 }
 
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+      "%11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_st_wait() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// D[tmem] (+)= A[tmem] * B[smem]^T, bf16, fp32 accumulate; one thread.
+__device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                            uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n"
+      " .reg .pred p;\n"
+      " setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n"
+      "}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
 }  // namespace
 
 template <int D>
@@ -100,10 +132,8 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
   extern __shared__ uint8_t smem_raw[];
   __shared__ TcShared sh;
   uint8_t* base = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  uint8_t* Qs = base;
-  uint8_t* Ks = Qs + C::kQBytes;
+  uint8_t* Ks = base;
   uint8_t* Vs = Ks + C::kStages * C::kKVBytes;
-  uint8_t* Ps = Vs + C::kStages * C::kKVBytes;
 
   const int mtile = blockIdx.x, split = blockIdx.y, item = blockIdx.z;
   const int r = item / p.Hkv, kvh = item % p.Hkv;
@@ -136,7 +166,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
 
   if (tid == 0) {
     sh.abort_flag = 0;
-    tc::mbar_init(&sh.q_full, 1);
+    tc::mbar_init(&sh.q_ready, 256);
     for (int s = 0; s < C::kStages; ++s) {
       tc::mbar_init(&sh.k_full[s], 1);
       tc::mbar_init(&sh.v_full[s], 1);
@@ -145,9 +175,8 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     }
     for (int b = 0; b < 2; ++b) {
       tc::mbar_init(&sh.s_full[b], 1);
-      tc::mbar_init(&sh.s_empty[b], 256);
       tc::mbar_init(&sh.p_full[b], 256);
-      tc::mbar_init(&sh.p_empty[b], 1);
+      tc::mbar_init(&sh.pv_done[b], 1);
     }
     tc::mbar_init(&sh.o_final, 1);
     for (int q = 0; q < 4; ++q) {
@@ -163,6 +192,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
   const uint32_t tmem = sh.tmem_base;
   const uint32_t tmem_o = tmem;
   const uint32_t tmem_s = tmem + C::kSCol;
+  const uint32_t tmem_q = tmem + C::kQCol;
 
   // tile index -> (is block tile, prefix tile number)
   auto tile_kind = [&](int j, int& ptile) -> bool {
@@ -183,14 +213,8 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
   if (warp == 0) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
-      tc::prefetch_tmap(&maps.q);
       tc::prefetch_tmap(&maps.kpool);
       tc::prefetch_tmap(&maps.vpool);
-      const int Bt = kRowsM / p.G;
-      tc::mbar_expect_tx(&sh.q_full, C::kQBytes);
-      for (int c = 0; c < C::kChunks; ++c)
-        tc::tma_load_4d(Qs + c * (kRowsM * 128), &maps.q, &sh.q_full, c * 64, kvh * p.G,
-                        mtile * Bt, r);
       const int box_rows = p.page_size < kTileN ? p.page_size : kTileN;
       // one K or V tile into its ring slot (waits for the slot to be free)
       auto load = [&](int j, int kv) -> bool {
@@ -235,7 +259,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     // ------------------------------------------------------------ MMA issuer
     const uint32_t id_s = tc::idesc_bf16(kRowsM, kTileN, false, false);
     const uint32_t id_o = tc::idesc_bf16(kRowsM, D, false, true);
-    bool ok = warp_wait(&sh.q_full, 0, &sh.abort_flag);
+    bool ok = warp_wait(&sh.q_ready, 0, &sh.abort_flag);
     auto issue_pv = [&](int i) -> bool {
       const int st = i % C::kStages;
       const int pb = i & 1;
@@ -258,14 +282,12 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
       __syncwarp();
       tc::fence_after_sync();
       if (lane == 0) {
-        const uint8_t* pbuf = Ps + pb * C::kPBytes;
 #pragma unroll
         for (int kk = 0; kk < kTileN / 16; ++kk) {
-          const uint64_t a = tc::sdesc_sw128(tc::smem_u32(pbuf + kk * 32), 16, 1024);
           const uint64_t b = tc::sdesc_sw128(tc::smem_u32(vst + kk * 2048), kTileN * 128, 1024);
-          tc::mma_bf16_ss(tmem_o, a, b, id_o, (i > 0 || kk > 0) ? 1u : 0u);
+          mma_bf16_ts(tmem_o, tmem_s + pb * kTileN + kk * 8, b, id_o, (i > 0 || kk > 0) ? 1u : 0u);
         }
-        tc::mma_commit(&sh.p_empty[pb]);
+        tc::mma_commit(&sh.pv_done[pb]);
         tc::mma_commit(&sh.v_empty[st]);
       }
       __syncwarp();
@@ -274,8 +296,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     for (int j = 0; j < n_tiles && ok; ++j) {
       const int st = j % C::kStages;
       const int sb = j & 1;
-      ok = warp_wait(&sh.k_full[st], (uint32_t)(j / C::kStages) & 1u, &sh.abort_flag) &&
-           warp_wait(&sh.s_empty[sb], ((uint32_t)(j >> 1) & 1u) ^ 1u, &sh.abort_flag);
+      ok = warp_wait(&sh.k_full[st], (uint32_t)(j / C::kStages) & 1u, &sh.abort_flag);
       if (!ok) break;
       tc::fence_after_sync();
       if (lane == 0) {
@@ -283,9 +304,8 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const int c = kk >> 2, off = (kk & 3) * 32;
-          const uint64_t a = tc::sdesc_sw128(tc::smem_u32(Qs + c * (kRowsM * 128) + off), 16, 1024);
           const uint64_t b = tc::sdesc_sw128(tc::smem_u32(kst + c * (kTileN * 128) + off), 16, 1024);
-          tc::mma_bf16_ss(tmem_s + sb * kTileN, a, b, id_s, kk > 0 ? 1u : 0u);
+          mma_bf16_ts(tmem_s + sb * kTileN, tmem_q + kk * 8, b, id_s, kk > 0 ? 1u : 0u);
         }
         tc::mma_commit(&sh.s_full[sb]);
         tc::mma_commit(&sh.k_empty[st]);
@@ -307,7 +327,33 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     const int m = mtile * kRowsM + row;
     const int trow = m / p.G;
     const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
-    constexpr int kDh = D / 2;  // output columns this half rescales / stores
+    constexpr int kDh = D / 2;  // Q elements / output columns this half handles
+
+    // Q row (this half's D/2 elements) into tensor memory as bf16 pairs
+    {
+      const int g = m % p.G;
+      const bool live = m < M;
+      const uint4* qrow = reinterpret_cast<const uint4*>(
+          static_cast<const __nv_bfloat16*>(p.q) +
+          (((size_t)r * p.B + (live ? trow : 0)) * p.Hq + kvh * p.G + g) * D + half * kDh);
+#pragma unroll 1
+      for (int c = 0; c < kDh / 2; c += 16) {  // 16 TMEM columns = 32 bf16 = 4 x 16 B
+        uint32_t w[16];
+#pragma unroll
+        for (int q4 = 0; q4 < 4; ++q4) {
+          const uint4 v = live ? qrow[c / 4 + q4] : make_uint4(0u, 0u, 0u, 0u);
+          w[4 * q4] = v.x;
+          w[4 * q4 + 1] = v.y;
+          w[4 * q4 + 2] = v.z;
+          w[4 * q4 + 3] = v.w;
+        }
+        tmem_st16(tmem_q + lane_off + half * (kDh / 2) + c, w);
+      }
+      tmem_st_wait();
+      tc::fence_before_sync();
+      tc::mbar_arrive(&sh.q_ready);
+    }
+
     float m_run = -INFINITY, l_run = 0.f;  // l_run: this half's share of the row sum
     bool ok = true;
     for (int j = 0; j < n_tiles; ++j) {
@@ -317,14 +363,11 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         break;
       }
       tc::fence_after_sync();
+      const uint32_t sbuf = tmem_s + lane_off + sb * kTileN;
       uint32_t sr[32];
-      tc::tmem_ld16(tmem_s + lane_off + sb * kTileN + 32 * half,
-                    *reinterpret_cast<uint32_t(*)[16]>(&sr[0]));
-      tc::tmem_ld16(tmem_s + lane_off + sb * kTileN + 32 * half + 16,
-                    *reinterpret_cast<uint32_t(*)[16]>(&sr[16]));
+      tc::tmem_ld16(sbuf + 32 * half, *reinterpret_cast<uint32_t(*)[16]>(&sr[0]));
+      tc::tmem_ld16(sbuf + 32 * half + 16, *reinterpret_cast<uint32_t(*)[16]>(&sr[16]));
       tc::tmem_ld_wait();
-      tc::fence_before_sync();
-      tc::mbar_arrive(&sh.s_empty[sb]);
 
       int pt;
       const bool blk = tile_kind(j, pt);
@@ -332,21 +375,25 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
       const bool full = !blk && valid == kTileN;  // prefix tile: no mask at all
       const int lim = full ? kTileN : ((blk && p.causal) ? min(valid, trow + 1) : valid);
       // tile maximum of the raw scores (scale >= 0 keeps the order)
-      float mt = -INFINITY;
+      float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
       for (int c = 0; c < 32; ++c)
-        if (full || 32 * half + c < lim) mt = fmaxf(mt, __uint_as_float(sr[c]));
-      // the partner has read this slot's previous value before it is overwritten
+        if (full || 32 * half + c < lim) mx[c & 3] = fmaxf(mx[c & 3], __uint_as_float(sr[c]));
+      float mt = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+      // the partner has read this slot's previous value before it is overwritten;
+      // this exchange also orders both halves' S reads before either writes P.
       if (j >= 1 && !warp_wait(&sh.xread[quarter], (uint32_t)(j - 1) & 1u, &sh.abort_flag)) {
         ok = false;
         break;
       }
       sh.xch[half * 128 + row] = mt;
+      tc::fence_before_sync();
       tc::mbar_arrive(&sh.xbar[quarter]);
       if (!warp_wait(&sh.xbar[quarter], (uint32_t)j & 1u, &sh.abort_flag)) {
         ok = false;
         break;
       }
+      tc::fence_after_sync();
       mt = fmaxf(mt, sh.xch[(1 - half) * 128 + row]);
       tc::mbar_arrive(&sh.xread[quarter]);
       const float m_new = fmaxf(m_run, mt * p.scale_log2);
@@ -356,14 +403,15 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
       if (warp_rescale) m_use = (j == 0 || m_new > m_run) ? m_new : m_run;
       const float corr = (j == 0) ? 0.f : tc::ex2(m_run - m_use);
       const float neg_m = -m_use;
-      float sum = 0.f;
+      float sum0 = 0.f, sum1 = 0.f;
       uint32_t pk[16];
       if (full) {
 #pragma unroll
         for (int c = 0; c < 32; c += 2) {
           const float p0 = tc::ex2(fmaf(__uint_as_float(sr[c]), p.scale_log2, neg_m));
           const float p1 = tc::ex2(fmaf(__uint_as_float(sr[c + 1]), p.scale_log2, neg_m));
-          sum += p0 + p1;
+          sum0 += p0;
+          sum1 += p1;
           __nv_bfloat162 h2 = __floats2bfloat162_rn(p0, p1);
           pk[c / 2] = *reinterpret_cast<uint32_t*>(&h2);
         }
@@ -375,21 +423,18 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
               col < lim ? tc::ex2(fmaf(__uint_as_float(sr[c]), p.scale_log2, neg_m)) : 0.f;
           const float p1 =
               col + 1 < lim ? tc::ex2(fmaf(__uint_as_float(sr[c + 1]), p.scale_log2, neg_m)) : 0.f;
-          sum += p0 + p1;
+          sum0 += p0;
+          sum1 += p1;
           __nv_bfloat162 h2 = __floats2bfloat162_rn(p0, p1);
           pk[c / 2] = *reinterpret_cast<uint32_t*>(&h2);
         }
       }
+      const float sum = sum0 + sum1;
       l_run = (j == 0) ? sum : l_run * corr + sum;
-      // P buffer free once the P.V of tile j-2 has completed
-      if (j >= 2 && !warp_wait(&sh.p_empty[sb], ((uint32_t)(j >> 1) & 1u) ^ 1u, &sh.abort_flag)) {
-        ok = false;
-        break;
-      }
       // rescale this half's O columns when the running max moved (P.V of tile j-1 done)
       if (warp_rescale && j >= 1) {
         const int pb = (j - 1) & 1;
-        if (!warp_wait(&sh.p_empty[pb], (uint32_t)((j - 1) >> 1) & 1u, &sh.abort_flag)) {
+        if (!warp_wait(&sh.pv_done[pb], (uint32_t)((j - 1) >> 1) & 1u, &sh.abort_flag)) {
           ok = false;
           break;
         }
@@ -401,25 +446,13 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
           tc::tmem_ld_wait();
 #pragma unroll
           for (int i = 0; i < 16; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * corr);
-          asm volatile(
-              "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, "
-              "%9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(tmem_o + lane_off + c),
-              "r"(o[0]), "r"(o[1]), "r"(o[2]), "r"(o[3]), "r"(o[4]), "r"(o[5]), "r"(o[6]),
-              "r"(o[7]), "r"(o[8]), "r"(o[9]), "r"(o[10]), "r"(o[11]), "r"(o[12]), "r"(o[13]),
-              "r"(o[14]), "r"(o[15])
-              : "memory");
+          tmem_st16(tmem_o + lane_off + c, o);
         }
-        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
       }
       m_run = m_use;
-      uint8_t* prow = Ps + sb * C::kPBytes + row * 128;
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int sw = (4 * half + q) ^ (row & 7);
-        *reinterpret_cast<uint4*>(prow + sw * 16) =
-            make_uint4(pk[q * 4], pk[q * 4 + 1], pk[q * 4 + 2], pk[q * 4 + 3]);
-      }
-      tc::fence_async_smem();
+      // P (bf16 pairs) over this half's 16 columns of the S buffer
+      tmem_st16(sbuf + 16 * half, pk);
+      tmem_st_wait();
       tc::fence_before_sync();
       tc::mbar_arrive(&sh.p_full[sb]);
     }
@@ -520,12 +553,6 @@ cudaError_t launch_tc_d(const SoftmaxParams& p, const SoftmaxPlan& plan, cudaStr
   using C = TcCfg<D>;
   TcMaps maps;
   const uint64_t e = 2;
-  {
-    const uint64_t dims[4] = {(uint64_t)D, (uint64_t)p.Hq, (uint64_t)p.B, (uint64_t)p.R};
-    const uint64_t str[3] = {D * e, (uint64_t)p.Hq * D * e, (uint64_t)p.B * p.Hq * D * e};
-    const uint32_t box[4] = {64, (uint32_t)p.G, (uint32_t)(kRowsM / p.G), 1};
-    if (!encode4(&maps.q, p.q, dims, str, box)) return cudaErrorInvalidValue;
-  }
   {
     const uint64_t dims[4] = {(uint64_t)D, (uint64_t)p.Hkv, (uint64_t)p.B, (uint64_t)p.R};
     const uint64_t str[3] = {D * e, (uint64_t)p.Hkv * D * e, (uint64_t)p.B * p.Hkv * D * e};
