@@ -59,8 +59,9 @@ template <int D>
 struct TcCfg {
   static constexpr int kChunks = D / 64;
   static constexpr int kKVBytes = kChunks * kTileN * 128;  // one K (or V) tile
-  static constexpr int kStages = D == 256 ? 3 : (D == 128 ? 6 : 8);
-  static constexpr int kSmem = 2 * kStages * kKVBytes;
+  static constexpr int kKStages = D == 256 ? 4 : (D == 128 ? 8 : 8);  // K ring depth
+  static constexpr int kVStages = D == 256 ? 2 : (D == 128 ? 4 : 8);  // V ring depth
+  static constexpr int kSmem = (kKStages + kVStages) * kKVBytes;
   // tensor memory: O [0, D), S/P buffers [D, D + 128), Q (bf16 pairs) [D + 128, D + 128 + D/2)
   static constexpr int kTmemCols = (D + 128 + D / 2) > 256 ? 512 : 256;
   static constexpr int kSCol = D;
@@ -133,7 +134,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
   __shared__ TcShared sh;
   uint8_t* base = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t* Ks = base;
-  uint8_t* Vs = Ks + C::kStages * C::kKVBytes;
+  uint8_t* Vs = Ks + C::kKStages * C::kKVBytes;
 
   const int mtile = blockIdx.x, split = blockIdx.y, item = blockIdx.z;
   const int r = item / p.Hkv, kvh = item % p.Hkv;
@@ -167,10 +168,12 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
   if (tid == 0) {
     sh.abort_flag = 0;
     tc::mbar_init(&sh.q_ready, 256);
-    for (int s = 0; s < C::kStages; ++s) {
+    for (int s = 0; s < C::kKStages; ++s) {
       tc::mbar_init(&sh.k_full[s], 1);
-      tc::mbar_init(&sh.v_full[s], 1);
       tc::mbar_init(&sh.k_empty[s], 1);
+    }
+    for (int s = 0; s < C::kVStages; ++s) {
+      tc::mbar_init(&sh.v_full[s], 1);
       tc::mbar_init(&sh.v_empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
@@ -218,8 +221,9 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
       const int box_rows = p.page_size < kTileN ? p.page_size : kTileN;
       // one K or V tile into its ring slot (waits for the slot to be free)
       auto load = [&](int j, int kv) -> bool {
-        const int st = j % C::kStages;
-        const uint32_t ph = (uint32_t)(j / C::kStages) & 1u;
+        const int ns = kv ? C::kVStages : C::kKStages;
+        const int st = j % ns;
+        const uint32_t ph = (uint32_t)(j / ns) & 1u;
         uint64_t* empty = kv ? &sh.v_empty[st] : &sh.k_empty[st];
         uint64_t* full = kv ? &sh.v_full[st] : &sh.k_full[st];
         uint8_t* dst = (kv ? Vs : Ks) + st * C::kKVBytes;
@@ -247,10 +251,13 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         }
         return true;
       };
-      // consumption order of the MMA warp: K0, K1, V0, K2, V1, ...
-      bool ok = load(0, 0);
+      // K runs two tiles ahead of V: K0, K1, K2, V0, K3, V1, ... (the MMA warp
+      // consumes K_j at S_j and V_j one step later, at P_j V_j)
+      constexpr int kLead = 2;
+      bool ok = true;
+      for (int j = 0; j < kLead && j < n_tiles && ok; ++j) ok = load(j, 0);
       for (int j = 0; j < n_tiles && ok && !aborted(sh); ++j) {
-        if (j + 1 < n_tiles) ok = load(j + 1, 0);
+        if (j + kLead < n_tiles) ok = load(j + kLead, 0);
         if (ok) ok = load(j, 1);
       }
       if (!ok) set_abort(sh, p.dev_status);
@@ -261,10 +268,10 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     const uint32_t id_o = tc::idesc_bf16(kRowsM, D, false, true);
     bool ok = warp_wait(&sh.q_ready, 0, &sh.abort_flag);
     auto issue_pv = [&](int i) -> bool {
-      const int st = i % C::kStages;
+      const int st = i % C::kVStages;
       const int pb = i & 1;
       if (!warp_wait(&sh.p_full[pb], (uint32_t)(i >> 1) & 1u, &sh.abort_flag)) return false;
-      if (!warp_wait(&sh.v_full[st], (uint32_t)(i / C::kStages) & 1u, &sh.abort_flag))
+      if (!warp_wait(&sh.v_full[st], (uint32_t)(i / C::kVStages) & 1u, &sh.abort_flag))
         return false;
       uint8_t* vst = Vs + st * C::kKVBytes;
       const int valid = tile_valid(i);
@@ -294,9 +301,9 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
       return true;
     };
     for (int j = 0; j < n_tiles && ok; ++j) {
-      const int st = j % C::kStages;
+      const int st = j % C::kKStages;
       const int sb = j & 1;
-      ok = warp_wait(&sh.k_full[st], (uint32_t)(j / C::kStages) & 1u, &sh.abort_flag);
+      ok = warp_wait(&sh.k_full[st], (uint32_t)(j / C::kKStages) & 1u, &sh.abort_flag);
       if (!ok) break;
       tc::fence_after_sync();
       if (lane == 0) {
