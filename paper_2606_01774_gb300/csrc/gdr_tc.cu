@@ -19,7 +19,9 @@
 //
 //   MMA 1   G   = [K;Q] K^T          M=128 (64 k rows, 64 q rows), N=Bp, K=dk
 //   MMA 2   W^T = S0^T [K;Q]^T       M=128 (c),  N=128, K=dk   (S0^T is MN-major)
-//   solve   T   = (I + A)^{-1}       64 threads, one column each, in registers
+//   solve   T   = (I + A)^{-1}       blocked by 16: diagonal blocks by forward
+//                                    substitution, off-diagonal blocks on
+//                                    warp-level tf32 MMA
 //   MMA 3   delta^T = X^T T^T        M=128 (c),  N=Bp,  K=Bp
 //   MMA 4   O2^T = delta^T M2^T      M=128 (c),  N=Bp,  K=Bp, M2[l][i] = exp(gamma_B-gamma_i) q_l.k_i
 //   out[l][c] = s (Gam_B W^T[c][64+l] + O2^T[c][l])
@@ -76,6 +78,25 @@ __device__ __forceinline__ bool lin_wait(uint64_t* bar, uint32_t parity, LinShar
   return all;
 }
 
+__device__ __forceinline__ uint32_t f2tf32(float x) {
+  uint32_t r;
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
+  return r;
+}
+
+// Warp-level D += A B on a 16x8x8 tile, tf32 inputs, fp32 accumulate.
+// Fragments (g = lane/4, q = lane%4): a0 A[g][q], a1 A[g+8][q], a2 A[g][q+4],
+// a3 A[g+8][q+4]; b0 B[q][g], b1 B[q+4][g]; d0 D[g][2q], d1 D[g][2q+1],
+// d2 D[g+8][2q], d3 D[g+8][2q+1].
+__device__ __forceinline__ void mma_tf32(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                         uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+      "{%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
 // 16 bf16 values (columns c0..c0+15) into row `row` of a K-major SW128 tile.
 __device__ __forceinline__ void store16_sw128(uint8_t* tile, int row, int c0, const float (&v)[16]) {
   uint8_t* p = tile + row * 128;
@@ -108,7 +129,7 @@ __global__ void __launch_bounds__(kLinThreads, 2)
   uint8_t* Xs = Ts + C::kT;
   float* A32 = reinterpret_cast<float*>(Xs);   // aliases X^T (A is dead before X is written)
   float* T32 = reinterpret_cast<float*>(KQs);  // fp32 T, in [K;Q] once MMA 1/2 have run
-  float* Ytmp = reinterpret_cast<float*>(Ts);  // 3 x 256 floats, dead until T is converted
+  float* Ytmp = reinterpret_cast<float*>(Ts);  // 4 x 256 floats, dead until T is converted
 
   const int item = blockIdx.x;
   const int r = item / p.Hv, j = item % p.Hv;
@@ -121,6 +142,22 @@ __global__ void __launch_bounds__(kLinThreads, 2)
   if (slot < 0 || slot >= p.nslots) {
     if (tid == 0) flag(p.dev_status, FLARE_DEV_BAD_SLOT);
     return;
+  }
+
+  // the state is the long-latency input: its loads go out before the set-up
+  constexpr int kPer = DK * DV / 4 / kLinThreads;
+  float4 s0buf[kPer];
+  {
+    const float4* S0g =
+        reinterpret_cast<const float4*>(p.state_pool + ((size_t)slot * p.Hv + j) * DK * DV);
+#pragma unroll
+    for (int n = 0; n < kPer; ++n) {
+      // volatile: keep every load issued here, ahead of the set-up below
+      const float4* a = S0g + tid + n * kLinThreads;
+      asm volatile("ld.global.nc.v4.f32 {%0, %1, %2, %3}, [%4];"
+                   : "=f"(s0buf[n].x), "=f"(s0buf[n].y), "=f"(s0buf[n].z), "=f"(s0buf[n].w)
+                   : "l"(a));
+    }
   }
 
   if (tid == 0) {
@@ -150,12 +187,7 @@ __global__ void __launch_bounds__(kLinThreads, 2)
   // S0 (fp32, global) -> bf16 S0^T operand, MN-major 128-byte swizzle:
   // element (c, i) in chunk c/64 at row i, 16-byte group ((c%64)/8) ^ (i%8).
   {
-    const float4* S0g =
-        reinterpret_cast<const float4*>(p.state_pool + ((size_t)slot * p.Hv + j) * DK * DV);
-    constexpr int kPer = DK * DV / 4 / kLinThreads;
-    float4 buf[kPer];
-#pragma unroll
-    for (int n = 0; n < kPer; ++n) buf[n] = __ldg(S0g + tid + n * kLinThreads);
+    const float4* buf = s0buf;
 #pragma unroll
     for (int n = 0; n < kPer; ++n) {
       const int f = tid + n * kLinThreads;
@@ -260,47 +292,89 @@ __global__ void __launch_bounds__(kLinThreads, 2)
   __syncthreads();
 
   // ---- T = (I + A)^{-1}, blocked by 16 (A is strictly lower triangular).
-  // Diagonal blocks: thread (blk, col) solves (I + A_kk) x = e_col in registers.
+  // Diagonal blocks: thread (blk, col) solves (I + A_kk) x = e_col by forward
+  // substitution, x kept in its own column of T32 (rolled loops: this code runs
+  // once per CTA, so it is kept small).
   if (tid < 64) {
     const int blk = tid >> 4, col = tid & 15, o = blk * 16;
-    float x[16];
-#pragma unroll
-    for (int t = 0; t < 16; ++t) {
-      float acc = (t == col) ? 1.f : 0.f;
-#pragma unroll
-      for (int i = 0; i < t; ++i) acc = fmaf(-A32[(o + t) * 64 + o + i], x[i], acc);
-      x[t] = acc;
+    float* xcol = T32 + o * 64 + o + col;          // x[i] at xcol[i * 64]
+    const float* arow0 = A32 + o * 64 + o;         // A_kk[t][i] at arow0[t * 64 + i]
+    xcol[col * 64] = 1.f;
+#pragma unroll 1
+    for (int t = col + 1; t < 16; ++t) {
+      float a0 = 0.f, a1 = 0.f;
+      int i = col;
+#pragma unroll 1
+      for (; i + 1 < t; i += 2) {
+        a0 = fmaf(arow0[t * 64 + i], xcol[i * 64], a0);
+        a1 = fmaf(arow0[t * 64 + i + 1], xcol[(i + 1) * 64], a1);
+      }
+      if (i < t) a0 = fmaf(arow0[t * 64 + i], xcol[i * 64], a0);
+      xcol[t * 64] = -(a0 + a1);
     }
-#pragma unroll
-    for (int t = 0; t < 16; ++t) T32[(o + t) * 64 + o + col] = x[t];
   }
   __syncthreads();
-  // Off-diagonal blocks by distance d = i - j:  T_ij = -T_ii sum_{k=j}^{i-1} A_ik T_kj
+  // Off-diagonal blocks by distance d = i - j:  T_ij = -T_ii sum_{k=j}^{i-1} A_ik T_kj.
+  // One warp per block, 16x16 tiles on warp-level tf32 MMA (m16n8k8); Y goes
+  // through shared memory to change from accumulator to operand layout.
 #pragma unroll 1
   for (int d = 1; d < 4; ++d) {
-    const int nel = (4 - d) * 256;
-#pragma unroll 1
-    for (int e = tid; e < nel; e += kLinThreads) {
-      const int bj = e >> 8, rr = (e >> 4) & 15, cc = e & 15, bi = bj + d;
-      const float* arow = A32 + (16 * bi + rr) * 64;
-      const float* tcol = T32 + 16 * bj + cc;
-      float a0 = 0.f, a1 = 0.f;
-#pragma unroll 4
-      for (int k = 16 * bj; k < 16 * bi; k += 2) {
-        a0 = fmaf(arow[k], tcol[k * 64], a0);
-        a1 = fmaf(arow[k + 1], tcol[(k + 1) * 64], a1);
+    const int bj = warp, bi = bj + d;
+    if (bi < 4) {
+      const int g = lane >> 2, q = lane & 3;
+      float y[2][4];
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) y[nt][e] = 0.f;
       }
-      Ytmp[e] = a0 + a1;
-    }
-    __syncthreads();
+      // Y = sum_k A_{bi,k} T_{k,bj}, k over the 16*d rows between the blocks
 #pragma unroll 1
-    for (int e = tid; e < nel; e += kLinThreads) {
-      const int bj = e >> 8, rr = (e >> 4) & 15, cc = e & 15, bi = bj + d;
-      const float* trow = T32 + (16 * bi + rr) * 64 + 16 * bi;
-      float acc = 0.f;
-#pragma unroll 4
-      for (int u = 0; u <= rr; ++u) acc = fmaf(trow[u], Ytmp[bj * 256 + u * 16 + cc], acc);
-      T32[(16 * bi + rr) * 64 + 16 * bj + cc] = -acc;
+      for (int k8 = 16 * bj; k8 < 16 * bi; k8 += 8) {
+        const float* ar = A32 + (16 * bi + g) * 64 + k8 + q;
+        const uint32_t a0 = f2tf32(ar[0]), a1 = f2tf32(ar[8 * 64]);
+        const uint32_t a2 = f2tf32(ar[4]), a3 = f2tf32(ar[8 * 64 + 4]);
+#pragma unroll
+        for (int nt = 0; nt < 2; ++nt) {
+          const float* br = T32 + (k8 + q) * 64 + 16 * bj + nt * 8 + g;
+          mma_tf32(y[nt], a0, a1, a2, a3, f2tf32(br[0]), f2tf32(br[4 * 64]));
+        }
+      }
+      float* Yw = Ytmp + warp * 256;  // 16 x 16
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt) {
+        Yw[g * 16 + nt * 8 + 2 * q] = y[nt][0];
+        Yw[g * 16 + nt * 8 + 2 * q + 1] = y[nt][1];
+        Yw[(g + 8) * 16 + nt * 8 + 2 * q] = y[nt][2];
+        Yw[(g + 8) * 16 + nt * 8 + 2 * q + 1] = y[nt][3];
+      }
+      __syncwarp();
+      // T_ij = -T_ii Y
+      float t[2][4];
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) t[nt][e] = 0.f;
+      }
+#pragma unroll
+      for (int k8 = 0; k8 < 16; k8 += 8) {
+        const float* ar = T32 + (16 * bi + g) * 64 + 16 * bi + k8 + q;
+        const uint32_t a0 = f2tf32(ar[0]), a1 = f2tf32(ar[8 * 64]);
+        const uint32_t a2 = f2tf32(ar[4]), a3 = f2tf32(ar[8 * 64 + 4]);
+#pragma unroll
+        for (int nt = 0; nt < 2; ++nt) {
+          const float* br = Yw + (k8 + q) * 16 + nt * 8 + g;
+          mma_tf32(t[nt], a0, a1, a2, a3, f2tf32(br[0]), f2tf32(br[4 * 16]));
+        }
+      }
+      float* to = T32 + (16 * bi) * 64 + 16 * bj;
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt) {
+        to[g * 64 + nt * 8 + 2 * q] = -t[nt][0];
+        to[g * 64 + nt * 8 + 2 * q + 1] = -t[nt][1];
+        to[(g + 8) * 64 + nt * 8 + 2 * q] = -t[nt][2];
+        to[(g + 8) * 64 + nt * 8 + 2 * q + 1] = -t[nt][3];
+      }
     }
     __syncthreads();
   }
