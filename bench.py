@@ -100,6 +100,34 @@ def commit_bytes(spec, accept):
             + 2 * R * B * Hv * 4)
 
 
+# ---------------------------------------------------------------- ncu traffic
+
+
+KERNEL_OF = {"linear": "gdr_denoise_tc_kernel", "softmax": "softmax_tc_kernel",
+             "commit": "gdr_commit_kernel"}
+
+
+def profiled_traffic(kernel, workload):
+    """DRAM bytes per launch from the committed ncu summary of `kernel` on
+    `workload` (profiles/<kernel>_<workload>_traffic.md), or None when there is
+    none or the kernel's source has changed since it was taken."""
+    import hashlib
+
+    path = os.path.join(ROOT, "profiles", f"{kernel}_{workload}_traffic.md")
+    try:
+        fields = {}
+        for line in open(path):
+            if ":" in line and not line.startswith(" "):
+                k, v = line.split(":", 1)
+                fields[k.strip()] = v.strip()
+        src = os.path.join(ROOT, fields["kernel_source"])
+        if hashlib.sha256(open(src, "rb").read()).hexdigest() != fields["kernel_source_sha256"]:
+            return None
+        return int(fields["traffic_bytes_per_launch"])
+    except (OSError, KeyError, ValueError):
+        return None
+
+
 # ---------------------------------------------------------------- clocks
 
 
@@ -283,6 +311,22 @@ class E2ERunner:
         torch.cuda.current_stream().synchronize()
 
 
+def max_over_ranks(x, distributed, device):
+    """Max of a per-rank scalar over all ranks (timing only: no data-path collective)."""
+    if not distributed:
+        return x
+    import torch.distributed as tdist
+
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def rank_seed_offset(rank):
+    """Each rank draws its own batch (independent requests: weak scaling)."""
+    return 1000 * rank
+
+
 def _elapsed_pairs(evs):
     return [evs[i].elapsed_time(evs[i + 1]) for i in range(0, len(evs), 2)]
 
@@ -293,7 +337,7 @@ def run_flare(args, spec, rank, world, local_rank):
     from paper_2606_01774_gb300 import flare
 
     flare.load()
-    fr = FlareRunner(spec, device, seed_offset=1000 * rank)
+    fr = FlareRunner(spec, device, seed_offset=rank_seed_offset(rank))
     dist = world > 1
     if dist:
         import torch.distributed as tdist
@@ -322,11 +366,7 @@ def run_flare(args, spec, rank, world, local_rank):
     if dist:
         tdist.barrier()
     clk = clocks.stop() if clocks else None
-    ms = t0.elapsed_time(t1)
-    if dist:
-        tt = torch.tensor([ms], dtype=torch.float64, device=device)
-        tdist.all_reduce(tt, op=tdist.ReduceOp.MAX)
-        ms = float(tt.item())
+    ms = max_over_ranks(t0.elapsed_time(t1), dist, device)
     ms_step = ms / args.steps
 
     # end-to-end through host buffers
@@ -340,11 +380,7 @@ def run_flare(args, spec, rank, world, local_rank):
         t_e = time.perf_counter()
         for _ in range(args.steps):
             e2e.step()
-        e2e_ms = (time.perf_counter() - t_e) * 1e3 / args.steps
-        if dist:
-            tt = torch.tensor([e2e_ms], dtype=torch.float64, device=device)
-            tdist.all_reduce(tt, op=tdist.ReduceOp.MAX)
-            e2e_ms = float(tt.item())
+        e2e_ms = max_over_ranks((time.perf_counter() - t_e) * 1e3 / args.steps, dist, device)
     st, bits = flare.flare_read_status(fr.status)
     if st != flare.FLARE_OK:
         raise RuntimeError(f"device status {bits:#x} after timing")
@@ -377,7 +413,7 @@ def run_flare(args, spec, rank, world, local_rank):
         roof = {"bound": "hbm", "achieved": kd["bytes"] / dur_s / 1e9,
                 "peak": peaks["hbm_gbs"], "unit": "GB/s"}
     roof["frac"] = roof["achieved"] / roof["peak"]
-    roof["traffic"] = None
+    roof["traffic"] = profiled_traffic(KERNEL_OF[dom], s.name)
     roof["kernel"] = kd["kernel"]
     roof["peak_source"] = f"{peaks['source']} ({'bf16_tflops_sustained' if roof['unit'] == 'TFLOP/s' else 'hbm_gbs'})"
     roof["algorithmic_per_launch"] = kd["flops"] if roof["bound"] == "tensor" else kd["bytes"]
