@@ -45,10 +45,13 @@ namespace {
 
 constexpr int kTileN = 64;     // keys per tile
 constexpr int kRowsM = 128;    // query rows per CTA (TMEM lanes)
-constexpr int kThreadsTC = 320;  // producer warp, MMA warp, 8 softmax warps
+constexpr int kSplit = 1;        // softmax warps per TMEM lane quarter (each takes 64/kSplit keys)
+constexpr int kSoftmaxThreads = 128 * kSplit;
+constexpr int kThreadsTC = 64 + kSoftmaxThreads;  // producer warp, MMA warp, softmax warps
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 
 struct TcMaps {
+  CUtensorMap q;      // (D, Hq, B, R)           box (64, G, 128/G, 1)
   CUtensorMap kblk;   // (D, Hkv, B, R)          box (64, 1, 64, 1)
   CUtensorMap vblk;
   CUtensorMap kpool;  // (D, p, Hkv, num_pages)  box (64, min(p,64), 1, 1)
@@ -59,19 +62,19 @@ template <int D>
 struct TcCfg {
   static constexpr int kChunks = D / 64;
   static constexpr int kKVBytes = kChunks * kTileN * 128;  // one K (or V) tile
-  static constexpr int kKStages = D == 256 ? 4 : (D == 128 ? 8 : 8);  // K ring depth
+  static constexpr int kQBytes = kChunks * kRowsM * 128;   // Q tile, K-major, 128-byte swizzle
+  static constexpr int kKStages = D == 256 ? 3 : (D == 128 ? 6 : 8);  // K ring depth
   static constexpr int kVStages = D == 256 ? 2 : (D == 128 ? 4 : 8);  // V ring depth
-  static constexpr int kSmem = (kKStages + kVStages) * kKVBytes;
-  // tensor memory: O [0, D), S/P buffers [D, D + 128), Q (bf16 pairs) [D + 128, D + 128 + D/2)
-  static constexpr int kTmemCols = (D + 128 + D / 2) > 256 ? 512 : 256;
+  static constexpr int kSmem = kQBytes + (kKStages + kVStages) * kKVBytes;
+  // tensor memory: O [0, D), three S/P buffers [D, D + 192)
+  static constexpr int kTmemCols = (D + 3 * kTileN) > 256 ? 512 : 256;
   static constexpr int kSCol = D;
-  static constexpr int kQCol = D + 128;
 };
 
 struct TcShared {
-  uint64_t q_ready;
+  uint64_t q_full;
   uint64_t k_full[8], v_full[8], k_empty[8], v_empty[8];
-  uint64_t s_full[2], p_full[2], pv_done[2];
+  uint64_t s_full[3], p_full[3], pv_done[3];
   uint64_t o_final;
   uint64_t xbar[4];     // row-pair exchange written, one per TMEM lane quarter (64 arrivals)
   uint64_t xread[4];    // row-pair exchange read (64 arrivals)
@@ -133,7 +136,8 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
   extern __shared__ uint8_t smem_raw[];
   __shared__ TcShared sh;
   uint8_t* base = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  uint8_t* Ks = base;
+  uint8_t* Qs = base;
+  uint8_t* Ks = Qs + C::kQBytes;
   uint8_t* Vs = Ks + C::kKStages * C::kKVBytes;
 
   const int mtile = blockIdx.x, split = blockIdx.y, item = blockIdx.z;
@@ -167,7 +171,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
 
   if (tid == 0) {
     sh.abort_flag = 0;
-    tc::mbar_init(&sh.q_ready, 256);
+    tc::mbar_init(&sh.q_full, 1);
     for (int s = 0; s < C::kKStages; ++s) {
       tc::mbar_init(&sh.k_full[s], 1);
       tc::mbar_init(&sh.k_empty[s], 1);
@@ -176,15 +180,15 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
       tc::mbar_init(&sh.v_full[s], 1);
       tc::mbar_init(&sh.v_empty[s], 1);
     }
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < 3; ++b) {
       tc::mbar_init(&sh.s_full[b], 1);
-      tc::mbar_init(&sh.p_full[b], 256);
+      tc::mbar_init(&sh.p_full[b], kSoftmaxThreads);
       tc::mbar_init(&sh.pv_done[b], 1);
     }
     tc::mbar_init(&sh.o_final, 1);
     for (int q = 0; q < 4; ++q) {
-      tc::mbar_init(&sh.xbar[q], 64);
-      tc::mbar_init(&sh.xread[q], 64);
+      tc::mbar_init(&sh.xbar[q], 32 * kSplit);
+      tc::mbar_init(&sh.xread[q], 32 * kSplit);
     }
     tc::fence_mbar_init();
   }
@@ -195,7 +199,6 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
   const uint32_t tmem = sh.tmem_base;
   const uint32_t tmem_o = tmem;
   const uint32_t tmem_s = tmem + C::kSCol;
-  const uint32_t tmem_q = tmem + C::kQCol;
 
   // tile index -> (is block tile, prefix tile number)
   auto tile_kind = [&](int j, int& ptile) -> bool {
@@ -218,6 +221,11 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     if (lane == 0) {
       tc::prefetch_tmap(&maps.kpool);
       tc::prefetch_tmap(&maps.vpool);
+      const int Bt = kRowsM / p.G;
+      tc::mbar_expect_tx(&sh.q_full, C::kQBytes);
+      for (int c = 0; c < C::kChunks; ++c)
+        tc::tma_load_4d(Qs + c * (kRowsM * 128), &maps.q, &sh.q_full, c * 64, kvh * p.G,
+                        mtile * Bt, r);
       const int box_rows = p.page_size < kTileN ? p.page_size : kTileN;
       // one K or V tile into its ring slot (waits for the slot to be free)
       auto load = [&](int j, int kv) -> bool {
@@ -266,11 +274,11 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     // ------------------------------------------------------------ MMA issuer
     const uint32_t id_s = tc::idesc_bf16(kRowsM, kTileN, false, false);
     const uint32_t id_o = tc::idesc_bf16(kRowsM, D, false, true);
-    bool ok = warp_wait(&sh.q_ready, 0, &sh.abort_flag);
+    bool ok = warp_wait(&sh.q_full, 0, &sh.abort_flag);
     auto issue_pv = [&](int i) -> bool {
       const int st = i % C::kVStages;
-      const int pb = i & 1;
-      if (!warp_wait(&sh.p_full[pb], (uint32_t)(i >> 1) & 1u, &sh.abort_flag)) return false;
+      const int pb = i % 3;
+      if (!warp_wait(&sh.p_full[pb], (uint32_t)(i / 3) & 1u, &sh.abort_flag)) return false;
       if (!warp_wait(&sh.v_full[st], (uint32_t)(i / C::kVStages) & 1u, &sh.abort_flag))
         return false;
       uint8_t* vst = Vs + st * C::kKVBytes;
@@ -300,27 +308,37 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
       __syncwarp();
       return true;
     };
-    for (int j = 0; j < n_tiles && ok; ++j) {
+    // S_j = Q K_j^T into S buffer j % 3
+    auto issue_s = [&](int j) -> bool {
       const int st = j % C::kKStages;
-      const int sb = j & 1;
-      ok = warp_wait(&sh.k_full[st], (uint32_t)(j / C::kKStages) & 1u, &sh.abort_flag);
-      if (!ok) break;
+      const int sb = j % 3;
+      if (!warp_wait(&sh.k_full[st], (uint32_t)(j / C::kKStages) & 1u, &sh.abort_flag))
+        return false;
       tc::fence_after_sync();
       if (lane == 0) {
         const uint8_t* kst = Ks + st * C::kKVBytes;
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const int c = kk >> 2, off = (kk & 3) * 32;
+          const uint64_t a = tc::sdesc_sw128(tc::smem_u32(Qs + c * (kRowsM * 128) + off), 16, 1024);
           const uint64_t b = tc::sdesc_sw128(tc::smem_u32(kst + c * (kTileN * 128) + off), 16, 1024);
-          mma_bf16_ts(tmem_s + sb * kTileN, tmem_q + kk * 8, b, id_s, kk > 0 ? 1u : 0u);
+          tc::mma_bf16_ss(tmem_s + sb * kTileN, a, b, id_s, kk > 0 ? 1u : 0u);
         }
         tc::mma_commit(&sh.s_full[sb]);
         tc::mma_commit(&sh.k_empty[st]);
       }
       __syncwarp();
-      if (j >= 1) ok = issue_pv(j - 1);
+      return true;
+    };
+    // Issue order S0, S1, S2, PV0, S3, PV1, ...: S_{j+2} is queued before the
+    // P.V of tile j waits on its probabilities, so the tensor pipe stays fed
+    // through the softmax; S_{j+2} reuses the buffer of tile j-1, whose P.V was
+    // issued (and, in issue order, executes) before it.
+    for (int j = 0; j < 2 && j < n_tiles && ok; ++j) ok = issue_s(j);
+    for (int j = 0; j < n_tiles && ok; ++j) {
+      if (j + 2 < n_tiles) ok = issue_s(j + 2);
+      if (ok) ok = issue_pv(j);
     }
-    if (ok) ok = issue_pv(n_tiles - 1);
     if (ok && lane == 0) tc::mma_commit(&sh.o_final);
     if (!ok && lane == 0) set_abort(sh, p.dev_status);
   } else {
@@ -334,46 +352,23 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     const int m = mtile * kRowsM + row;
     const int trow = m / p.G;
     const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
-    constexpr int kDh = D / 2;  // Q elements / output columns this half handles
-
-    // Q row (this half's D/2 elements) into tensor memory as bf16 pairs
-    {
-      const int g = m % p.G;
-      const bool live = m < M;
-      const uint4* qrow = reinterpret_cast<const uint4*>(
-          static_cast<const __nv_bfloat16*>(p.q) +
-          (((size_t)r * p.B + (live ? trow : 0)) * p.Hq + kvh * p.G + g) * D + half * kDh);
-#pragma unroll 1
-      for (int c = 0; c < kDh / 2; c += 16) {  // 16 TMEM columns = 32 bf16 = 4 x 16 B
-        uint32_t w[16];
-#pragma unroll
-        for (int q4 = 0; q4 < 4; ++q4) {
-          const uint4 v = live ? qrow[c / 4 + q4] : make_uint4(0u, 0u, 0u, 0u);
-          w[4 * q4] = v.x;
-          w[4 * q4 + 1] = v.y;
-          w[4 * q4 + 2] = v.z;
-          w[4 * q4 + 3] = v.w;
-        }
-        tmem_st16(tmem_q + lane_off + half * (kDh / 2) + c, w);
-      }
-      tmem_st_wait();
-      tc::fence_before_sync();
-      tc::mbar_arrive(&sh.q_ready);
-    }
+    constexpr int kDh = D / kSplit;       // Q elements / output columns this warp handles
+    constexpr int kCols = kTileN / kSplit;  // key columns of each tile this warp handles
 
     float m_run = -INFINITY, l_run = 0.f;  // l_run: this half's share of the row sum
     bool ok = true;
     for (int j = 0; j < n_tiles; ++j) {
-      const int sb = j & 1;
-      if (!warp_wait(&sh.s_full[sb], (uint32_t)(j >> 1) & 1u, &sh.abort_flag)) {
+      const int sb = j % 3;
+      if (!warp_wait(&sh.s_full[sb], (uint32_t)(j / 3) & 1u, &sh.abort_flag)) {
         ok = false;
         break;
       }
       tc::fence_after_sync();
       const uint32_t sbuf = tmem_s + lane_off + sb * kTileN;
-      uint32_t sr[32];
-      tc::tmem_ld16(sbuf + 32 * half, *reinterpret_cast<uint32_t(*)[16]>(&sr[0]));
-      tc::tmem_ld16(sbuf + 32 * half + 16, *reinterpret_cast<uint32_t(*)[16]>(&sr[16]));
+      uint32_t sr[kCols];
+#pragma unroll
+      for (int c = 0; c < kCols; c += 16)
+        tc::tmem_ld16(sbuf + kCols * half + c, *reinterpret_cast<uint32_t(*)[16]>(&sr[c]));
       tc::tmem_ld_wait();
 
       int pt;
@@ -384,25 +379,27 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
       // tile maximum of the raw scores (scale >= 0 keeps the order)
       float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-      for (int c = 0; c < 32; ++c)
-        if (full || 32 * half + c < lim) mx[c & 3] = fmaxf(mx[c & 3], __uint_as_float(sr[c]));
+      for (int c = 0; c < kCols; ++c)
+        if (full || kCols * half + c < lim) mx[c & 3] = fmaxf(mx[c & 3], __uint_as_float(sr[c]));
       float mt = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
       // the partner has read this slot's previous value before it is overwritten;
       // this exchange also orders both halves' S reads before either writes P.
-      if (j >= 1 && !warp_wait(&sh.xread[quarter], (uint32_t)(j - 1) & 1u, &sh.abort_flag)) {
-        ok = false;
-        break;
+      if (kSplit > 1) {
+        if (j >= 1 && !warp_wait(&sh.xread[quarter], (uint32_t)(j - 1) & 1u, &sh.abort_flag)) {
+          ok = false;
+          break;
+        }
+        sh.xch[half * 128 + row] = mt;
+        tc::fence_before_sync();
+        tc::mbar_arrive(&sh.xbar[quarter]);
+        if (!warp_wait(&sh.xbar[quarter], (uint32_t)j & 1u, &sh.abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc::fence_after_sync();
+        mt = fmaxf(mt, sh.xch[(1 - half) * 128 + row]);
+        tc::mbar_arrive(&sh.xread[quarter]);
       }
-      sh.xch[half * 128 + row] = mt;
-      tc::fence_before_sync();
-      tc::mbar_arrive(&sh.xbar[quarter]);
-      if (!warp_wait(&sh.xbar[quarter], (uint32_t)j & 1u, &sh.abort_flag)) {
-        ok = false;
-        break;
-      }
-      tc::fence_after_sync();
-      mt = fmaxf(mt, sh.xch[(1 - half) * 128 + row]);
-      tc::mbar_arrive(&sh.xread[quarter]);
       const float m_new = fmaxf(m_run, mt * p.scale_log2);
       const bool need = (j == 0) || (m_new > m_run + kRescaleThreshold);
       const bool warp_rescale = __any_sync(0xffffffffu, need);
@@ -411,10 +408,10 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
       const float corr = (j == 0) ? 0.f : tc::ex2(m_run - m_use);
       const float neg_m = -m_use;
       float sum0 = 0.f, sum1 = 0.f;
-      uint32_t pk[16];
+      uint32_t pk[kCols / 2];
       if (full) {
 #pragma unroll
-        for (int c = 0; c < 32; c += 2) {
+        for (int c = 0; c < kCols; c += 2) {
           const float p0 = tc::ex2(fmaf(__uint_as_float(sr[c]), p.scale_log2, neg_m));
           const float p1 = tc::ex2(fmaf(__uint_as_float(sr[c + 1]), p.scale_log2, neg_m));
           sum0 += p0;
@@ -424,8 +421,8 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         }
       } else {
 #pragma unroll
-        for (int c = 0; c < 32; c += 2) {
-          const int col = 32 * half + c;
+        for (int c = 0; c < kCols; c += 2) {
+          const int col = kCols * half + c;
           const float p0 =
               col < lim ? tc::ex2(fmaf(__uint_as_float(sr[c]), p.scale_log2, neg_m)) : 0.f;
           const float p1 =
@@ -440,8 +437,8 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
       l_run = (j == 0) ? sum : l_run * corr + sum;
       // rescale this half's O columns when the running max moved (P.V of tile j-1 done)
       if (warp_rescale && j >= 1) {
-        const int pb = (j - 1) & 1;
-        if (!warp_wait(&sh.pv_done[pb], (uint32_t)((j - 1) >> 1) & 1u, &sh.abort_flag)) {
+        const int pb = (j - 1) % 3;
+        if (!warp_wait(&sh.pv_done[pb], (uint32_t)((j - 1) / 3) & 1u, &sh.abort_flag)) {
           ok = false;
           break;
         }
@@ -457,16 +454,19 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         }
       }
       m_run = m_use;
-      // P (bf16 pairs) over this half's 16 columns of the S buffer
-      tmem_st16(sbuf + 16 * half, pk);
+      // P (bf16 pairs) over this warp's kCols / 2 columns of the S buffer
+#pragma unroll
+      for (int c = 0; c < kCols / 2; c += 16)
+        tmem_st16(sbuf + (kCols / 2) * half + c, *reinterpret_cast<uint32_t(*)[16]>(&pk[c]));
       tmem_st_wait();
       tc::fence_before_sync();
       tc::mbar_arrive(&sh.p_full[sb]);
     }
     // row sum = the two halves' shares
-    if (ok && !warp_wait(&sh.xread[quarter], (uint32_t)(n_tiles - 1) & 1u, &sh.abort_flag))
+    if (kSplit > 1 && ok &&
+        !warp_wait(&sh.xread[quarter], (uint32_t)(n_tiles - 1) & 1u, &sh.abort_flag))
       ok = false;
-    if (ok) {
+    if (kSplit > 1 && ok) {
       sh.xch[half * 128 + row] = l_run;
       tc::mbar_arrive(&sh.xbar[quarter]);
       if (!warp_wait(&sh.xbar[quarter], (uint32_t)n_tiles & 1u, &sh.abort_flag)) ok = false;
@@ -560,6 +560,12 @@ cudaError_t launch_tc_d(const SoftmaxParams& p, const SoftmaxPlan& plan, cudaStr
   using C = TcCfg<D>;
   TcMaps maps;
   const uint64_t e = 2;
+  {
+    const uint64_t dims[4] = {(uint64_t)D, (uint64_t)p.Hq, (uint64_t)p.B, (uint64_t)p.R};
+    const uint64_t str[3] = {D * e, (uint64_t)p.Hq * D * e, (uint64_t)p.B * p.Hq * D * e};
+    const uint32_t box[4] = {64, (uint32_t)p.G, (uint32_t)(kRowsM / p.G), 1};
+    if (!encode4(&maps.q, p.q, dims, str, box)) return cudaErrorInvalidValue;
+  }
   {
     const uint64_t dims[4] = {(uint64_t)D, (uint64_t)p.Hkv, (uint64_t)p.B, (uint64_t)p.R};
     const uint64_t str[3] = {D * e, (uint64_t)p.Hkv * D * e, (uint64_t)p.B * p.Hkv * D * e};
