@@ -16,6 +16,8 @@ of the paper it follows, is documented in the C file:
 * :func:`gather_prefix` -- dense copy of a request's paged prefix.
 * :func:`block_softmax` -- softmax retrieval (Eq. softmax-retrieval) under the
   Diffusion-Trust block mask over the paged prefix plus the block.
+* :func:`append_kv` -- the state-update pass's append of the block's keys and
+  values to the paged cache.
 
 Inputs may be bf16 (passed as raw ``uint16`` bit patterns), fp32 or fp64.
 """
@@ -66,6 +68,8 @@ def _load():
         lib.oracle_gather_prefix.restype = I
         lib.oracle_block_softmax.argtypes = [I] * 8 + [D, I, I, P, P, P, P, P, P, P, P, P, I]
         lib.oracle_block_softmax.restype = I
+        lib.oracle_append_kv.argtypes = [I] * 8 + [P] * 7
+        lib.oracle_append_kv.restype = I
         lib.oracle_max_threads.argtypes = []
         lib.oracle_max_threads.restype = I
         _lib = lib
@@ -218,3 +222,30 @@ def block_softmax(q, k_blk, v_blk, k_pool, v_pool, page_table, prefix_len, *, sc
     if rc != 0:
         raise ValueError("oracle_block_softmax: invalid page id or prefix length")
     return out, lse
+
+
+def append_kv(k_blk, v_blk, k_pool, v_pool, page_table, prefix_len, append_len=None):
+    """Returns copies of (k_pool, v_pool) with the first append_len[r] (default B)
+    block tokens of every request written at prefix positions prefix_len[r] + t.
+    Works on any element type bit for bit (numpy arrays or CPU torch tensors)."""
+    def raw(x):
+        if hasattr(x, "detach"):
+            import torch
+
+            x = x.detach().cpu().contiguous()
+            if x.dtype == torch.bfloat16:
+                return x.view(torch.int16).numpy().view(np.uint16)
+            return x.numpy()
+        return np.ascontiguousarray(x)
+    kb, vb = raw(k_blk), raw(v_blk)
+    kp, vp = raw(k_pool).copy(), raw(v_pool).copy()
+    tab, lens = _i32(page_table), _i32(prefix_len)
+    acc = None if append_len is None else _i32(append_len)
+    R, B, Hkv, D = kb.shape
+    num_pages, _, p, _ = kp.shape
+    rc = _load().oracle_append_kv(R, B, Hkv, D, p, num_pages, tab.shape[1], kb.itemsize,
+                                  _ptr(kb), _ptr(vb), _ptr(kp), _ptr(vp), _ptr(tab), _ptr(lens),
+                                  _ptr(acc))
+    if rc != 0:
+        raise ValueError("oracle_append_kv: invalid page id or length")
+    return kp, vp

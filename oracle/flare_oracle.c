@@ -369,3 +369,45 @@ int oracle_block_softmax(int R, int B, int Hq, int Hkv, int D, int page_size, in
   }
   return 0;
 }
+
+/*
+ * KV append of the state-update pass (serving appendix: after the last denoise
+ * step the token-causal pass appends the block's keys and values to the cache):
+ * for request r the first n = append_len[r] block tokens (all B when
+ * append_len is NULL) go to prefix positions prefix_len[r] + t, i.e. page
+ * page_table[r][(P + t) / page_size], row (P + t) % page_size, of both pools
+ * ([num_pages, Hkv, page_size, D]).  Elements are copied bit for bit; nothing
+ * else in the pools changes and prefix_len is not updated (that is the
+ * caller's bookkeeping).  elem_bytes is the size of one element.
+ * Returns -1 (and writes nothing) if any request's range or page is invalid.
+ */
+int oracle_append_kv(int R, int B, int Hkv, int D, int page_size, int num_pages, int max_pages,
+                     int elem_bytes, const void* k_blk, const void* v_blk, void* k_pool,
+                     void* v_pool, const int32_t* page_table, const int32_t* prefix_len,
+                     const int32_t* append_len) {
+  for (int r = 0; r < R; ++r) {
+    const int P = prefix_len[r];
+    const int n = append_len ? append_len[r] : B;
+    if (n < 0 || n > B || P < 0 || P + n > max_pages * page_size) return -1;
+    for (int t = 0; t < n; ++t) {
+      const int page = page_table[(size_t)r * max_pages + (P + t) / page_size];
+      if (page < 0 || page >= num_pages) return -1;
+    }
+  }
+  const size_t row = (size_t)D * elem_bytes;
+  for (int r = 0; r < R; ++r) {
+    const int P = prefix_len[r];
+    const int n = append_len ? append_len[r] : B;
+    for (int t = 0; t < n; ++t) {
+      const int pos = P + t;
+      const int page = page_table[(size_t)r * max_pages + pos / page_size];
+      for (int hk = 0; hk < Hkv; ++hk) {
+        const size_t dst = (((size_t)page * Hkv + hk) * page_size + pos % page_size) * row;
+        const size_t src = (((size_t)r * B + t) * Hkv + hk) * row;
+        memcpy((char*)k_pool + dst, (const char*)k_blk + src, row);
+        memcpy((char*)v_pool + dst, (const char*)v_blk + src, row);
+      }
+    }
+  }
+  return 0;
+}

@@ -373,3 +373,50 @@ def test_softmax_rejects_bad_page():
     c["table"][2, 0] = c["kp"].shape[0]
     with pytest.raises(ValueError):
         oracle.block_softmax(c["q"], c["kb"], c["vb"], c["kp"], c["vp"], c["table"], c["lens"])
+
+
+# ---------------------------------------------------------------- KV append
+
+
+def test_append_then_gather_is_prefix_plus_block():
+    """The state-update pass appends the block to the cache: gathering the
+    longer prefix returns the old prefix followed by the appended tokens, and
+    no other pool row changes."""
+    c = _paged_case(R=3, B=4, lens=(5, 0, 12), p=4, seed=21, poison=True)
+    # give every request room for the block: extra pages after its last one
+    R, B, Hkv, D = c["kb"].shape
+    num_pages = c["kp"].shape[0]
+    extra = num_pages
+    kp = np.concatenate([c["kp"], np.full((6,) + c["kp"].shape[1:], np.nan)], 0)
+    vp = np.concatenate([c["vp"], np.full((6,) + c["vp"].shape[1:], np.nan)], 0)
+    table = -np.ones((R, 8), np.int32)
+    table[:, :c["table"].shape[1]] = c["table"]
+    for r, P in enumerate(c["lens"]):
+        first_free = -(-int(P) // 4)
+        for q in range(first_free, -(-(int(P) + B) // 4)):
+            table[r, q] = extra
+            extra += 1
+    append = np.array([4, 2, 0], np.int32)
+    k2, v2 = oracle.append_kv(c["kb"], c["vb"], kp, vp, table, c["lens"], append)
+    for r in range(R):
+        P, n = int(c["lens"][r]), int(append[r])
+        got = oracle.gather_prefix(r, k2, table, c["lens"] + append, 4)
+        want = np.concatenate([c["dense_k"][r], c["kb"][r, :n]], 0)
+        assert np.array_equal(got, want)
+    # rows outside the appended positions are bit-identical (NaN included)
+    touched = np.zeros(kp.shape[0] * 4, bool)
+    for r in range(R):
+        for t in range(int(append[r])):
+            pos = int(c["lens"][r]) + t
+            touched[table[r, pos // 4] * 4 + pos % 4] = True
+    same = lambda a, b: np.array_equal(a.view(np.uint64), b.view(np.uint64))
+    for pg in range(kp.shape[0]):
+        for row in range(4):
+            if not touched[pg * 4 + row]:
+                assert same(k2[pg, :, row], kp[pg, :, row]) and same(v2[pg, :, row], vp[pg, :, row])
+
+
+def test_append_rejects_overflow():
+    c = _paged_case(R=3, B=4, lens=(5, 0, 12), p=4, seed=22)
+    with pytest.raises(ValueError):
+        oracle.append_kv(c["kb"], c["vb"], c["kp"], c["vp"], c["table"], c["lens"])
