@@ -191,6 +191,32 @@ flare_status flare_block_softmax_attn(const flare_softmax_desc* desc, const void
                                       void* workspace, size_t workspace_bytes,
                                       int32_t* dev_status, void* stream);
 
+/*
+ * KV append of the state-update pass (serving appendix, Diffusion-Trust
+ * serving loop: after the last denoise step the token-causal pass writes the
+ * recurrent state back and appends the block's keys and values to the cache).
+ * For request r the first n = append_len[r] block tokens (all B when
+ * append_len is NULL) are copied bit for bit to prefix positions
+ * prefix_len[r] + t, t < n, i.e. page page_table[r][(P + t) / p], row
+ * (P + t) % p of both pools.  Page allocation is the caller's: the table
+ * entries for those positions must already name pages.  prefix_len is not
+ * updated (advance it by n afterwards).  Nothing else in the pools changes.
+ *   k_blk, v_blk   [R, B, Hkv, D]             act_dtype (desc->act_dtype)
+ *   k_pool, v_pool [num_pages, Hkv, p, D]     act_dtype, written in place
+ *   page_table     [R, max_pages_per_req]     int32
+ *   prefix_len     [R]                        int32
+ *   append_len     [R]                        int32 in [0, B], nullable
+ *   dev_status     FLARE_DEV_BAD_ACCEPT_LEN (n out of range),
+ *                  FLARE_DEV_BAD_PREFIX_LEN (P + n beyond the table),
+ *                  FLARE_DEV_BAD_PAGE; the request is skipped.
+ * Only the shape fields, page_size, num_pages, max_pages_per_req and
+ * act_dtype of desc are used.
+ */
+flare_status flare_append_kv(const flare_softmax_desc* desc, const void* k_blk, const void* v_blk,
+                             void* k_pool, void* v_pool, const int32_t* page_table,
+                             const int32_t* prefix_len, const int32_t* append_len,
+                             int32_t* dev_status, void* stream);
+
 /* Size of the library-owned scratch array used by flare_block_softmax_attn_noalloc. */
 #define FLARE_NOALLOC_SCRATCH_BYTES (64u * 1024u * 1024u)
 

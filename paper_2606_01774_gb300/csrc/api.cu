@@ -283,6 +283,29 @@ flare_status flare_block_softmax_attn(const flare_softmax_desc* d, const void* q
   return e == cudaSuccess ? FLARE_OK : FLARE_ERR_CUDA;
 }
 
+flare_status flare_append_kv(const flare_softmax_desc* d, const void* k_blk, const void* v_blk,
+                             void* k_pool, void* v_pool, const int32_t* page_table,
+                             const int32_t* prefix_len, const int32_t* append_len,
+                             int32_t* dev_status, void* stream) {
+  flare_status st = check_softmax(d);
+  if (st != FLARE_OK) return st;
+  if (!k_blk || !v_blk || !k_pool || !v_pool || !page_table || !prefix_len || !dev_status)
+    return FLARE_ERR_INVALID_ARGUMENT;
+  if (!aligned16(k_blk) || !aligned16(v_blk) || !aligned16(k_pool) || !aligned16(v_pool))
+    return FLARE_ERR_INVALID_ARGUMENT;
+  if (d->num_requests == 0) return FLARE_OK;
+  SoftmaxParams p = softmax_params(d);
+  p.k_blk = k_blk;
+  p.v_blk = v_blk;
+  p.page_table = page_table;
+  p.prefix_len = prefix_len;
+  p.dev_status = dev_status;
+  const int elem = d->act_dtype == FLARE_DT_BF16 ? 2 : 4;
+  const cudaError_t e = launch_append_kv(p, append_len, k_pool, v_pool, elem,
+                                         static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? FLARE_OK : FLARE_ERR_CUDA;
+}
+
 flare_status flare_debug_gather_prefix(const flare_softmax_desc* d, const void* k_pool,
                                        const void* v_pool, const int32_t* page_table,
                                        const int32_t* prefix_len, int32_t request, void* k_out,

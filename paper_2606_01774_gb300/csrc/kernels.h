@@ -75,6 +75,8 @@ cudaError_t launch_softmax_tc(const SoftmaxParams& p, const SoftmaxPlan& plan,
                               cudaStream_t stream);
 cudaError_t launch_softmax_combine(const SoftmaxParams& p, bool bf16, cudaStream_t stream);
 bool softmax_tc_supported(int B, int Hq, int Hkv, int D, int page_size);
+cudaError_t launch_append_kv(const SoftmaxParams& p, const int32_t* append_len, void* k_pool,
+                             void* v_pool, int elem_bytes, cudaStream_t stream);
 cudaError_t launch_gather_prefix(const SoftmaxParams& p, int request, void* k_out, void* v_out,
                                  bool bf16, cudaStream_t stream);
 

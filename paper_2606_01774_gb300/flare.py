@@ -79,6 +79,7 @@ def load() -> ctypes.CDLL:
         "flare_softmax_workspace_size": [smx, ctypes.POINTER(S)],
         "flare_block_softmax_attn": [smx] + [P] * 10 + [S, P, P],
         "flare_block_softmax_attn_noalloc": [smx] + [P] * 11,
+        "flare_append_kv": [smx] + [P] * 9,
         "flare_debug_gather_prefix": [smx, P, P, P, P, I32, P, P, P, P],
         "flare_read_status": [P, P, ctypes.POINTER(I32)],
     }
@@ -154,6 +155,13 @@ def flare_block_softmax_attn(desc, q, k_blk, v_blk, k_pool, v_pool, page_table, 
         ctypes.byref(desc), _p(q), _p(k_blk), _p(v_blk), _p(k_pool), _p(v_pool), _p(page_table),
         _p(prefix_len), _p(out), _p(lse), _p(workspace), int(workspace_bytes), _p(dev_status),
         _stream(stream))
+
+
+def flare_append_kv(desc, k_blk, v_blk, k_pool, v_pool, page_table, prefix_len, append_len,
+                    dev_status, stream=None) -> int:
+    return load().flare_append_kv(
+        ctypes.byref(desc), _p(k_blk), _p(v_blk), _p(k_pool), _p(v_pool), _p(page_table),
+        _p(prefix_len), _p(append_len), _p(dev_status), _stream(stream))
 
 
 FLARE_NOALLOC_SCRATCH_BYTES = 64 * 1024 * 1024
