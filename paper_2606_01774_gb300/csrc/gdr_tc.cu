@@ -7,9 +7,8 @@
 //
 //   gamma_t = sum_{i<=t} g_i,  Gam_t = exp(gamma_t)             (cumulative log-gate)
 //   A[t][i] = beta_t exp(gamma_t - gamma_i) (k_t . k_i),  i < t
-//   T       = (I + A)^{-1}                                     (unit lower triangular)
 //   X       = diag(beta) (V - diag(Gam) K S0)
-//   delta   = T X                                              (per-step delta updates)
+//   (I + A) delta = X                                          (per-step delta updates)
 //   out[l]  = s (Gam_B S0^T q_l + sum_i exp(gamma_B - gamma_i) (q_l . k_i) delta_i)
 //
 // Every product with S0 or delta is computed transposed, with the value
@@ -19,16 +18,16 @@
 //
 //   MMA 1   G   = [K;Q] K^T          M=128 (64 k rows, 64 q rows), N=Bp, K=dk
 //   MMA 2   W^T = S0^T [K;Q]^T       M=128 (c),  N=128, K=dk   (S0^T is MN-major)
-//   solve   T   = (I + A)^{-1}       blocked by 16: diagonal blocks by forward
-//                                    substitution, off-diagonal blocks on
-//                                    warp-level tf32 MMA
-//   MMA 3   delta^T = X^T T^T        M=128 (c),  N=Bp,  K=Bp
+//   solve   (I + A) delta = X        unit lower triangular, 16 rows at a time:
+//                                    off-diagonal terms on warp-level tf32 MMA,
+//                                    diagonal blocks by fp32 forward substitution
 //   MMA 4   O2^T = delta^T M2^T      M=128 (c),  N=Bp,  K=Bp, M2[l][i] = exp(gamma_B-gamma_i) q_l.k_i
 //   out[l][c] = s (Gam_B W^T[c][64+l] + O2^T[c][l])
 //
-// Inputs bf16, state fp32 read once and rounded to bf16 for the MMA, all
-// accumulation fp32.  One CTA per (request, value head); 128 threads; 97 KiB
-// shared memory and 256 TMEM columns, so two CTAs share an SM.
+// Bp = B rounded up to 16.  Inputs bf16, state fp32 read once and rounded to
+// bf16 for the MMA, all accumulation fp32.  One CTA per (request, value
+// head); 128 threads; 107 KiB shared memory and 256 TMEM
+// columns, so two CTAs share an SM.
 #include <cudaTypedefs.h>
 
 #include "common.cuh"
@@ -41,15 +40,21 @@ namespace {
 
 constexpr int kLinThreads = 128;
 constexpr int kBmax = 64;
+constexpr int kATs = kBmax + 8;  // row stride of A^T: conflict-free tf32 fragment loads
 
 template <int DK, int DV>
 struct LinCfg {
   static constexpr int kKQ = (DK / 64) * 128 * 128;  // [K;Q]: DK/64 chunks of 128 rows x 128 B
-  static constexpr int kS0 = 2 * DK * 128;           // S0^T, MN-major: 2 chunks of DK rows x 128 B
-  static constexpr int kM2 = kBmax * 128;             // [l][i] K-major
-  static constexpr int kT = kBmax * 128;              // [t][i] K-major
-  static constexpr int kX = 128 * 128;                // X^T / delta^T [c][t] K-major; also A (fp32 64x64)
-  static constexpr int kSmem = kKQ + kS0 + kM2 + kT + kX;
+  static constexpr int kAT = kBmax * kATs * 4;       // A^T fp32 [i][t], row stride kATs
+  static constexpr int kR1 = kKQ > kAT ? kKQ : kAT;  // [K;Q], then A^T
+  static constexpr int kS0 = (DV / 64) * DK * 128;   // S0^T, MN-major: DV/64 chunks of DK rows x 128 B
+  static constexpr int kDs = DV + 8;                 // row stride of delta fp32
+  static constexpr int kD32 = kBmax * kDs * 4;       // delta fp32 [t][c]
+  static constexpr int kR2 = kS0 > kD32 ? kS0 : kD32;  // S0^T, then delta
+  static constexpr int kV = (DV / 64) * kBmax * 128;  // V [t][c], DV/64 chunks of 64 rows x 128 B
+  static constexpr int kM2 = kBmax * 128;             // M2 [l][i] K-major
+  static constexpr int kD = 128 * 128;                // delta^T [c][t] K-major
+  static constexpr int kSmem = kR1 + kR2 + kV + kM2 + kD;
 };
 
 struct LinShared {
@@ -123,13 +128,12 @@ __global__ void __launch_bounds__(kLinThreads, 2)
   __shared__ LinShared sh;
   uint8_t* base = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t* KQs = base;
-  uint8_t* S0s = KQs + C::kKQ;
-  uint8_t* M2s = S0s + C::kS0;
-  uint8_t* Ts = M2s + C::kM2;
-  uint8_t* Xs = Ts + C::kT;
-  float* A32 = reinterpret_cast<float*>(Xs);   // aliases X^T (A is dead before X is written)
-  float* T32 = reinterpret_cast<float*>(KQs);  // fp32 T, in [K;Q] once MMA 1/2 have run
-  float* Ytmp = reinterpret_cast<float*>(Ts);  // 4 x 256 floats, dead until T is converted
+  uint8_t* S0s = KQs + C::kR1;
+  uint8_t* Vs = S0s + C::kR2;
+  uint8_t* M2s = Vs + C::kV;
+  uint8_t* Ds = M2s + C::kM2;
+  float* AT = reinterpret_cast<float*>(KQs);   // A^T[i][t], once MMA 1/2 have run
+  float* D32 = reinterpret_cast<float*>(S0s);  // delta[t][c], once MMA 2 has run
 
   const int item = blockIdx.x;
   const int r = item / p.Hv, j = item % p.Hv;
@@ -172,7 +176,7 @@ __global__ void __launch_bounds__(kLinThreads, 2)
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = sh.tmem_base;
-  const uint32_t tmA = tmem;        // G, then delta^T, then O2^T   (64 columns)
+  const uint32_t tmA = tmem;        // G, then O2^T                 (64 columns)
   const uint32_t tmW = tmem + 128;  // W^T = S0^T [K;Q]^T           (128 columns)
   const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
 
@@ -182,6 +186,9 @@ __global__ void __launch_bounds__(kLinThreads, 2)
       tc::tma_load_4d(KQs + c * 16384, &maps.k, &sh.bar_kq, c * 64, h, 0, r);
       tc::tma_load_4d(KQs + c * 16384 + 8192, &maps.q, &sh.bar_kq, c * 64, h, 0, r);
     }
+    tc::mbar_expect_tx(&sh.bar_v, (DV / 64) * kBmax * 128);
+    for (int c = 0; c < DV / 64; ++c)
+      tc::tma_load_4d(Vs + c * (kBmax * 128), &maps.v, &sh.bar_v, c * 64, j, 0, r);
   }
 
   // S0 (fp32, global) -> bf16 S0^T operand, MN-major 128-byte swizzle:
@@ -243,20 +250,14 @@ __global__ void __launch_bounds__(kLinThreads, 2)
   }
   if (!lin_wait(&sh.bar_mma, 0, sh, p.dev_status)) goto done;
   tc::fence_after_sync();
-  // the S0^T operand is dead: stage the V tile there while A, M2 and T are built
-  if (tid == 0) {
-    tc::mbar_expect_tx(&sh.bar_v, (DV / 64) * kBmax * 128);
-    for (int c = 0; c < DV / 64; ++c)
-      tc::tma_load_4d(S0s + c * (kBmax * 128), &maps.v, &sh.bar_v, c * 64, j, 0, r);
-  }
 
-  // ---- A (rows 0..63 of G) and M2 (rows 64..127), 16 columns at a time
+  // ---- A^T (from rows 0..63 of G, fp32) and M2 (rows 64..127, bf16 operand)
   {
     const int row = tid & 63;
     const float gB = sh.gam2[B - 1];
     const float bt = sh.beta[row], gt = sh.gam2[row];
 #pragma unroll 1
-    for (int c0 = 0; c0 < 64; c0 += 16) {
+    for (int c0 = 0; c0 < Bp; c0 += 16) {
       uint32_t gr[16];
       tc::tmem_ld16(tmA + lane_off + c0, gr);
       tc::tmem_ld_wait();
@@ -265,12 +266,10 @@ __global__ void __launch_bounds__(kLinThreads, 2)
 #pragma unroll
         for (int e = 0; e < 16; ++e) {
           const int i = c0 + e;
-          v[e] = (i < row && row < B) ? bt * tc::ex2(gt - sh.gam2[i]) * __uint_as_float(gr[e]) : 0.f;
+          // A[t][i] = beta_t exp(gamma_t - gamma_i) (k_t . k_i), i < t < B
+          AT[i * kATs + row] =
+              (i < row && row < B) ? bt * tc::ex2(gt - sh.gam2[i]) * __uint_as_float(gr[e]) : 0.f;
         }
-        float4* arow = reinterpret_cast<float4*>(A32 + row * 64 + c0);
-#pragma unroll
-        for (int q4 = 0; q4 < 4; ++q4)
-          arow[q4] = make_float4(v[4 * q4], v[4 * q4 + 1], v[4 * q4 + 2], v[4 * q4 + 3]);
       } else {
 #pragma unroll
         for (int e = 0; e < 16; ++e) {
@@ -281,162 +280,93 @@ __global__ void __launch_bounds__(kLinThreads, 2)
       }
     }
   }
-  // T32 (fp32 [64][64], in the dead [K;Q] operand) starts at zero
-  {
-    float4* t4 = reinterpret_cast<float4*>(T32);
-#pragma unroll
-    for (int n = 0; n < 64 * 64 / 4 / kLinThreads; ++n)
-      t4[tid + n * kLinThreads] = make_float4(0.f, 0.f, 0.f, 0.f);
-  }
-  tc::fence_before_sync();
-  __syncthreads();
+  if (!lin_wait(&sh.bar_v, 0, sh, p.dev_status)) goto done;  // also publishes A^T
 
-  // ---- T = (I + A)^{-1}, blocked by 16 (A is strictly lower triangular).
-  // Diagonal blocks: thread (blk, col) solves (I + A_kk) x = e_col by forward
-  // substitution, x kept in its own column of T32 (rolled loops: this code runs
-  // once per CTA, so it is kept small).
-  if (tid < 64) {
-    const int blk = tid >> 4, col = tid & 15, o = blk * 16;
-    float* xcol = T32 + o * 64 + o + col;          // x[i] at xcol[i * 64]
-    const float* arow0 = A32 + o * 64 + o;         // A_kk[t][i] at arow0[t * 64 + i]
-    xcol[col * 64] = 1.f;
-#pragma unroll 1
-    for (int t = col + 1; t < 16; ++t) {
-      float a0 = 0.f, a1 = 0.f;
-      int i = col;
-#pragma unroll 1
-      for (; i + 1 < t; i += 2) {
-        a0 = fmaf(arow0[t * 64 + i], xcol[i * 64], a0);
-        a1 = fmaf(arow0[t * 64 + i + 1], xcol[(i + 1) * 64], a1);
-      }
-      if (i < t) a0 = fmaf(arow0[t * 64 + i], xcol[i * 64], a0);
-      xcol[t * 64] = -(a0 + a1);
-    }
-  }
-  __syncthreads();
-  // Off-diagonal blocks by distance d = i - j:  T_ij = -T_ii sum_{k=j}^{i-1} A_ik T_kj.
-  // One warp per block, 16x16 tiles on warp-level tf32 MMA (m16n8k8); Y goes
-  // through shared memory to change from accumulator to operand layout.
-#pragma unroll 1
-  for (int d = 1; d < 4; ++d) {
-    const int bj = warp, bi = bj + d;
-    if (bi < 4) {
-      const int g = lane >> 2, q = lane & 3;
-      float y[2][4];
-#pragma unroll
-      for (int nt = 0; nt < 2; ++nt) {
-#pragma unroll
-        for (int e = 0; e < 4; ++e) y[nt][e] = 0.f;
-      }
-      // Y = sum_k A_{bi,k} T_{k,bj}, k over the 16*d rows between the blocks
-#pragma unroll 1
-      for (int k8 = 16 * bj; k8 < 16 * bi; k8 += 8) {
-        const float* ar = A32 + (16 * bi + g) * 64 + k8 + q;
-        const uint32_t a0 = f2tf32(ar[0]), a1 = f2tf32(ar[8 * 64]);
-        const uint32_t a2 = f2tf32(ar[4]), a3 = f2tf32(ar[8 * 64 + 4]);
-#pragma unroll
-        for (int nt = 0; nt < 2; ++nt) {
-          const float* br = T32 + (k8 + q) * 64 + 16 * bj + nt * 8 + g;
-          mma_tf32(y[nt], a0, a1, a2, a3, f2tf32(br[0]), f2tf32(br[4 * 64]));
-        }
-      }
-      float* Yw = Ytmp + warp * 256;  // 16 x 16
-#pragma unroll
-      for (int nt = 0; nt < 2; ++nt) {
-        Yw[g * 16 + nt * 8 + 2 * q] = y[nt][0];
-        Yw[g * 16 + nt * 8 + 2 * q + 1] = y[nt][1];
-        Yw[(g + 8) * 16 + nt * 8 + 2 * q] = y[nt][2];
-        Yw[(g + 8) * 16 + nt * 8 + 2 * q + 1] = y[nt][3];
-      }
-      __syncwarp();
-      // T_ij = -T_ii Y
-      float t[2][4];
-#pragma unroll
-      for (int nt = 0; nt < 2; ++nt) {
-#pragma unroll
-        for (int e = 0; e < 4; ++e) t[nt][e] = 0.f;
-      }
-#pragma unroll
-      for (int k8 = 0; k8 < 16; k8 += 8) {
-        const float* ar = T32 + (16 * bi + g) * 64 + 16 * bi + k8 + q;
-        const uint32_t a0 = f2tf32(ar[0]), a1 = f2tf32(ar[8 * 64]);
-        const uint32_t a2 = f2tf32(ar[4]), a3 = f2tf32(ar[8 * 64 + 4]);
-#pragma unroll
-        for (int nt = 0; nt < 2; ++nt) {
-          const float* br = Yw + (k8 + q) * 16 + nt * 8 + g;
-          mma_tf32(t[nt], a0, a1, a2, a3, f2tf32(br[0]), f2tf32(br[4 * 16]));
-        }
-      }
-      float* to = T32 + (16 * bi) * 64 + 16 * bj;
-#pragma unroll
-      for (int nt = 0; nt < 2; ++nt) {
-        to[g * 64 + nt * 8 + 2 * q] = -t[nt][0];
-        to[g * 64 + nt * 8 + 2 * q + 1] = -t[nt][1];
-        to[(g + 8) * 64 + nt * 8 + 2 * q] = -t[nt][2];
-        to[(g + 8) * 64 + nt * 8 + 2 * q + 1] = -t[nt][3];
-      }
-    }
-    __syncthreads();
-  }
-  // T (bf16) into the K-major operand tile, one row per thread
-  if (tid < 64) {
-#pragma unroll 1
-    for (int c0 = 0; c0 < 64; c0 += 16) {
-      float v[16];
-#pragma unroll
-      for (int e = 0; e < 16; ++e) v[e] = T32[tid * 64 + c0 + e];
-      store16_sw128(Ts, tid, c0, v);
-    }
-  }
-  __syncthreads();  // A is dead from here on; its buffer becomes X^T
-
-  // ---- X^T[c][t] = beta_t (V[t][c] - Gam_t (K S0)[t][c])
+  // ---- delta = (I + A)^{-1} X by forward substitution, X = diag(beta)(V - diag(Gam) K S0).
+  // The system acts on each column c on its own; warp w owns columns
+  // 32w..32w+31 and walks the rows 16 at a time:
+  //   x_b  = X_b - A[b, <b] delta_<b     warp-level tf32 MMA (rows x columns tile)
+  //   delta_b = (I + A[b,b])^{-1} x_b    fp32 forward substitution, thread c on column c
+  // The two layouts meet in the fp32 delta buffer, inside the warp.
   {
+    constexpr int kS = C::kDs;
     const int c = tid;
-    if (!lin_wait(&sh.bar_v, 0, sh, p.dev_status)) goto done;
-    const uint8_t* vcol = S0s + ((c & (DV - 1)) >> 6) * (kBmax * 128) + (c & 63) * 2;
+    const bool col_ok = c < DV;  // warp-uniform
+    const int g = lane >> 2, q = lane & 3;
+    const uint8_t* vcol = Vs + ((c & (DV - 1)) >> 6) * (kBmax * 128) + (c & 63) * 2;
 #pragma unroll 1
-    for (int c0 = 0; c0 < 64; c0 += 16) {
+    for (int b0 = 0; b0 < Bp; b0 += 16) {
       uint32_t w[16];
-      tc::tmem_ld16(tmW + lane_off + c0, w);  // (K S0)^T[c][t]
+      tc::tmem_ld16(tmW + lane_off + b0, w);  // (K S0)^T[c][t]
       tc::tmem_ld_wait();
-      float xv[16];
+      float x[16];
 #pragma unroll
       for (int e = 0; e < 16; ++e) {
-        const int t = c0 + e;
+        const int t = b0 + e;
         const float vt =
             __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(vcol + t * 128));
-        xv[e] = (t < B && c < DV) ? sh.beta[t] * (vt - sh.Gam[t] * __uint_as_float(w[e])) : 0.f;
+        x[e] = (t < B && col_ok) ? sh.beta[t] * (vt - sh.Gam[t] * __uint_as_float(w[e])) : 0.f;
       }
-      store16_sw128(Xs, c, c0, xv);
-    }
-  }
-  tc::fence_async_smem();
-  tc::fence_before_sync();
-  __syncthreads();
-
-  // ---- MMA 3: delta^T = X^T T^T
-  if (tid == 0) {
-    tc::fence_after_sync();
-    const uint32_t id = tc::idesc_bf16(128, Bp, false, false);
-    for (int kk = 0; kk < Bp / 16; ++kk) {
-      const uint64_t a = tc::sdesc_sw128(tc::smem_u32(Xs + kk * 32), 16, 1024);
-      const uint64_t b = tc::sdesc_sw128(tc::smem_u32(Ts + kk * 32), 16, 1024);
-      tc::mma_bf16_ss(tmA, a, b, id, kk > 0);
-    }
-    tc::mma_commit(&sh.bar_mma);
-  }
-  if (!lin_wait(&sh.bar_mma, 1, sh, p.dev_status)) goto done;
-  tc::fence_after_sync();
-#pragma unroll 1
-  for (int c0 = 0; c0 < 64; c0 += 16) {
-    uint32_t dd[16];
-    tc::tmem_ld16(tmA + lane_off + c0, dd);
-    tc::tmem_ld_wait();
-    float v[16];
+      if (col_ok) {
+        if (b0 > 0) {
+          // x_b -= A[b0.., 0..b0) delta[0..b0, warp's columns]
 #pragma unroll
-    for (int e = 0; e < 16; ++e) v[e] = (c0 + e < B) ? __uint_as_float(dd[e]) : 0.f;
-    store16_sw128(Xs, tid, c0, v);  // delta^T replaces X^T (MMA 3 has completed)
+          for (int e = 0; e < 16; ++e) D32[(b0 + e) * kS + c] = x[e];
+          __syncwarp();
+          const int cw = warp * 32;
+          float acc[4][4];
+#pragma unroll
+          for (int nt = 0; nt < 4; ++nt) {
+            const float2 lo = *reinterpret_cast<const float2*>(D32 + (b0 + g) * kS + cw + nt * 8 + 2 * q);
+            const float2 hi = *reinterpret_cast<const float2*>(D32 + (b0 + g + 8) * kS + cw + nt * 8 + 2 * q);
+            acc[nt][0] = lo.x;
+            acc[nt][1] = lo.y;
+            acc[nt][2] = hi.x;
+            acc[nt][3] = hi.y;
+          }
+#pragma unroll 1
+          for (int i0 = 0; i0 < b0; i0 += 8) {
+            // -A[t][i] = -A^T[i][t]
+            const float* ar = AT + (i0 + q) * kATs + b0 + g;
+            const uint32_t a0 = f2tf32(-ar[0]), a1 = f2tf32(-ar[8]);
+            const uint32_t a2 = f2tf32(-ar[4 * kATs]), a3 = f2tf32(-ar[4 * kATs + 8]);
+#pragma unroll
+            for (int nt = 0; nt < 4; ++nt) {
+              const float* br = D32 + (i0 + q) * kS + cw + nt * 8 + g;
+              mma_tf32(acc[nt], a0, a1, a2, a3, f2tf32(br[0]), f2tf32(br[4 * kS]));
+            }
+          }
+          __syncwarp();
+#pragma unroll
+          for (int nt = 0; nt < 4; ++nt) {
+            *reinterpret_cast<float2*>(D32 + (b0 + g) * kS + cw + nt * 8 + 2 * q) =
+                make_float2(acc[nt][0], acc[nt][1]);
+            *reinterpret_cast<float2*>(D32 + (b0 + g + 8) * kS + cw + nt * 8 + 2 * q) =
+                make_float2(acc[nt][2], acc[nt][3]);
+          }
+          __syncwarp();
+#pragma unroll
+          for (int e = 0; e < 16; ++e) x[e] = D32[(b0 + e) * kS + c];
+        }
+        // diagonal block: x_t -= A[t][i] delta_i for b0 <= i < t
+#pragma unroll
+        for (int e = 0; e < 15; ++e) {
+          const float4* a4 = reinterpret_cast<const float4*>(AT + (b0 + e) * kATs + b0);
+#pragma unroll
+          for (int qq = e / 4; qq < 4; ++qq) {
+            const float4 a = a4[qq];
+            if (4 * qq > e) x[4 * qq] = fmaf(-a.x, x[e], x[4 * qq]);
+            if (4 * qq + 1 > e) x[4 * qq + 1] = fmaf(-a.y, x[e], x[4 * qq + 1]);
+            if (4 * qq + 2 > e) x[4 * qq + 2] = fmaf(-a.z, x[e], x[4 * qq + 2]);
+            if (4 * qq + 3 > e) x[4 * qq + 3] = fmaf(-a.w, x[e], x[4 * qq + 3]);
+          }
+        }
+#pragma unroll
+        for (int e = 0; e < 16; ++e) D32[(b0 + e) * kS + c] = x[e];
+        __syncwarp();  // the next block's MMA reads this block's delta across the warp
+      }
+      store16_sw128(Ds, c, b0, x);  // delta^T, bf16 operand of MMA 4
+    }
   }
   tc::fence_async_smem();
   tc::fence_before_sync();
@@ -447,13 +377,13 @@ __global__ void __launch_bounds__(kLinThreads, 2)
     tc::fence_after_sync();
     const uint32_t id = tc::idesc_bf16(128, Bp, false, false);
     for (int kk = 0; kk < Bp / 16; ++kk) {
-      const uint64_t a = tc::sdesc_sw128(tc::smem_u32(Xs + kk * 32), 16, 1024);
+      const uint64_t a = tc::sdesc_sw128(tc::smem_u32(Ds + kk * 32), 16, 1024);
       const uint64_t b = tc::sdesc_sw128(tc::smem_u32(M2s + kk * 32), 16, 1024);
       tc::mma_bf16_ss(tmA, a, b, id, kk > 0);
     }
     tc::mma_commit(&sh.bar_mma);
   }
-  if (!lin_wait(&sh.bar_mma, 0, sh, p.dev_status)) goto done;
+  if (!lin_wait(&sh.bar_mma, 1, sh, p.dev_status)) goto done;
   tc::fence_after_sync();
   {
     const int c = tid;
@@ -461,7 +391,7 @@ __global__ void __launch_bounds__(kLinThreads, 2)
     __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.out_blockend) +
                          ((size_t)r * B * p.Hv + j) * DV + c;
 #pragma unroll 1
-    for (int c0 = 0; c0 < 64; c0 += 16) {
+    for (int c0 = 0; c0 < Bp; c0 += 16) {
       uint32_t o2[16], wq[16];
       tc::tmem_ld16(tmA + lane_off + c0, o2);
       tc::tmem_ld16(tmW + lane_off + 64 + c0, wq);  // (Q S0)^T[c][l]
