@@ -157,7 +157,8 @@ flare_status flare_commit_state(const flare_linear_desc* desc, const void* q, co
 
 /*
  * Bytes of device workspace flare_block_softmax_attn needs for `desc`
- * (partial outputs of split prefixes).  May be 0.  Host-only, no GPU work.
+ * (the longest-first order of the work units and the partial outputs of split
+ * prefixes).  May be 0.  Host-only, no GPU work.
  */
 flare_status flare_softmax_workspace_size(const flare_softmax_desc* desc, size_t* bytes);
 

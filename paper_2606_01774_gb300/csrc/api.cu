@@ -128,7 +128,9 @@ SoftmaxPlan plan_softmax(int R, int B, int Hq, int Hkv, int D, int page_size, in
     pl.ws_o_bytes = (rows * D * sizeof(float) + 255) / 256 * 256;
     pl.ws_lse_bytes = (rows * sizeof(float) + 255) / 256 * 256;
   }
-  pl.workspace_bytes = pl.ws_o_bytes + pl.ws_lse_bytes;
+  // tensor-core kernel: the work units in longest-first order
+  if (pl.kernel == 1) pl.ws_order_bytes = ((size_t)R * pl.n_split * sizeof(int32_t) + 255) / 256 * 256;
+  pl.workspace_bytes = pl.ws_o_bytes + pl.ws_lse_bytes + pl.ws_order_bytes;
   return pl;
 }
 
@@ -274,8 +276,13 @@ flare_status flare_block_softmax_attn(const flare_softmax_desc* d, const void* q
   p.n_split = plan.n_split;
   p.split_len = plan.split_len;
   if (plan.workspace_bytes) {
-    p.ws_o = static_cast<float*>(workspace);
-    p.ws_lse = reinterpret_cast<float*>(static_cast<char*>(workspace) + plan.ws_o_bytes);
+    char* ws = static_cast<char*>(workspace);
+    if (plan.ws_o_bytes) {
+      p.ws_o = reinterpret_cast<float*>(ws);
+      p.ws_lse = reinterpret_cast<float*>(ws + plan.ws_o_bytes);
+    }
+    if (plan.ws_order_bytes)
+      p.order = reinterpret_cast<int32_t*>(ws + plan.ws_o_bytes + plan.ws_lse_bytes);
   }
   p.dev_status = dev_status;
   const cudaError_t e = launch_softmax(p, plan, d->act_dtype == FLARE_DT_BF16,

@@ -45,6 +45,7 @@ struct SoftmaxParams {
   float* ws_o;                // split partial outputs [R*Hkv][n_split][B*G][D]
   float* ws_lse;              // split partial lse     [R*Hkv][n_split][B*G]
   int n_split, split_len;
+  int32_t* order;             // [R*n_split] work units (r, split), longest first, or nullptr
   int32_t* dev_status;
 };
 
@@ -55,7 +56,7 @@ struct SoftmaxPlan {
   int rows_per_cta;
   int n_split;
   int split_len;
-  size_t ws_o_bytes, ws_lse_bytes;
+  size_t ws_o_bytes, ws_lse_bytes, ws_order_bytes;
   size_t workspace_bytes;
 };
 

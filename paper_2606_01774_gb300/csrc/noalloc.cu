@@ -6,8 +6,9 @@
 // cudaMalloc/cudaFree while requests are in flight (those calls synchronize
 // the device and can fail under memory pressure), or a plugin host that only
 // passes the tensors of the request itself.  This entry point takes the same
-// inputs and outputs as flare_block_softmax_attn but draws the split-prefix
-// partials from one statically sized device array owned by this library.
+// inputs and outputs as flare_block_softmax_attn but draws its workspace (the
+// work order and the split-prefix partials) from one statically sized device
+// array owned by this library.
 //
 // The array lives for as long as the library is loaded and every GPU that
 // loads it holds its FLARE_NOALLOC_SCRATCH_BYTES.  In host code the array's

@@ -11,26 +11,28 @@
 // every prefix token; the mask only touches the ragged prefix end and the
 // block tile (bidirectional, or token-causal for the state-update pass).
 //
-// Tensor memory holds Q (bf16, loaded once), the O accumulator and two S
-// buffers; each S buffer is overwritten in place by its bf16 probabilities P,
-// which the P.V MMA reads straight from tensor memory.  Shared memory only
-// holds a ring of K and V tiles, so per tile the SM moves each K/V byte in
-// once (TMA) and out once (MMA operand read).
+// Tensor memory holds Q (bf16 pairs, loaded once), the O accumulator and the
+// S buffers (three for D <= 128, two for D = 256); each S buffer is
+// overwritten in place by its bf16 probabilities P.  Both products read their
+// A operand from tensor memory (S = Q K^T and O += P V), so shared memory only
+// holds the K and V rings: per tile the SM moves each K/V byte in once (TMA)
+// and out once (MMA operand read), and the rings take all of shared memory,
+// since a tile load takes about a microsecond from issue to arrival.
 //
-// Warp roles (320 threads):
-//   warp 0     TMA producer: K and V tiles (one box per page and 64-column
-//              chunk, 128-byte swizzle) in the order the MMA warp consumes
-//              them (K runs one tile ahead of V).
+// Warp roles (224 threads):
+//   warp 0     K producer, warp 6 V producer: one TMA box per page and
+//              64-column chunk (128-byte swizzle) into their own rings.
 //   warp 1     tensor-memory owner and MMA issuer: S_j = Q K_j^T, then
-//              O += P_{j-1} V_{j-1}; zeroes V rows past the prefix end so
-//              poisoned cache rows never meet a zero probability (0 * NaN).
-//              MMAs from this one thread execute in issue order, which is what
-//              lets S_{j+2} reuse the buffer P_j lives in.
-//   warps 2-9  softmax: two warps per TMEM lane quarter, each thread one query
-//              row and half of the tile's 64 key columns; online base-2
-//              softmax with a lazily moved running max (O is rescaled only when
-//              the max grows by more than 2^8); epilogue divides by the row sum
-//              and stores the output (or a split partial).
+//              O += P_j V_j; zeroes V rows past the prefix end so poisoned
+//              cache rows never meet a zero probability (0 * NaN).  MMAs from
+//              this one thread execute in issue order, which is what lets an
+//              S buffer be reused once the P.V that reads it was issued.
+//   warps 2-5  softmax, one per TMEM lane quarter: load the Q rows into tensor
+//              memory, then per tile each thread takes one query row and the
+//              tile's 64 key columns; online base-2 softmax with a lazily
+//              moved running max (O is rescaled only when the max grows by
+//              more than 2^8); epilogue divides by the row sum and stores the
+//              output (or a split partial).
 // Every wait is bounded (tc::mbar_wait); a timeout sets FLARE_DEV_WAIT_TIMEOUT,
 // the CTA stops issuing work, writes nothing, frees its TMEM and exits.
 #include <cudaTypedefs.h>
@@ -47,11 +49,11 @@ constexpr int kTileN = 64;     // keys per tile
 constexpr int kRowsM = 128;    // query rows per CTA (TMEM lanes)
 constexpr int kSplit = 1;        // softmax warps per TMEM lane quarter (each takes 64/kSplit keys)
 constexpr int kSoftmaxThreads = 128 * kSplit;
-constexpr int kThreadsTC = 64 + kSoftmaxThreads;  // producer warp, MMA warp, softmax warps
+constexpr int kVWarp = 2 + kSoftmaxThreads / 32;   // V producer, after the softmax warps
+constexpr int kThreadsTC = 64 + kSoftmaxThreads + 32;  // K producer, MMA, softmax, V producer
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 
 struct TcMaps {
-  CUtensorMap q;      // (D, Hq, B, R)           box (64, G, 128/G, 1)
   CUtensorMap kblk;   // (D, Hkv, B, R)          box (64, 1, 64, 1)
   CUtensorMap vblk;
   CUtensorMap kpool;  // (D, p, Hkv, num_pages)  box (64, min(p,64), 1, 1)
@@ -62,20 +64,24 @@ template <int D>
 struct TcCfg {
   static constexpr int kChunks = D / 64;
   static constexpr int kKVBytes = kChunks * kTileN * 128;  // one K (or V) tile
-  static constexpr int kQBytes = kChunks * kRowsM * 128;   // Q tile, K-major, 128-byte swizzle
+  // K and V rings fill shared memory: a tile's load takes about a microsecond
+  // from issue to arrival, so the depth of the rings sets the tile rate.
   static constexpr int kKStages = D == 256 ? 3 : (D == 128 ? 6 : 8);  // K ring depth
-  static constexpr int kVStages = D == 256 ? 2 : (D == 128 ? 4 : 8);  // V ring depth
-  static constexpr int kSmem = kQBytes + (kKStages + kVStages) * kKVBytes;
-  // tensor memory: O [0, D), three S/P buffers [D, D + 192)
-  static constexpr int kTmemCols = (D + 3 * kTileN) > 256 ? 512 : 256;
-  static constexpr int kSCol = D;
+  static constexpr int kVStages = D == 256 ? 4 : (D == 128 ? 7 : 8);  // V ring depth
+  static constexpr int kSmem = (kKStages + kVStages) * kKVBytes;
+  // tensor memory: O [0, D), Q as bf16 pairs [D, D + D/2), S/P buffers after
+  static constexpr int kQCol = D;
+  static constexpr int kSCol = D + D / 2;
+  static constexpr int kSBuf = (kSCol + 3 * kTileN) <= 512 ? 3 : 2;  // S/P buffers
+  static constexpr int kTmemCols = (kSCol + kSBuf * kTileN) > 256 ? 512 : 256;
 };
 
 struct TcShared {
-  uint64_t q_full;
+  uint64_t q_ready;
   uint64_t k_full[8], v_full[8], k_empty[8], v_empty[8];
   uint64_t s_full[3], p_full[3], pv_done[3];
   uint64_t o_final;
+  uint64_t v_fix;       // the partial prefix tile's V rows past the prefix end are zeroed
   uint64_t xbar[4];     // row-pair exchange written, one per TMEM lane quarter (64 arrivals)
   uint64_t xread[4];    // row-pair exchange read (64 arrivals)
   float xch[256];       // [half][128 rows]
@@ -129,6 +135,68 @@ __device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, ui
 
 }  // namespace
 
+// Longest-first order of the work units u = (request r, prefix split), by
+// their tile count: a counting sort on one CTA (1024 threads, keys capped at
+// 4095 tiles).  Units with equal counts come in any order; each unit writes
+// its own outputs, so the results do not depend on it.
+constexpr int kOrderThreads = 1024;
+constexpr int kOrderKeys = 4 * kOrderThreads;
+
+__global__ void __launch_bounds__(kOrderThreads) softmax_order_kernel(SoftmaxParams p) {
+  __shared__ int start[kOrderKeys];
+  __shared__ int wsum[kOrderThreads / 32];
+  const int U = p.R * p.n_split;
+  const int tps = p.split_len / kTileN;
+  const int t = threadIdx.x;
+  auto key_of = [&](int u) -> int {
+    const int r = u / p.n_split, split = u % p.n_split;
+    const int P = max(0, p.prefix_len[r]);  // bad lengths are flagged by the attention kernel
+    const int n_pref = (P + kTileN - 1) / kTileN;
+    const int j0 = split * tps;
+    const int here = max(0, min(n_pref, j0 + tps) - j0);
+    return min(here + (split == p.n_split - 1 ? 1 : 0), kOrderKeys - 1);
+  };
+  for (int i = t; i < kOrderKeys; i += kOrderThreads) start[i] = 0;
+  __syncthreads();
+  for (int u = t; u < U; u += kOrderThreads) atomicAdd(&start[key_of(u)], 1);
+  __syncthreads();
+  // start[k] = number of units with a larger key; thread t owns the keys at
+  // descending positions 4t .. 4t+3
+  int v[4], sum = 0;
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    v[e] = start[kOrderKeys - 1 - (4 * t + e)];
+    sum += v[e];
+  }
+  int incl = sum;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int n = __shfl_up_sync(0xffffffffu, incl, o);
+    if ((t & 31) >= o) incl += n;
+  }
+  if ((t & 31) == 31) wsum[t >> 5] = incl;
+  __syncthreads();
+  if (t < 32) {
+    const int w = wsum[t];
+    int wi = w;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int n = __shfl_up_sync(0xffffffffu, wi, o);
+      if (t >= o) wi += n;
+    }
+    wsum[t] = wi - w;
+  }
+  __syncthreads();
+  int run = wsum[t >> 5] + incl - sum;
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    start[kOrderKeys - 1 - (4 * t + e)] = run;
+    run += v[e];
+  }
+  __syncthreads();
+  for (int u = t; u < U; u += kOrderThreads) p.order[atomicAdd(&start[key_of(u)], 1)] = u;
+}
+
 template <int D>
 __global__ void __launch_bounds__(kThreadsTC, 1)
     softmax_tc_kernel(const __grid_constant__ TcMaps maps, SoftmaxParams p) {
@@ -136,13 +204,20 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
   extern __shared__ uint8_t smem_raw[];
   __shared__ TcShared sh;
   uint8_t* base = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  uint8_t* Qs = base;
-  uint8_t* Ks = Qs + C::kQBytes;
+  uint8_t* Ks = base;
   uint8_t* Vs = Ks + C::kKStages * C::kKVBytes;
 
-  const int mtile = blockIdx.x, split = blockIdx.y, item = blockIdx.z;
-  const int r = item / p.Hkv, kvh = item % p.Hkv;
+  // flat grid: (query-row tile, kv head) fastest, then the work units
+  // (request, prefix split) in longest-first order, so that the CTAs that share
+  // a unit's K/V run together and the longest units start first
   const int M = p.B * p.G;
+  const int n_mt = (M + kRowsM - 1) / kRowsM;
+  const int mtile = blockIdx.x % n_mt;
+  const int kvh = (blockIdx.x / n_mt) % p.Hkv;
+  const int z = blockIdx.x / (n_mt * p.Hkv);
+  const int unit = p.order ? p.order[z] : z;
+  const int r = unit / p.n_split, split = unit % p.n_split;
+  const int item = r * p.Hkv + kvh;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
   const int P = p.prefix_len[r];
@@ -158,6 +233,8 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
   const int j1 = min(n_pref, j0 + tps);
   const int n_pref_here = max(0, j1 - j0);
   const bool has_blk = split == p.n_split - 1;
+  // the last prefix tile of this split when it ends inside the tile, else -1
+  const int j_part = (n_pref_here > 0 && j1 == n_pref && (P % kTileN) != 0) ? n_pref_here - 1 : -1;
   const int n_tiles = n_pref_here + (has_blk ? 1 : 0);
   const size_t ws_row0 = ((size_t)item * p.n_split + split) * M;
 
@@ -171,7 +248,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
 
   if (tid == 0) {
     sh.abort_flag = 0;
-    tc::mbar_init(&sh.q_full, 1);
+    tc::mbar_init(&sh.q_ready, kSoftmaxThreads);
     for (int s = 0; s < C::kKStages; ++s) {
       tc::mbar_init(&sh.k_full[s], 1);
       tc::mbar_init(&sh.k_empty[s], 1);
@@ -186,6 +263,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
       tc::mbar_init(&sh.pv_done[b], 1);
     }
     tc::mbar_init(&sh.o_final, 1);
+    tc::mbar_init(&sh.v_fix, 1);
     for (int q = 0; q < 4; ++q) {
       tc::mbar_init(&sh.xbar[q], 32 * kSplit);
       tc::mbar_init(&sh.xread[q], 32 * kSplit);
@@ -198,7 +276,9 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
   tc::fence_after_sync();
   const uint32_t tmem = sh.tmem_base;
   const uint32_t tmem_o = tmem;
+  const uint32_t tmem_q = tmem + C::kQCol;
   const uint32_t tmem_s = tmem + C::kSCol;
+  constexpr int kSB = C::kSBuf;
 
   // tile index -> (is block tile, prefix tile number)
   auto tile_kind = [&](int j, int& ptile) -> bool {
@@ -216,131 +296,134 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     return min(kTileN, P - pt * kTileN);
   };
 
-  if (warp == 0) {
-    // ------------------------------------------------------------ producer
+  if (warp == 0 || warp == kVWarp) {
+    // ------------------------------------------------------------ producers
+    // warp 0 streams the K tiles and warp kVWarp the V tiles, each into its
+    // own ring, so neither waits behind the other's slot.
     if (lane == 0) {
-      tc::prefetch_tmap(&maps.kpool);
-      tc::prefetch_tmap(&maps.vpool);
-      const int Bt = kRowsM / p.G;
-      tc::mbar_expect_tx(&sh.q_full, C::kQBytes);
-      for (int c = 0; c < C::kChunks; ++c)
-        tc::tma_load_4d(Qs + c * (kRowsM * 128), &maps.q, &sh.q_full, c * 64, kvh * p.G,
-                        mtile * Bt, r);
+      const int kv = warp == 0 ? 0 : 1;
+      const CUtensorMap* pool_map = kv ? &maps.vpool : &maps.kpool;
+      const CUtensorMap* blk_map = kv ? &maps.vblk : &maps.kblk;
+      tc::prefetch_tmap(pool_map);
       const int box_rows = p.page_size < kTileN ? p.page_size : kTileN;
-      // one K or V tile into its ring slot (waits for the slot to be free)
-      auto load = [&](int j, int kv) -> bool {
-        const int ns = kv ? C::kVStages : C::kKStages;
+      const int ns = kv ? C::kVStages : C::kKStages;
+      uint8_t* ring = kv ? Vs : Ks;
+      bool ok = true;
+      for (int j = 0; j < n_tiles && ok && !aborted(sh); ++j) {
         const int st = j % ns;
         const uint32_t ph = (uint32_t)(j / ns) & 1u;
         uint64_t* empty = kv ? &sh.v_empty[st] : &sh.k_empty[st];
         uint64_t* full = kv ? &sh.v_full[st] : &sh.k_full[st];
-        uint8_t* dst = (kv ? Vs : Ks) + st * C::kKVBytes;
-        if (!tc::mbar_wait(empty, ph ^ 1u, &sh.abort_flag)) return false;
+        uint8_t* dst = ring + st * C::kKVBytes;
+        if (!tc::mbar_wait(empty, ph ^ 1u, &sh.abort_flag)) {
+          ok = false;
+          break;
+        }
         int pt;
         if (tile_kind(j, pt)) {
           tc::mbar_expect_tx(full, C::kKVBytes);
-          const CUtensorMap* m = kv ? &maps.vblk : &maps.kblk;
           for (int c = 0; c < C::kChunks; ++c)
-            tc::tma_load_4d(dst + c * (kTileN * 128), m, full, c * 64, kvh, 0, r);
+            tc::tma_load_4d(dst + c * (kTileN * 128), blk_map, full, c * 64, kvh, 0, r);
         } else {
           const int tok0 = pt * kTileN;
           const int valid = min(kTileN, P - tok0);
           const int nbox = (valid + box_rows - 1) / box_rows;
           tc::mbar_expect_tx(full, (uint32_t)(C::kChunks * nbox * box_rows * 128));
-          const CUtensorMap* m = kv ? &maps.vpool : &maps.kpool;
-          for (int b = 0; b < nbox; ++b) {
-            const int tok = tok0 + b * box_rows;
+          for (int bx = 0; bx < nbox; ++bx) {
+            const int tok = tok0 + bx * box_rows;
             const int page = p.page_table[(size_t)r * p.max_pages + tok / p.page_size];
             const int row0 = tok % p.page_size;
             for (int c = 0; c < C::kChunks; ++c)
-              tc::tma_load_4d(dst + c * (kTileN * 128) + b * box_rows * 128, m, full, c * 64,
-                              row0, kvh, page);
+              tc::tma_load_4d(dst + c * (kTileN * 128) + bx * box_rows * 128, pool_map, full,
+                              c * 64, row0, kvh, page);
+          }
+          if (kv && j == j_part) {
+            // rows past the prefix end hold stale (possibly poisoned) cache
+            // rows; zero them once the load has landed so that a zero
+            // probability never meets a NaN (0 * NaN) in P.V
+            if (!tc::mbar_wait(full, ph, &sh.abort_flag)) {
+              ok = false;
+              break;
+            }
+            const int nrow = kTileN - valid;
+            for (int c = 0; c < C::kChunks; ++c)
+              for (int e = 0; e < nrow * 8; ++e)
+                *reinterpret_cast<uint4*>(dst + c * (kTileN * 128) + (valid + e / 8) * 128 +
+                                          (e % 8) * 16) = make_uint4(0u, 0u, 0u, 0u);
+            tc::fence_async_smem();
+            tc::mbar_arrive(&sh.v_fix);
           }
         }
-        return true;
-      };
-      // K runs two tiles ahead of V: K0, K1, K2, V0, K3, V1, ... (the MMA warp
-      // consumes K_j at S_j and V_j one step later, at P_j V_j)
-      constexpr int kLead = 2;
-      bool ok = true;
-      for (int j = 0; j < kLead && j < n_tiles && ok; ++j) ok = load(j, 0);
-      for (int j = 0; j < n_tiles && ok && !aborted(sh); ++j) {
-        if (j + kLead < n_tiles) ok = load(j + kLead, 0);
-        if (ok) ok = load(j, 1);
       }
       if (!ok) set_abort(sh, p.dev_status);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
-    const uint32_t id_s = tc::idesc_bf16(kRowsM, kTileN, false, false);
-    const uint32_t id_o = tc::idesc_bf16(kRowsM, D, false, true);
-    bool ok = warp_wait(&sh.q_full, 0, &sh.abort_flag);
-    auto issue_pv = [&](int i) -> bool {
-      const int st = i % C::kVStages;
-      const int pb = i % 3;
-      if (!warp_wait(&sh.p_full[pb], (uint32_t)(i / 3) & 1u, &sh.abort_flag)) return false;
-      if (!warp_wait(&sh.v_full[st], (uint32_t)(i / C::kVStages) & 1u, &sh.abort_flag))
-        return false;
-      uint8_t* vst = Vs + st * C::kKVBytes;
-      const int valid = tile_valid(i);
-      int pt;
-      if (!tile_kind(i, pt) && valid < kTileN) {
-        // zero the V rows past the prefix end (stale or poisoned cache rows)
-        const int nrow = kTileN - valid;
-        for (int e = lane; e < C::kChunks * nrow * 8; e += 32) {
-          const int c = e / (nrow * 8), rr = valid + (e / 8) % nrow, q16 = e % 8;
-          *reinterpret_cast<uint4*>(vst + c * (kTileN * 128) + rr * 128 + q16 * 16) =
-              make_uint4(0u, 0u, 0u, 0u);
-        }
-        tc::fence_async_smem();
-      }
-      __syncwarp();
-      tc::fence_after_sync();
-      if (lane == 0) {
+    // One thread waits and issues; operand descriptors advance by adding the
+    // byte offset (>> 4) to the start-address field of a base descriptor.
+    if (lane == 0) {
+      const uint32_t id_s = tc::idesc_bf16(kRowsM, kTileN, false, false);
+      const uint32_t id_o = tc::idesc_bf16(kRowsM, D, false, true);
+      const uint64_t kdesc0 = tc::sdesc_sw128(tc::smem_u32(Ks), 16, 1024);
+      const uint64_t vdesc0 = tc::sdesc_sw128(tc::smem_u32(Vs), kTileN * 128, 1024);
+      bool ok = tc::mbar_wait(&sh.q_ready, 0, &sh.abort_flag);
+      auto issue_pv = [&](int i) -> bool {
+        const int st = i % C::kVStages;
+        const int pb = i % kSB;
+        if (!tc::mbar_wait(&sh.p_full[pb], (uint32_t)(i / kSB) & 1u, &sh.abort_flag))
+          return false;
+        const bool ready = i == j_part
+                               ? tc::mbar_wait(&sh.v_fix, 0, &sh.abort_flag)
+                               : tc::mbar_wait(&sh.v_full[st], (uint32_t)(i / C::kVStages) & 1u,
+                                               &sh.abort_flag);
+        if (!ready) return false;
+        tc::fence_after_sync();
+        const uint64_t vd = vdesc0 + (uint64_t)((st * C::kKVBytes) >> 4);
 #pragma unroll
-        for (int kk = 0; kk < kTileN / 16; ++kk) {
-          const uint64_t b = tc::sdesc_sw128(tc::smem_u32(vst + kk * 2048), kTileN * 128, 1024);
-          mma_bf16_ts(tmem_o, tmem_s + pb * kTileN + kk * 8, b, id_o, (i > 0 || kk > 0) ? 1u : 0u);
-        }
+        for (int kk = 0; kk < kTileN / 16; ++kk)
+          mma_bf16_ts(tmem_o, tmem_s + pb * kTileN + kk * 8, vd + (uint64_t)(kk * (2048 >> 4)),
+                      id_o, (i > 0 || kk > 0) ? 1u : 0u);
         tc::mma_commit(&sh.pv_done[pb]);
         tc::mma_commit(&sh.v_empty[st]);
-      }
-      __syncwarp();
-      return true;
-    };
-    // S_j = Q K_j^T into S buffer j % 3
-    auto issue_s = [&](int j) -> bool {
-      const int st = j % C::kKStages;
-      const int sb = j % 3;
-      if (!warp_wait(&sh.k_full[st], (uint32_t)(j / C::kKStages) & 1u, &sh.abort_flag))
-        return false;
-      tc::fence_after_sync();
-      if (lane == 0) {
-        const uint8_t* kst = Ks + st * C::kKVBytes;
+        return true;
+      };
+      // S_j = Q K_j^T into S buffer j % kSB (Q from tensor memory)
+      auto issue_s = [&](int j) -> bool {
+        const int st = j % C::kKStages;
+        const int sb = j % kSB;
+        if (!tc::mbar_wait(&sh.k_full[st], (uint32_t)(j / C::kKStages) & 1u, &sh.abort_flag))
+          return false;
+        tc::fence_after_sync();
+        const uint64_t kd = kdesc0 + (uint64_t)((st * C::kKVBytes) >> 4);
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const int c = kk >> 2, off = (kk & 3) * 32;
-          const uint64_t a = tc::sdesc_sw128(tc::smem_u32(Qs + c * (kRowsM * 128) + off), 16, 1024);
-          const uint64_t b = tc::sdesc_sw128(tc::smem_u32(kst + c * (kTileN * 128) + off), 16, 1024);
-          tc::mma_bf16_ss(tmem_s + sb * kTileN, a, b, id_s, kk > 0 ? 1u : 0u);
+          mma_bf16_ts(tmem_s + sb * kTileN, tmem_q + kk * 8,
+                      kd + (uint64_t)((c * (kTileN * 128) + off) >> 4), id_s, kk > 0 ? 1u : 0u);
         }
         tc::mma_commit(&sh.s_full[sb]);
         tc::mma_commit(&sh.k_empty[st]);
+        return true;
+      };
+      // Three S buffers: issue order S0, S1, S2, PV0, S3, PV1, ...: S_{j+2} is
+      // queued before the P.V of tile j waits on its probabilities and reuses
+      // the buffer of tile j-1, whose P.V was issued (and, in issue order,
+      // executes) before it.  Two buffers: S0, S1, PV0, S2, PV1, S3, ...:
+      // S_{j+2} reuses the buffer of tile j, so it follows P_j V_j.
+      for (int j = 0; j < 2 && j < n_tiles && ok; ++j) ok = issue_s(j);
+      for (int j = 0; j < n_tiles && ok; ++j) {
+        if (kSB == 3) {
+          if (j + 2 < n_tiles) ok = issue_s(j + 2);
+          if (ok) ok = issue_pv(j);
+        } else {
+          ok = issue_pv(j);
+          if (ok && j + 2 < n_tiles) ok = issue_s(j + 2);
+        }
       }
-      __syncwarp();
-      return true;
-    };
-    // Issue order S0, S1, S2, PV0, S3, PV1, ...: S_{j+2} is queued before the
-    // P.V of tile j waits on its probabilities, so the tensor pipe stays fed
-    // through the softmax; S_{j+2} reuses the buffer of tile j-1, whose P.V was
-    // issued (and, in issue order, executes) before it.
-    for (int j = 0; j < 2 && j < n_tiles && ok; ++j) ok = issue_s(j);
-    for (int j = 0; j < n_tiles && ok; ++j) {
-      if (j + 2 < n_tiles) ok = issue_s(j + 2);
-      if (ok) ok = issue_pv(j);
+      if (ok) tc::mma_commit(&sh.o_final);
+      if (!ok) set_abort(sh, p.dev_status);
     }
-    if (ok && lane == 0) tc::mma_commit(&sh.o_final);
-    if (!ok && lane == 0) set_abort(sh, p.dev_status);
+    __syncwarp();
   } else {
     // ------------------------------------------------------------ softmax warps
     // Eight warps: warp w reads TMEM lanes 32*(w%4).. (its 32 rows) and key
@@ -355,11 +438,42 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     constexpr int kDh = D / kSplit;       // Q elements / output columns this warp handles
     constexpr int kCols = kTileN / kSplit;  // key columns of each tile this warp handles
 
+    // Q row (this warp's D/kSplit elements) into tensor memory as bf16 pairs,
+    // the A operand of S = Q K^T; rows past the block's B*G are zero
+    {
+      const int g = m % p.G;
+      const bool live = m < M;
+      const uint4* qrow = reinterpret_cast<const uint4*>(
+          static_cast<const __nv_bfloat16*>(p.q) +
+          (((size_t)r * p.B + (live ? trow : 0)) * p.Hq + kvh * p.G + g) * D + half * kDh);
+      constexpr int kWords = kDh / 2;                        // TMEM columns of this warp
+      constexpr int kBatch = kWords < 64 ? kWords : 64;      // columns per batch of loads
+#pragma unroll 1
+      for (int c0 = 0; c0 < kWords; c0 += kBatch) {
+        uint32_t w[kBatch];
+#pragma unroll
+        for (int q4 = 0; q4 < kBatch / 4; ++q4) {
+          const uint4 v = live ? qrow[(c0 / 4) + q4] : make_uint4(0u, 0u, 0u, 0u);
+          w[4 * q4] = v.x;
+          w[4 * q4 + 1] = v.y;
+          w[4 * q4 + 2] = v.z;
+          w[4 * q4 + 3] = v.w;
+        }
+#pragma unroll
+        for (int c = 0; c < kBatch; c += 16)
+          tmem_st16(tmem_q + lane_off + half * kWords + c0 + c,
+                    *reinterpret_cast<uint32_t(*)[16]>(&w[c]));
+      }
+      tmem_st_wait();
+      tc::fence_before_sync();
+      tc::mbar_arrive(&sh.q_ready);
+    }
+
     float m_run = -INFINITY, l_run = 0.f;  // l_run: this half's share of the row sum
     bool ok = true;
     for (int j = 0; j < n_tiles; ++j) {
-      const int sb = j % 3;
-      if (!warp_wait(&sh.s_full[sb], (uint32_t)(j / 3) & 1u, &sh.abort_flag)) {
+      const int sb = j % kSB;
+      if (!warp_wait(&sh.s_full[sb], (uint32_t)(j / kSB) & 1u, &sh.abort_flag)) {
         ok = false;
         break;
       }
@@ -437,8 +551,8 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
       l_run = (j == 0) ? sum : l_run * corr + sum;
       // rescale this half's O columns when the running max moved (P.V of tile j-1 done)
       if (warp_rescale && j >= 1) {
-        const int pb = (j - 1) % 3;
-        if (!warp_wait(&sh.pv_done[pb], (uint32_t)((j - 1) / 3) & 1u, &sh.abort_flag)) {
+        const int pb = (j - 1) % kSB;
+        if (!warp_wait(&sh.pv_done[pb], (uint32_t)((j - 1) / kSB) & 1u, &sh.abort_flag)) {
           ok = false;
           break;
         }
@@ -561,12 +675,6 @@ cudaError_t launch_tc_d(const SoftmaxParams& p, const SoftmaxPlan& plan, cudaStr
   TcMaps maps;
   const uint64_t e = 2;
   {
-    const uint64_t dims[4] = {(uint64_t)D, (uint64_t)p.Hq, (uint64_t)p.B, (uint64_t)p.R};
-    const uint64_t str[3] = {D * e, (uint64_t)p.Hq * D * e, (uint64_t)p.B * p.Hq * D * e};
-    const uint32_t box[4] = {64, (uint32_t)p.G, (uint32_t)(kRowsM / p.G), 1};
-    if (!encode4(&maps.q, p.q, dims, str, box)) return cudaErrorInvalidValue;
-  }
-  {
     const uint64_t dims[4] = {(uint64_t)D, (uint64_t)p.Hkv, (uint64_t)p.B, (uint64_t)p.R};
     const uint64_t str[3] = {D * e, (uint64_t)p.Hkv * D * e, (uint64_t)p.B * p.Hkv * D * e};
     const uint32_t box[4] = {64, 1, (uint32_t)kTileN, 1};
@@ -592,8 +700,15 @@ cudaError_t launch_tc_d(const SoftmaxParams& p, const SoftmaxPlan& plan, cudaStr
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (err != cudaSuccess) return err;
   const int M = p.B * p.G;
-  dim3 grid((M + kRowsM - 1) / kRowsM, plan.n_split, p.R * p.Hkv);
-  softmax_tc_kernel<D><<<grid, kThreadsTC, smem, stream>>>(maps, p);
+  if (p.order) {
+    softmax_order_kernel<<<1, kOrderThreads, 0, stream>>>(p);
+    note_launches(1);
+    err = cudaGetLastError();
+    if (err != cudaSuccess) return err;
+  }
+  const long long n_cta = (long long)((M + kRowsM - 1) / kRowsM) * p.Hkv * p.R * plan.n_split;
+  if (n_cta > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+  softmax_tc_kernel<D><<<(unsigned)n_cta, kThreadsTC, smem, stream>>>(maps, p);
   note_launches(1);
   err = cudaGetLastError();
   if (err != cudaSuccess || plan.n_split == 1) return err;
