@@ -229,7 +229,7 @@ flare_status flare_append_kv(const flare_softmax_desc* desc, const void* k_blk, 
  * requests are in flight (they synchronize the device and can fail under
  * memory pressure), or a plugin host that passes only the request's own
  * tensors.  Same arguments, layouts, outputs and status bits as
- * flare_block_softmax_attn, minus the workspace: the split partials live in a
+ * flare_block_softmax_attn, minus the workspace: the workspace (work order and split partials) lives in a
  * file-scope device array of FLARE_NOALLOC_SCRATCH_BYTES that the library
  * holds on every GPU that loads it, until the process exits.
  *  - This call allocates nothing (no cudaMalloc, cudaFree or allocating
