@@ -92,17 +92,19 @@ SoftmaxPlan plan_softmax(int R, int B, int Hq, int Hkv, int D, int page_size, in
   const int G = Hq / Hkv, M = B * G;
   const long prefix_max = (long)max_pages * page_size;
   if (bf16 && softmax_tc_supported(B, Hq, Hkv, D, page_size)) {
-    // tensor-core kernel: 128 query rows per CTA, one CTA per SM; split the
-    // prefix only when the batch gives fewer than two CTAs per SM, and keep
-    // at least 16 tiles (1024 keys) per split so partials stay small.
+    // tensor-core kernel: 128 query rows per CTA, one CTA per SM, work units
+    // started longest first.  Split the prefix only when the batch has fewer
+    // work items than SMs (then aim at two CTAs per SM), and keep at least 16
+    // tiles (1024 keys) per split so partials stay small.
     pl.kernel = 1;
     pl.rows_per_cta = 128;
     const long items = (long)R * Hkv * ((M + 127) / 128);
     const long tiles = (prefix_max + 63) / 64;
     long ns = 1;
-    if (items > 0 && items < 2L * num_sms) ns = (2L * num_sms + items - 1) / items;
+    if (items > 0 && items < num_sms) ns = (2L * num_sms + items - 1) / items;
     const long cap = tiles / 16 > 1 ? tiles / 16 : 1;
     if (ns > cap) ns = cap;
+    if (ns > 64) ns = 64;  // the merge keeps 128 x n_split weights in shared memory
     const long tps = ns > 0 ? (tiles + ns - 1) / ns : 1;
     pl.split_len = (int)((tps > 0 ? tps : 1) * 64);
     pl.n_split = tiles > 0 ? (int)((tiles + tps - 1) / tps) : 1;
@@ -128,9 +130,15 @@ SoftmaxPlan plan_softmax(int R, int B, int Hq, int Hkv, int D, int page_size, in
     pl.ws_o_bytes = (rows * D * sizeof(float) + 255) / 256 * 256;
     pl.ws_lse_bytes = (rows * sizeof(float) + 255) / 256 * 256;
   }
-  // tensor-core kernel: the work units in longest-first order
-  if (pl.kernel == 1) pl.ws_order_bytes = ((size_t)R * pl.n_split * sizeof(int32_t) + 255) / 256 * 256;
-  pl.workspace_bytes = pl.ws_o_bytes + pl.ws_lse_bytes + pl.ws_order_bytes;
+  // tensor-core kernel: the work units in longest-first order, and per row
+  // tile a count of finished splits (the last one merges the partials)
+  if (pl.kernel == 1) {
+    pl.ws_order_bytes = ((size_t)R * pl.n_split * sizeof(int32_t) + 255) / 256 * 256;
+    if (pl.n_split > 1)
+      pl.ws_count_bytes =
+          ((size_t)R * Hkv * ((M + 127) / 128) * sizeof(int32_t) + 255) / 256 * 256;
+  }
+  pl.workspace_bytes = pl.ws_o_bytes + pl.ws_lse_bytes + pl.ws_order_bytes + pl.ws_count_bytes;
   return pl;
 }
 
@@ -283,6 +291,9 @@ flare_status flare_block_softmax_attn(const flare_softmax_desc* d, const void* q
     }
     if (plan.ws_order_bytes)
       p.order = reinterpret_cast<int32_t*>(ws + plan.ws_o_bytes + plan.ws_lse_bytes);
+    if (plan.ws_count_bytes)
+      p.counters = reinterpret_cast<int32_t*>(ws + plan.ws_o_bytes + plan.ws_lse_bytes +
+                                              plan.ws_order_bytes);
   }
   p.dev_status = dev_status;
   const cudaError_t e = launch_softmax(p, plan, d->act_dtype == FLARE_DT_BF16,

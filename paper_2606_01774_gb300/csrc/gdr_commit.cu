@@ -5,11 +5,13 @@
 // from the left, so column c of S evolves on its own (Eq. per-step-fwd):
 //     u_t[c] = v_t[c] - alpha_t (S^T k_t)[c],   delta_t[c] = beta_t u_t[c],
 //     S[:, c] <- alpha_t S[:, c] + k_t delta_t[c].
-// Two threads share column c, each holding half of its d_k rows in registers
-// (lanes l and l+16 of a warp, so the two halves of k_t . S[:, c] meet with one
-// shuffle).  The block's keys (and queries, for the token-causal outputs) and
-// values are staged once in shared memory as fp32 with 16-byte loads issued
-// together with the state loads.
+// Each thread holds a block of 4 columns x d_k/8 rows of S in registers: lane
+// = 4 * row_group + column_group, so the 8 row groups of a column sit in one
+// warp and meet with three shuffles, each loaded key value serves 4 columns,
+// and the state moves in 16-byte pieces (a warp covers 16 columns, 8 warps a
+// 128-column state).  The block's keys (and queries, for the token-causal
+// outputs) and values are staged once in shared memory as fp32 with 16-byte
+// loads issued together with the state loads.
 //
 // The decay is applied lazily: the thread keeps S~ = S / Gam_t with
 // Gam_t = alpha_1 ... alpha_t (since the last fold), so a step is
@@ -17,9 +19,9 @@
 // one multiply-add per element for the product and one for the update.  When
 // Gam_t would fall below 2^-40 the decay is folded into the state instead
 // (S <- Gam_t S~ + k_t delta_t, Gam <- 1), so 1/Gam_t stays bounded.  After the
-// first n = accept_len tokens Gam_n S~ is written back in place (coalesced);
-// n = 0 leaves the slot untouched.  Exact fp32 arithmetic throughout, which is
-// what the committed state's accuracy needs.
+// first n = accept_len tokens Gam_n S~ is written back in place; n = 0 leaves
+// the slot untouched.  Exact fp32 arithmetic throughout, which is what the
+// committed state's accuracy needs.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -70,8 +72,8 @@ __device__ __forceinline__ void stage_rows(float* dst, const T* src, size_t stri
 
 template <typename T, int DK, int DV, bool CAUSAL>
 __global__ void __launch_bounds__(2 * DV, 2) gdr_commit_kernel(GdrParams p) {
-  constexpr int kThreads = 2 * DV;
-  constexpr int kHalf = DK / 2;  // state rows per thread
+  constexpr int kThreads = 2 * DV;   // DV / 16 warps
+  constexpr int kR = DK / 8;         // state rows per thread
   extern __shared__ float smc[];
   __shared__ float alpha_s[kCBmax], beta_s[kCBmax];
 
@@ -79,8 +81,8 @@ __global__ void __launch_bounds__(2 * DV, 2) gdr_commit_kernel(GdrParams p) {
   const int r = item / p.Hv, j = item % p.Hv;
   const int h = j / (p.Hv / p.Hk);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int half = lane >> 4;               // which half of the rows
-  const int c = warp * 16 + (lane & 15);    // value column
+  const int rg = lane >> 2;                      // row group: rows rg*kR ..
+  const int c0 = warp * 16 + (lane & 3) * 4;     // columns c0 .. c0+3
   const int B = p.B;
 
   const int slot = p.state_slot[r];
@@ -100,11 +102,10 @@ __global__ void __launch_bounds__(2 * DV, 2) gdr_commit_kernel(GdrParams p) {
   float* Qs = Ks + steps * DK;                       // [steps][DK] (CAUSAL only)
   float* Vs = Qs + (CAUSAL ? steps * DK : 0);        // [steps][DV]
 
-  // state rows half*kHalf .. half*kHalf + kHalf - 1 of column c
-  float* Sg = p.state_pool + ((size_t)slot * p.Hv + j) * DK * DV + (size_t)half * kHalf * DV + c;
-  float s[kHalf];
+  float* Sg = p.state_pool + ((size_t)slot * p.Hv + j) * DK * DV + (size_t)rg * kR * DV + c0;
+  float4 s[kR];  // S~[rg*kR + m][c0 .. c0+3]
 #pragma unroll
-  for (int m = 0; m < kHalf; ++m) s[m] = Sg[(size_t)m * DV];
+  for (int m = 0; m < kR; ++m) s[m] = *reinterpret_cast<const float4*>(Sg + (size_t)m * DV);
 
   const T* kg = static_cast<const T*>(p.k) + ((size_t)r * B * p.Hk + h) * DK;
   const T* vg = static_cast<const T*>(p.v) + ((size_t)r * B * p.Hv + j) * DV;
@@ -121,66 +122,103 @@ __global__ void __launch_bounds__(2 * DV, 2) gdr_commit_kernel(GdrParams p) {
   }
   __syncthreads();
 
-  float gam = 1.f;  // S = gam * s
+  float gam = 1.f;  // S = gam * S~
 #pragma unroll 1
   for (int t = 0; t < steps; ++t) {
-    const float4* k4 = reinterpret_cast<const float4*>(Ks + t * DK + half * kHalf);
-    float d0 = 0.f, d1 = 0.f, d2 = 0.f, d3 = 0.f;
+    float k[kR];
+    {
+      const float4* k4 = reinterpret_cast<const float4*>(Ks + t * DK + rg * kR);
 #pragma unroll
-    for (int m4 = 0; m4 < kHalf / 4; ++m4) {
-      const float4 kk = k4[m4];
-      d0 = fmaf(s[4 * m4], kk.x, d0);
-      d1 = fmaf(s[4 * m4 + 1], kk.y, d1);
-      d2 = fmaf(s[4 * m4 + 2], kk.z, d2);
-      d3 = fmaf(s[4 * m4 + 3], kk.w, d3);
-    }
-    float dot = (d0 + d1) + (d2 + d3);
-    dot += __shfl_xor_sync(0xffffffffu, dot, 16);
-    const float gt = gam * alpha_s[t];
-    const float delta = beta_s[t] * (Vs[t * DV + c] - gt * dot);
-    __syncwarp();  // re-read k from shared memory below instead of holding it in registers
-    if (gt >= kMinGam) {  // uniform across the CTA: the gates are per head
-      const float w = delta / gt;
-#pragma unroll
-      for (int m4 = 0; m4 < kHalf / 4; ++m4) {
+      for (int m4 = 0; m4 < kR / 4; ++m4) {
         const float4 kk = k4[m4];
-        s[4 * m4] = fmaf(kk.x, w, s[4 * m4]);
-        s[4 * m4 + 1] = fmaf(kk.y, w, s[4 * m4 + 1]);
-        s[4 * m4 + 2] = fmaf(kk.z, w, s[4 * m4 + 2]);
-        s[4 * m4 + 3] = fmaf(kk.w, w, s[4 * m4 + 3]);
+        k[4 * m4] = kk.x;
+        k[4 * m4 + 1] = kk.y;
+        k[4 * m4 + 2] = kk.z;
+        k[4 * m4 + 3] = kk.w;
+      }
+    }
+    // (S~^T k)[c] over this row group, then over the 8 row groups of the warp
+    float4 d = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int m = 0; m < kR; ++m) {
+      d.x = fmaf(s[m].x, k[m], d.x);
+      d.y = fmaf(s[m].y, k[m], d.y);
+      d.z = fmaf(s[m].z, k[m], d.z);
+      d.w = fmaf(s[m].w, k[m], d.w);
+    }
+#pragma unroll
+    for (int o = 4; o < 32; o <<= 1) {
+      d.x += __shfl_xor_sync(0xffffffffu, d.x, o);
+      d.y += __shfl_xor_sync(0xffffffffu, d.y, o);
+      d.z += __shfl_xor_sync(0xffffffffu, d.z, o);
+      d.w += __shfl_xor_sync(0xffffffffu, d.w, o);
+    }
+    const float gt = gam * alpha_s[t];
+    const float bt = beta_s[t];
+    const float4 v = *reinterpret_cast<const float4*>(Vs + t * DV + c0);
+    float4 delta;
+    delta.x = bt * (v.x - gt * d.x);
+    delta.y = bt * (v.y - gt * d.y);
+    delta.z = bt * (v.z - gt * d.z);
+    delta.w = bt * (v.w - gt * d.w);
+    if (gt >= kMinGam) {  // uniform across the CTA: the gates are per head
+      const float ig = 1.f / gt;
+      const float4 w = make_float4(delta.x * ig, delta.y * ig, delta.z * ig, delta.w * ig);
+#pragma unroll
+      for (int m = 0; m < kR; ++m) {
+        s[m].x = fmaf(k[m], w.x, s[m].x);
+        s[m].y = fmaf(k[m], w.y, s[m].y);
+        s[m].z = fmaf(k[m], w.z, s[m].z);
+        s[m].w = fmaf(k[m], w.w, s[m].w);
       }
       gam = gt;
     } else {  // fold the decay into the state
 #pragma unroll
-      for (int m4 = 0; m4 < kHalf / 4; ++m4) {
-        const float4 kk = k4[m4];
-        s[4 * m4] = fmaf(kk.x, delta, gt * s[4 * m4]);
-        s[4 * m4 + 1] = fmaf(kk.y, delta, gt * s[4 * m4 + 1]);
-        s[4 * m4 + 2] = fmaf(kk.z, delta, gt * s[4 * m4 + 2]);
-        s[4 * m4 + 3] = fmaf(kk.w, delta, gt * s[4 * m4 + 3]);
+      for (int m = 0; m < kR; ++m) {
+        s[m].x = fmaf(k[m], delta.x, gt * s[m].x);
+        s[m].y = fmaf(k[m], delta.y, gt * s[m].y);
+        s[m].z = fmaf(k[m], delta.z, gt * s[m].z);
+        s[m].w = fmaf(k[m], delta.w, gt * s[m].w);
       }
       gam = 1.f;
     }
     if (t + 1 == n) {
 #pragma unroll
-      for (int m = 0; m < kHalf; ++m) Sg[(size_t)m * DV] = gam * s[m];
+      for (int m = 0; m < kR; ++m)
+        *reinterpret_cast<float4*>(Sg + (size_t)m * DV) =
+            make_float4(gam * s[m].x, gam * s[m].y, gam * s[m].z, gam * s[m].w);
     }
     if (CAUSAL) {
-      const float4* q4 = reinterpret_cast<const float4*>(Qs + t * DK + half * kHalf);
-      float o0 = 0.f, o1 = 0.f, o2 = 0.f, o3 = 0.f;
+      const float4* q4 = reinterpret_cast<const float4*>(Qs + t * DK + rg * kR);
+      float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-      for (int m4 = 0; m4 < kHalf / 4; ++m4) {
+      for (int m4 = 0; m4 < kR / 4; ++m4) {
         const float4 qq = q4[m4];
-        o0 = fmaf(s[4 * m4], qq.x, o0);
-        o1 = fmaf(s[4 * m4 + 1], qq.y, o1);
-        o2 = fmaf(s[4 * m4 + 2], qq.z, o2);
-        o3 = fmaf(s[4 * m4 + 3], qq.w, o3);
+        const float qv[4] = {qq.x, qq.y, qq.z, qq.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int m = 4 * m4 + e;
+          o.x = fmaf(s[m].x, qv[e], o.x);
+          o.y = fmaf(s[m].y, qv[e], o.y);
+          o.z = fmaf(s[m].z, qv[e], o.z);
+          o.w = fmaf(s[m].w, qv[e], o.w);
+        }
       }
-      float o = (o0 + o1) + (o2 + o3);
-      o += __shfl_xor_sync(0xffffffffu, o, 16);
-      if (half == 0)
-        static_cast<T*>(p.out_causal)[(((size_t)r * B + t) * p.Hv + j) * DV + c] =
-            from_f32<T>(p.scale * gam * o);
+#pragma unroll
+      for (int sh = 4; sh < 32; sh <<= 1) {
+        o.x += __shfl_xor_sync(0xffffffffu, o.x, sh);
+        o.y += __shfl_xor_sync(0xffffffffu, o.y, sh);
+        o.z += __shfl_xor_sync(0xffffffffu, o.z, sh);
+        o.w += __shfl_xor_sync(0xffffffffu, o.w, sh);
+      }
+      if (rg == 0) {
+        T* out = static_cast<T*>(p.out_causal) + (((size_t)r * B + t) * p.Hv + j) * DV + c0;
+        const float sc = p.scale * gam;
+        out[0] = from_f32<T>(sc * o.x);
+        out[1] = from_f32<T>(sc * o.y);
+        out[2] = from_f32<T>(sc * o.z);
+        out[3] = from_f32<T>(sc * o.w);
+      }
     }
   }
 }

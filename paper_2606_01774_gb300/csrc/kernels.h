@@ -46,6 +46,7 @@ struct SoftmaxParams {
   float* ws_lse;              // split partial lse     [R*Hkv][n_split][B*G]
   int n_split, split_len;
   int32_t* order;             // [R*n_split] work units (r, split), longest first, or nullptr
+  int32_t* counters;          // [R*Hkv*ceil(B*G/128)] finished splits per row tile (n_split > 1)
   int32_t* dev_status;
 };
 
@@ -56,7 +57,7 @@ struct SoftmaxPlan {
   int rows_per_cta;
   int n_split;
   int split_len;
-  size_t ws_o_bytes, ws_lse_bytes, ws_order_bytes;
+  size_t ws_o_bytes, ws_lse_bytes, ws_order_bytes, ws_count_bytes;
   size_t workspace_bytes;
 };
 

@@ -87,6 +87,7 @@ struct TcShared {
   float xch[256];       // [half][128 rows]
   uint32_t tmem_base;
   int abort_flag;
+  int last_split;       // this CTA merges the split partials of its row tile
 };
 
 // All lanes of the warp wait; the outcome is made warp-uniform so that the
@@ -135,6 +136,93 @@ __device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, ui
 
 }  // namespace
 
+// Merge of the split partials of one row tile (rows mtile*128 ..) of one
+// (request, kv head): out = sum_s w_s o_s with w_s = exp(lse_s - lse) and
+// lse = log sum_s exp(lse_s) (the splits' partial outputs are already
+// normalised by their own row sums).  The weights go to shared memory first
+// (one thread per row); then every thread combines 8 (row, 4-column) pieces at
+// a time with all their loads in flight.  All threads of the CTA call this;
+// `wts` holds 128 * n_split floats.
+template <int D>
+__device__ void merge_splits(const SoftmaxParams& p, int item, int r, int kvh, int mtile,
+                             float* wts) {
+  const int M = p.B * p.G;
+  const int ns = p.n_split;
+  const int m0 = mtile * kRowsM;
+  const int rows = min(kRowsM, M - m0);
+  const size_t base = (size_t)item * ns * M + m0;  // row i of split s at base + s * M + i
+  for (int i = threadIdx.x; i < rows; i += blockDim.x) {
+    float mx = -INFINITY;
+    for (int s = 0; s < ns; ++s) mx = fmaxf(mx, p.ws_lse[base + (size_t)s * M + i]);
+    float den = 0.f;
+    for (int s = 0; s < ns; ++s) {
+      const float l = p.ws_lse[base + (size_t)s * M + i];
+      const float e = l == -INFINITY ? 0.f : expf(l - mx);
+      wts[i * ns + s] = e;
+      den += e;
+    }
+    const float inv = 1.f / den;
+    for (int s = 0; s < ns; ++s) wts[i * ns + s] *= inv;
+    const int m = m0 + i, t = m / p.G, g = m % p.G;
+    if (p.lse) p.lse[((size_t)r * p.B + t) * p.Hq + kvh * p.G + g] = mx + logf(den);
+  }
+  __syncthreads();
+  constexpr int kC = D / 4;  // 4-column pieces per row
+  constexpr int kBatch = 8;
+  const int n_items = rows * kC;
+  for (int i0 = threadIdx.x; i0 < n_items; i0 += kBatch * blockDim.x) {
+    float4 acc[kBatch];
+#pragma unroll
+    for (int k = 0; k < kBatch; ++k) acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int s = 0; s < ns; ++s) {
+      float4 o[kBatch];
+#pragma unroll
+      for (int k = 0; k < kBatch; ++k) {
+        const int it = i0 + k * blockDim.x;
+        o[k] = it < n_items ? *reinterpret_cast<const float4*>(
+                                  p.ws_o + (base + (size_t)s * M + it / kC) * D + (it % kC) * 4)
+                            : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+#pragma unroll
+      for (int k = 0; k < kBatch; ++k) {
+        const int it = i0 + k * blockDim.x;
+        const float w = it < n_items ? wts[(it / kC) * ns + s] : 0.f;
+        acc[k].x = fmaf(w, o[k].x, acc[k].x);
+        acc[k].y = fmaf(w, o[k].y, acc[k].y);
+        acc[k].z = fmaf(w, o[k].z, acc[k].z);
+        acc[k].w = fmaf(w, o[k].w, acc[k].w);
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < kBatch; ++k) {
+      const int it = i0 + k * blockDim.x;
+      if (it >= n_items) continue;
+      const int m = m0 + it / kC, t = m / p.G, g = m % p.G;
+      const size_t orow = ((size_t)r * p.B + t) * p.Hq + kvh * p.G + g;
+      __nv_bfloat162 lo = __floats2bfloat162_rn(acc[k].x, acc[k].y);
+      __nv_bfloat162 hi = __floats2bfloat162_rn(acc[k].z, acc[k].w);
+      *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(p.out) + orow * D + (it % kC) * 4) =
+          make_uint2(*reinterpret_cast<uint32_t*>(&lo), *reinterpret_cast<uint32_t*>(&hi));
+    }
+  }
+}
+
+// Publishes this CTA's split partial and, if it is the last split of its row
+// tile to finish, merges them all (all threads of the CTA call this).
+template <int D>
+__device__ void finish_split(const SoftmaxParams& p, int item, int r, int kvh, int mtile,
+                             int n_mt, int* last_flag, float* wts) {
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0)
+    *last_flag = atomicAdd(&p.counters[(size_t)item * n_mt + mtile], 1) == p.n_split - 1;
+  __syncthreads();
+  if (*last_flag) {
+    __threadfence();
+    merge_splits<D>(p, item, r, kvh, mtile, wts);
+  }
+}
+
 // Longest-first order of the work units u = (request r, prefix split), by
 // their tile count: a counting sort on one CTA (1024 threads, keys capped at
 // 4095 tiles).  Units with equal counts come in any order; each unit writes
@@ -157,6 +245,10 @@ __global__ void __launch_bounds__(kOrderThreads) softmax_order_kernel(SoftmaxPar
     return min(here + (split == p.n_split - 1 ? 1 : 0), kOrderKeys - 1);
   };
   for (int i = t; i < kOrderKeys; i += kOrderThreads) start[i] = 0;
+  if (p.counters) {
+    const int n_cnt = p.R * p.Hkv * ((p.B * p.G + kRowsM - 1) / kRowsM);
+    for (int i = t; i < n_cnt; i += kOrderThreads) p.counters[i] = 0;
+  }
   __syncthreads();
   for (int u = t; u < U; u += kOrderThreads) atomicAdd(&start[key_of(u)], 1);
   __syncthreads();
@@ -238,11 +330,12 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
   const int n_tiles = n_pref_here + (has_blk ? 1 : 0);
   const size_t ws_row0 = ((size_t)item * p.n_split + split) * M;
 
-  if (n_tiles == 0) {  // empty split: mark its partial as empty for the combine pass
+  if (n_tiles == 0) {  // empty split: mark its partial as empty for the merge
     for (int i = tid; i < kRowsM; i += blockDim.x) {
       const int m = mtile * kRowsM + i;
       if (m < M) p.ws_lse[ws_row0 + m] = -INFINITY;
     }
+    finish_split<D>(p, item, r, kvh, mtile, n_mt, &sh.last_split, reinterpret_cast<float*>(Ks));
     return;
   }
 
@@ -636,6 +729,9 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     tc::fence_after_sync();
     tc::tmem_dealloc(tmem, C::kTmemCols);
   }
+  // a CTA that gave up wrote no partial: its row tile is never merged
+  if (p.n_split > 1 && !aborted(sh))  // the K/V rings are free: merge weights go there
+    finish_split<D>(p, item, r, kvh, mtile, n_mt, &sh.last_split, reinterpret_cast<float*>(Ks));
 }
 
 // ------------------------------------------------------------------ host side
@@ -710,9 +806,7 @@ cudaError_t launch_tc_d(const SoftmaxParams& p, const SoftmaxPlan& plan, cudaStr
   if (n_cta > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
   softmax_tc_kernel<D><<<(unsigned)n_cta, kThreadsTC, smem, stream>>>(maps, p);
   note_launches(1);
-  err = cudaGetLastError();
-  if (err != cudaSuccess || plan.n_split == 1) return err;
-  return launch_softmax_combine(p, true, stream);
+  return cudaGetLastError();
 }
 
 }  // namespace
