@@ -133,7 +133,13 @@ SoftmaxPlan plan_softmax(int R, int B, int Hq, int Hkv, int D, int page_size, in
   // tensor-core kernel: the work units in longest-first order, and per row
   // tile a count of finished splits (the last one merges the partials)
   if (pl.kernel == 1) {
-    pl.ws_order_bytes = ((size_t)R * pl.n_split * sizeof(int32_t) + 255) / 256 * 256;
+    // order [R*n_split], n_valid [1], bad-request mask [ceil(R/32)]
+    pl.ws_order_bytes =
+        (((size_t)R * pl.n_split + 1 + (size_t)(R + 31) / 32) * sizeof(int32_t) + 255) / 256 * 256;
+    // one CTA per work item when the prefix is split, else one per SM (at most
+    // one per work item) walking the items
+    const long n_items = (long)((M + 127) / 128) * Hkv * R * pl.n_split;
+    pl.num_ctas = (int)(pl.n_split > 1 ? n_items : (n_items < num_sms ? n_items : num_sms));
     if (pl.n_split > 1)
       pl.ws_count_bytes =
           ((size_t)R * Hkv * ((M + 127) / 128) * sizeof(int32_t) + 255) / 256 * 256;
@@ -289,8 +295,11 @@ flare_status flare_block_softmax_attn(const flare_softmax_desc* d, const void* q
       p.ws_o = reinterpret_cast<float*>(ws);
       p.ws_lse = reinterpret_cast<float*>(ws + plan.ws_o_bytes);
     }
-    if (plan.ws_order_bytes)
+    if (plan.ws_order_bytes) {
       p.order = reinterpret_cast<int32_t*>(ws + plan.ws_o_bytes + plan.ws_lse_bytes);
+      p.n_valid = p.order + (size_t)p.R * plan.n_split;
+      p.bad_mask = reinterpret_cast<uint32_t*>(p.n_valid + 1);
+    }
     if (plan.ws_count_bytes)
       p.counters = reinterpret_cast<int32_t*>(ws + plan.ws_o_bytes + plan.ws_lse_bytes +
                                               plan.ws_order_bytes);

@@ -45,7 +45,9 @@ struct SoftmaxParams {
   float* ws_o;                // split partial outputs [R*Hkv][n_split][B*G][D]
   float* ws_lse;              // split partial lse     [R*Hkv][n_split][B*G]
   int n_split, split_len;
-  int32_t* order;             // [R*n_split] work units (r, split), longest first, or nullptr
+  int32_t* order;             // [R*n_split] valid work units (r, split), longest first
+  int32_t* n_valid;           // number of valid work units in `order`
+  uint32_t* bad_mask;         // [ceil(R/32)] requests with a bad prefix length or page id
   int32_t* counters;          // [R*Hkv*ceil(B*G/128)] finished splits per row tile (n_split > 1)
   int32_t* dev_status;
 };
@@ -57,6 +59,7 @@ struct SoftmaxPlan {
   int rows_per_cta;
   int n_split;
   int split_len;
+  int num_ctas;  // tensor-core kernel: CTAs launched
   size_t ws_o_bytes, ws_lse_bytes, ws_order_bytes, ws_count_bytes;
   size_t workspace_bytes;
 };

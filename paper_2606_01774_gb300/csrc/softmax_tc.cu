@@ -11,7 +11,14 @@
 // every prefix token; the mask only touches the ragged prefix end and the
 // block tile (bidirectional, or token-causal for the state-update pass).
 //
-// Tensor memory holds Q (bf16 pairs, loaded once), the O accumulator and the
+// A one-CTA pre-pass validates every request (prefix length, page ids), drops
+// bad ones from the work list and orders the work units longest first.  When
+// prefixes are not split, one CTA per SM walks its share of the items (snake
+// order over the CTAs), so setup happens once per CTA and the next item's
+// loads and S products overlap the current item's epilogue; when they are,
+// one CTA runs each item and the last split of a row tile merges the partials.
+//
+// Tensor memory holds Q (bf16 pairs, loaded per item), the O accumulator and the
 // S buffers (three for D <= 128, two for D = 256); each S buffer is
 // overwritten in place by its bf16 probabilities P.  Both products read their
 // A operand from tensor memory (S = Q K^T and O += P V), so shared memory only
@@ -46,11 +53,10 @@ namespace flare {
 namespace {
 
 constexpr int kTileN = 64;     // keys per tile
-constexpr int kRowsM = 128;    // query rows per CTA (TMEM lanes)
-constexpr int kSplit = 1;        // softmax warps per TMEM lane quarter (each takes 64/kSplit keys)
-constexpr int kSoftmaxThreads = 128 * kSplit;
-constexpr int kVWarp = 2 + kSoftmaxThreads / 32;   // V producer, after the softmax warps
-constexpr int kThreadsTC = 64 + kSoftmaxThreads + 32;  // K producer, MMA, softmax, V producer
+constexpr int kRowsM = 128;    // query rows per work item (TMEM lanes)
+constexpr int kSoftmaxThreads = 128;  // warps 2-5, one per TMEM lane quarter
+constexpr int kVWarp = 6;             // V producer
+constexpr int kThreadsTC = 224;       // K producer, MMA issuer, 4 softmax warps, V producer
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 
 struct TcMaps {
@@ -77,17 +83,15 @@ struct TcCfg {
 };
 
 struct TcShared {
-  uint64_t q_ready;
   uint64_t k_full[8], v_full[8], k_empty[8], v_empty[8];
   uint64_t s_full[3], p_full[3], pv_done[3];
-  uint64_t o_final;
-  uint64_t v_fix;       // the partial prefix tile's V rows past the prefix end are zeroed
-  uint64_t xbar[4];     // row-pair exchange written, one per TMEM lane quarter (64 arrivals)
-  uint64_t xread[4];    // row-pair exchange read (64 arrivals)
-  float xch[256];       // [half][128 rows]
+  uint64_t q_ready;   // a work item's Q rows are in tensor memory (one phase per item)
+  uint64_t o_final;   // a work item's last P.V has completed
+  uint64_t o_free;    // a work item's O has been read out (the next item may overwrite it)
+  uint64_t v_fix;     // a partial prefix tile's V rows past the prefix end are zeroed
   uint32_t tmem_base;
   int abort_flag;
-  int last_split;       // this CTA merges the split partials of its row tile
+  int last_split;     // this CTA merges the split partials of its row tile
 };
 
 // All lanes of the warp wait; the outcome is made warp-uniform so that the
@@ -132,6 +136,37 @@ __device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, ui
       "}\n" ::"r"(d_tmem),
       "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
       : "memory");
+}
+
+// One work item: query rows mtile*128 .. of (request r, kv head kvh) against
+// prefix split `split`: prefix tiles j0 .. j0 + n_pref_here - 1, then (last
+// split only) the tile holding the block's own keys.
+struct TcWork {
+  int r, kvh, mtile, split, item, P;
+  int j0, n_pref_here, n_tiles, j_part;
+};
+
+// Work item `idx` of the flat list: (row tile, kv head) fastest, then the
+// valid work units (request, prefix split) in longest-first order.
+__device__ __forceinline__ TcWork tc_work(const SoftmaxParams& p, int n_mt, int idx) {
+  TcWork w;
+  w.mtile = idx % n_mt;
+  w.kvh = (idx / n_mt) % p.Hkv;
+  const int unit = p.order[idx / (n_mt * p.Hkv)];
+  w.r = unit / p.n_split;
+  w.split = unit % p.n_split;
+  w.item = w.r * p.Hkv + w.kvh;
+  w.P = p.prefix_len[w.r];
+  const int n_pref = (w.P + kTileN - 1) / kTileN;
+  const int tps = p.split_len / kTileN;
+  w.j0 = w.split * tps;
+  const int j1 = min(n_pref, w.j0 + tps);
+  w.n_pref_here = max(0, j1 - w.j0);
+  w.n_tiles = w.n_pref_here + (w.split == p.n_split - 1 ? 1 : 0);
+  // the last prefix tile when the prefix ends inside it (its V rows past the
+  // end are zeroed), else -1
+  w.j_part = (w.n_pref_here > 0 && j1 == n_pref && (w.P % kTileN) != 0) ? w.n_pref_here - 1 : -1;
+  return w;
 }
 
 }  // namespace
@@ -223,37 +258,74 @@ __device__ void finish_split(const SoftmaxParams& p, int item, int r, int kvh, i
   }
 }
 
-// Longest-first order of the work units u = (request r, prefix split), by
-// their tile count: a counting sort on one CTA (1024 threads, keys capped at
-// 4095 tiles).  Units with equal counts come in any order; each unit writes
-// its own outputs, so the results do not depend on it.
+// Validation and longest-first order of the work units u = (request r, prefix
+// split), on one CTA:
+//  - a request whose prefix length is out of range or whose prefix uses a page
+//    id outside [0, num_pages) is flagged in the status word and left out of
+//    the order (its outputs stay untouched);
+//  - the other units are counting-sorted by their tile count (keys capped at
+//    4095 tiles), longest first; *n_valid receives their number.
+// Units with equal counts come in any order; each unit writes its own
+// outputs, so the results do not depend on it.  Also zeroes the split-merge
+// counters.
 constexpr int kOrderThreads = 1024;
 constexpr int kOrderKeys = 4 * kOrderThreads;
 
 __global__ void __launch_bounds__(kOrderThreads) softmax_order_kernel(SoftmaxParams p) {
   __shared__ int start[kOrderKeys];
   __shared__ int wsum[kOrderThreads / 32];
+  __shared__ int n_valid;
   const int U = p.R * p.n_split;
   const int tps = p.split_len / kTileN;
   const int t = threadIdx.x;
+  const int nw = (p.R + 31) / 32;
+  const long long prefix_cap = (long long)p.max_pages * p.page_size;
+  for (int i = t; i < kOrderKeys; i += kOrderThreads) start[i] = 0;
+  for (int i = t; i < nw; i += kOrderThreads) p.bad_mask[i] = 0u;
+  if (p.counters) {
+    const int n_cnt = p.R * p.Hkv * ((p.B * p.G + kRowsM - 1) / kRowsM);
+    for (int i = t; i < n_cnt; i += kOrderThreads) p.counters[i] = 0;
+  }
+  if (t == 0) n_valid = 0;
+  __syncthreads();
+  for (int r = t; r < p.R; r += kOrderThreads) {
+    const int P = p.prefix_len[r];
+    if (P < 0 || P > prefix_cap) {
+      atomicOr(&p.bad_mask[r >> 5], 1u << (r & 31));
+      flag(p.dev_status, FLARE_DEV_BAD_PREFIX_LEN);
+    }
+  }
+  const long long n_entries = (long long)p.R * p.max_pages;
+  for (long long i = t; i < n_entries; i += kOrderThreads) {
+    const int r = (int)(i / p.max_pages), pg = (int)(i % p.max_pages);
+    const int P = p.prefix_len[r];
+    if (P < 0 || P > prefix_cap || (long long)pg * p.page_size >= P) continue;  // page unused
+    const int id = p.page_table[i];
+    if (id < 0 || id >= p.num_pages) {
+      atomicOr(&p.bad_mask[r >> 5], 1u << (r & 31));
+      flag(p.dev_status, FLARE_DEV_BAD_PAGE);
+    }
+  }
+  __syncthreads();
   auto key_of = [&](int u) -> int {
     const int r = u / p.n_split, split = u % p.n_split;
-    const int P = max(0, p.prefix_len[r]);  // bad lengths are flagged by the attention kernel
+    if (p.bad_mask[r >> 5] & (1u << (r & 31))) return -1;
+    const int P = p.prefix_len[r];
     const int n_pref = (P + kTileN - 1) / kTileN;
     const int j0 = split * tps;
     const int here = max(0, min(n_pref, j0 + tps) - j0);
     return min(here + (split == p.n_split - 1 ? 1 : 0), kOrderKeys - 1);
   };
-  for (int i = t; i < kOrderKeys; i += kOrderThreads) start[i] = 0;
-  if (p.counters) {
-    const int n_cnt = p.R * p.Hkv * ((p.B * p.G + kRowsM - 1) / kRowsM);
-    for (int i = t; i < n_cnt; i += kOrderThreads) p.counters[i] = 0;
+  for (int u = t; u < U; u += kOrderThreads) {
+    const int k = key_of(u);
+    if (k >= 0) {
+      atomicAdd(&start[k], 1);
+      atomicAdd(&n_valid, 1);
+    }
   }
   __syncthreads();
-  for (int u = t; u < U; u += kOrderThreads) atomicAdd(&start[key_of(u)], 1);
-  __syncthreads();
-  // start[k] = number of units with a larger key; thread t owns the keys at
-  // descending positions 4t .. 4t+3
+  // start[k] = number of valid units with a larger key; thread t owns the
+  // keys at descending positions 4t .. 4t+3
   int v[4], sum = 0;
 #pragma unroll
   for (int e = 0; e < 4; ++e) {
@@ -286,62 +358,61 @@ __global__ void __launch_bounds__(kOrderThreads) softmax_order_kernel(SoftmaxPar
     run += v[e];
   }
   __syncthreads();
-  for (int u = t; u < U; u += kOrderThreads) p.order[atomicAdd(&start[key_of(u)], 1)] = u;
+  for (int u = t; u < U; u += kOrderThreads) {
+    const int k = key_of(u);
+    if (k >= 0) p.order[atomicAdd(&start[k], 1)] = u;
+  }
+  if (t == 0) *p.n_valid = n_valid;
 }
 
+// The attention kernel.  Unsplit prefixes (n_split == 1): one CTA per SM walks
+// the work items in snake order over the CTAs (round k takes items k*G ..
+// k*G + G - 1, in reverse on odd rounds), so that tensor memory, barriers and
+// tensor maps are set up once and the next item's loads and S products
+// overlap the current item's epilogue.  Split prefixes: one CTA per work item,
+// and the last split of a row tile to finish merges the partials.
 template <int D>
 __global__ void __launch_bounds__(kThreadsTC, 1)
     softmax_tc_kernel(const __grid_constant__ TcMaps maps, SoftmaxParams p) {
   using C = TcCfg<D>;
+  constexpr int kSB = C::kSBuf;
   extern __shared__ uint8_t smem_raw[];
   __shared__ TcShared sh;
   uint8_t* base = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t* Ks = base;
   uint8_t* Vs = Ks + C::kKStages * C::kKVBytes;
 
-  // flat grid: (query-row tile, kv head) fastest, then the work units
-  // (request, prefix split) in longest-first order, so that the CTAs that share
-  // a unit's K/V run together and the longest units start first
   const int M = p.B * p.G;
   const int n_mt = (M + kRowsM - 1) / kRowsM;
-  const int mtile = blockIdx.x % n_mt;
-  const int kvh = (blockIdx.x / n_mt) % p.Hkv;
-  const int z = blockIdx.x / (n_mt * p.Hkv);
-  const int unit = p.order ? p.order[z] : z;
-  const int r = unit / p.n_split, split = unit % p.n_split;
-  const int item = r * p.Hkv + kvh;
+  const int n_items = n_mt * p.Hkv * *p.n_valid;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-
-  const int P = p.prefix_len[r];
-  const int bad = check_request_pages(p.page_table, P, r, p.max_pages, p.page_size, p.num_pages);
-  if (bad) {
-    if (tid == 0) flag(p.dev_status, bad);
-    return;
-  }
-  // tiles of this split: prefix tiles [j0, j1) then (last split only) the block tile
-  const int n_pref = (P + kTileN - 1) / kTileN;
-  const int tps = p.split_len / kTileN;
-  const int j0 = split * tps;
-  const int j1 = min(n_pref, j0 + tps);
-  const int n_pref_here = max(0, j1 - j0);
-  const bool has_blk = split == p.n_split - 1;
-  // the last prefix tile of this split when it ends inside the tile, else -1
-  const int j_part = (n_pref_here > 0 && j1 == n_pref && (P % kTileN) != 0) ? n_pref_here - 1 : -1;
-  const int n_tiles = n_pref_here + (has_blk ? 1 : 0);
-  const size_t ws_row0 = ((size_t)item * p.n_split + split) * M;
-
-  if (n_tiles == 0) {  // empty split: mark its partial as empty for the merge
-    for (int i = tid; i < kRowsM; i += blockDim.x) {
-      const int m = mtile * kRowsM + i;
-      if (m < M) p.ws_lse[ws_row0 + m] = -INFINITY;
+  const bool split_mode = p.n_split > 1;
+  // k-th work item of this CTA, or -1
+  auto item_of = [&](int k) -> int {
+    const int G = gridDim.x, b = blockIdx.x;
+    if (split_mode) return (k == 0 && b < n_items) ? b : -1;
+    const int idx = k * G + ((k & 1) ? G - 1 - b : b);
+    return idx < n_items ? idx : -1;
+  };
+  const int idx0 = item_of(0);
+  if (idx0 < 0) return;
+  if (split_mode) {
+    const TcWork w = tc_work(p, n_mt, idx0);
+    if (w.n_tiles == 0) {  // empty split: mark its partial as empty for the merge
+      const size_t ws_row0 = ((size_t)w.item * p.n_split + w.split) * M;
+      for (int i = tid; i < kRowsM; i += blockDim.x) {
+        const int m = w.mtile * kRowsM + i;
+        if (m < M) p.ws_lse[ws_row0 + m] = -INFINITY;
+      }
+      finish_split<D>(p, w.item, w.r, w.kvh, w.mtile, n_mt, &sh.last_split,
+                      reinterpret_cast<float*>(Ks));
+      return;
     }
-    finish_split<D>(p, item, r, kvh, mtile, n_mt, &sh.last_split, reinterpret_cast<float*>(Ks));
-    return;
   }
 
   if (tid == 0) {
     sh.abort_flag = 0;
-    tc::mbar_init(&sh.q_ready, kSoftmaxThreads);
+    sh.last_split = 0;
     for (int s = 0; s < C::kKStages; ++s) {
       tc::mbar_init(&sh.k_full[s], 1);
       tc::mbar_init(&sh.k_empty[s], 1);
@@ -355,12 +426,10 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
       tc::mbar_init(&sh.p_full[b], kSoftmaxThreads);
       tc::mbar_init(&sh.pv_done[b], 1);
     }
+    tc::mbar_init(&sh.q_ready, kSoftmaxThreads);
     tc::mbar_init(&sh.o_final, 1);
+    tc::mbar_init(&sh.o_free, kSoftmaxThreads);
     tc::mbar_init(&sh.v_fix, 1);
-    for (int q = 0; q < 4; ++q) {
-      tc::mbar_init(&sh.xbar[q], 32 * kSplit);
-      tc::mbar_init(&sh.xread[q], 32 * kSplit);
-    }
     tc::fence_mbar_init();
   }
   if (warp == 1) tc::tmem_alloc(&sh.tmem_base, C::kTmemCols);
@@ -371,66 +440,56 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
   const uint32_t tmem_o = tmem;
   const uint32_t tmem_q = tmem + C::kQCol;
   const uint32_t tmem_s = tmem + C::kSCol;
-  constexpr int kSB = C::kSBuf;
-
-  // tile index -> (is block tile, prefix tile number)
-  auto tile_kind = [&](int j, int& ptile) -> bool {
-    if (j < n_pref_here) {
-      ptile = j0 + j;
-      return false;
-    }
-    ptile = -1;
-    return true;
-  };
-  // valid key columns of a tile
-  auto tile_valid = [&](int j) -> int {
-    int pt;
-    if (tile_kind(j, pt)) return p.B;
-    return min(kTileN, P - pt * kTileN);
-  };
 
   if (warp == 0 || warp == kVWarp) {
     // ------------------------------------------------------------ producers
-    // warp 0 streams the K tiles and warp kVWarp the V tiles, each into its
-    // own ring, so neither waits behind the other's slot.
+    // warp 0 streams the K tiles and warp kVWarp the V tiles of every work
+    // item of this CTA, each into its own ring (slot = running tile count mod
+    // ring depth), so neither waits behind the other's slot.
     if (lane == 0) {
       const int kv = warp == 0 ? 0 : 1;
       const CUtensorMap* pool_map = kv ? &maps.vpool : &maps.kpool;
       const CUtensorMap* blk_map = kv ? &maps.vblk : &maps.kblk;
       tc::prefetch_tmap(pool_map);
+      tc::prefetch_tmap(blk_map);
       const int box_rows = p.page_size < kTileN ? p.page_size : kTileN;
       const int ns = kv ? C::kVStages : C::kKStages;
       uint8_t* ring = kv ? Vs : Ks;
       bool ok = true;
-      for (int j = 0; j < n_tiles && ok && !aborted(sh); ++j) {
-        const int st = j % ns;
-        const uint32_t ph = (uint32_t)(j / ns) & 1u;
-        uint64_t* empty = kv ? &sh.v_empty[st] : &sh.k_empty[st];
-        uint64_t* full = kv ? &sh.v_full[st] : &sh.k_full[st];
-        uint8_t* dst = ring + st * C::kKVBytes;
-        if (!tc::mbar_wait(empty, ph ^ 1u, &sh.abort_flag)) {
-          ok = false;
-          break;
-        }
-        int pt;
-        if (tile_kind(j, pt)) {
-          tc::mbar_expect_tx(full, C::kKVBytes);
-          for (int c = 0; c < C::kChunks; ++c)
-            tc::tma_load_4d(dst + c * (kTileN * 128), blk_map, full, c * 64, kvh, 0, r);
-        } else {
-          const int tok0 = pt * kTileN;
-          const int valid = min(kTileN, P - tok0);
+      int g = 0;  // running tile count
+      for (int k = 0; ok && !aborted(sh); ++k) {
+        const int idx = item_of(k);
+        if (idx < 0) break;
+        const TcWork w = tc_work(p, n_mt, idx);
+        for (int j = 0; j < w.n_tiles; ++j, ++g) {
+          const int st = g % ns;
+          const uint32_t ph = (uint32_t)(g / ns) & 1u;
+          uint64_t* empty = kv ? &sh.v_empty[st] : &sh.k_empty[st];
+          uint64_t* full = kv ? &sh.v_full[st] : &sh.k_full[st];
+          uint8_t* dst = ring + st * C::kKVBytes;
+          if (!tc::mbar_wait(empty, ph ^ 1u, &sh.abort_flag)) {
+            ok = false;
+            break;
+          }
+          if (j >= w.n_pref_here) {  // the block's own keys / values
+            tc::mbar_expect_tx(full, C::kKVBytes);
+            for (int c = 0; c < C::kChunks; ++c)
+              tc::tma_load_4d(dst + c * (kTileN * 128), blk_map, full, c * 64, w.kvh, 0, w.r);
+            continue;
+          }
+          const int tok0 = (w.j0 + j) * kTileN;
+          const int valid = min(kTileN, w.P - tok0);
           const int nbox = (valid + box_rows - 1) / box_rows;
           tc::mbar_expect_tx(full, (uint32_t)(C::kChunks * nbox * box_rows * 128));
           for (int bx = 0; bx < nbox; ++bx) {
             const int tok = tok0 + bx * box_rows;
-            const int page = p.page_table[(size_t)r * p.max_pages + tok / p.page_size];
+            const int page = p.page_table[(size_t)w.r * p.max_pages + tok / p.page_size];
             const int row0 = tok % p.page_size;
             for (int c = 0; c < C::kChunks; ++c)
               tc::tma_load_4d(dst + c * (kTileN * 128) + bx * box_rows * 128, pool_map, full,
-                              c * 64, row0, kvh, page);
+                              c * 64, row0, w.kvh, page);
           }
-          if (kv && j == j_part) {
+          if (kv && j == w.j_part) {
             // rows past the prefix end hold stale (possibly poisoned) cache
             // rows; zero them once the load has landed so that a zero
             // probability never meets a NaN (0 * NaN) in P.V
@@ -459,241 +518,252 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
       const uint32_t id_o = tc::idesc_bf16(kRowsM, D, false, true);
       const uint64_t kdesc0 = tc::sdesc_sw128(tc::smem_u32(Ks), 16, 1024);
       const uint64_t vdesc0 = tc::sdesc_sw128(tc::smem_u32(Vs), kTileN * 128, 1024);
-      bool ok = tc::mbar_wait(&sh.q_ready, 0, &sh.abort_flag);
-      auto issue_pv = [&](int i) -> bool {
-        const int st = i % C::kVStages;
-        const int pb = i % kSB;
-        if (!tc::mbar_wait(&sh.p_full[pb], (uint32_t)(i / kSB) & 1u, &sh.abort_flag))
-          return false;
-        const bool ready = i == j_part
-                               ? tc::mbar_wait(&sh.v_fix, 0, &sh.abort_flag)
-                               : tc::mbar_wait(&sh.v_full[st], (uint32_t)(i / C::kVStages) & 1u,
-                                               &sh.abort_flag);
-        if (!ready) return false;
-        tc::fence_after_sync();
-        const uint64_t vd = vdesc0 + (uint64_t)((st * C::kKVBytes) >> 4);
-#pragma unroll
-        for (int kk = 0; kk < kTileN / 16; ++kk)
-          mma_bf16_ts(tmem_o, tmem_s + pb * kTileN + kk * 8, vd + (uint64_t)(kk * (2048 >> 4)),
-                      id_o, (i > 0 || kk > 0) ? 1u : 0u);
-        tc::mma_commit(&sh.pv_done[pb]);
-        tc::mma_commit(&sh.v_empty[st]);
-        return true;
-      };
-      // S_j = Q K_j^T into S buffer j % kSB (Q from tensor memory)
-      auto issue_s = [&](int j) -> bool {
-        const int st = j % C::kKStages;
-        const int sb = j % kSB;
-        if (!tc::mbar_wait(&sh.k_full[st], (uint32_t)(j / C::kKStages) & 1u, &sh.abort_flag))
-          return false;
-        tc::fence_after_sync();
-        const uint64_t kd = kdesc0 + (uint64_t)((st * C::kKVBytes) >> 4);
-#pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const int c = kk >> 2, off = (kk & 3) * 32;
-          mma_bf16_ts(tmem_s + sb * kTileN, tmem_q + kk * 8,
-                      kd + (uint64_t)((c * (kTileN * 128) + off) >> 4), id_s, kk > 0 ? 1u : 0u);
+      bool ok = true;
+      int g = 0;     // running tile count
+      int nfix = 0;  // partial tiles seen
+      for (int k = 0; ok && !aborted(sh); ++k) {
+        const int idx = item_of(k);
+        if (idx < 0) break;
+        const TcWork w = tc_work(p, n_mt, idx);
+        if (!tc::mbar_wait(&sh.q_ready, (uint32_t)k & 1u, &sh.abort_flag)) {
+          ok = false;
+          break;
         }
-        tc::mma_commit(&sh.s_full[sb]);
-        tc::mma_commit(&sh.k_empty[st]);
-        return true;
-      };
-      // Three S buffers: issue order S0, S1, S2, PV0, S3, PV1, ...: S_{j+2} is
-      // queued before the P.V of tile j waits on its probabilities and reuses
-      // the buffer of tile j-1, whose P.V was issued (and, in issue order,
-      // executes) before it.  Two buffers: S0, S1, PV0, S2, PV1, S3, ...:
-      // S_{j+2} reuses the buffer of tile j, so it follows P_j V_j.
-      for (int j = 0; j < 2 && j < n_tiles && ok; ++j) ok = issue_s(j);
-      for (int j = 0; j < n_tiles && ok; ++j) {
-        if (kSB == 3) {
-          if (j + 2 < n_tiles) ok = issue_s(j + 2);
-          if (ok) ok = issue_pv(j);
-        } else {
-          ok = issue_pv(j);
-          if (ok && j + 2 < n_tiles) ok = issue_s(j + 2);
+        auto issue_pv = [&](int j) -> bool {
+          const int gg = g + j;
+          const int st = gg % C::kVStages;
+          const int pb = gg % kSB;
+          if (!tc::mbar_wait(&sh.p_full[pb], (uint32_t)(gg / kSB) & 1u, &sh.abort_flag))
+            return false;
+          // the first P.V of an item overwrites O: the previous item's O must be out
+          if (j == 0 && k > 0 &&
+              !tc::mbar_wait(&sh.o_free, (uint32_t)(k - 1) & 1u, &sh.abort_flag))
+            return false;
+          bool ready;
+          if (j == w.j_part) {
+            ready = tc::mbar_wait(&sh.v_fix, (uint32_t)nfix & 1u, &sh.abort_flag);
+            ++nfix;
+          } else {
+            ready = tc::mbar_wait(&sh.v_full[st], (uint32_t)(gg / C::kVStages) & 1u,
+                                  &sh.abort_flag);
+          }
+          if (!ready) return false;
+          tc::fence_after_sync();
+          const uint64_t vd = vdesc0 + (uint64_t)((st * C::kKVBytes) >> 4);
+#pragma unroll
+          for (int kk = 0; kk < kTileN / 16; ++kk)
+            mma_bf16_ts(tmem_o, tmem_s + pb * kTileN + kk * 8, vd + (uint64_t)(kk * (2048 >> 4)),
+                        id_o, (j > 0 || kk > 0) ? 1u : 0u);
+          tc::mma_commit(&sh.pv_done[pb]);
+          tc::mma_commit(&sh.v_empty[st]);
+          return true;
+        };
+        // S_j = Q K_j^T into S buffer (g + j) % kSB (Q from tensor memory)
+        auto issue_s = [&](int j) -> bool {
+          const int gg = g + j;
+          const int st = gg % C::kKStages;
+          const int sb = gg % kSB;
+          if (!tc::mbar_wait(&sh.k_full[st], (uint32_t)(gg / C::kKStages) & 1u, &sh.abort_flag))
+            return false;
+          tc::fence_after_sync();
+          const uint64_t kd = kdesc0 + (uint64_t)((st * C::kKVBytes) >> 4);
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const int c = kk >> 2, off = (kk & 3) * 32;
+            mma_bf16_ts(tmem_s + sb * kTileN, tmem_q + kk * 8,
+                        kd + (uint64_t)((c * (kTileN * 128) + off) >> 4), id_s, kk > 0 ? 1u : 0u);
+          }
+          tc::mma_commit(&sh.s_full[sb]);
+          tc::mma_commit(&sh.k_empty[st]);
+          return true;
+        };
+        // Three S buffers: issue order S0, S1, S2, PV0, S3, PV1, ...: S_{j+2}
+        // is queued before the P.V of tile j waits on its probabilities and
+        // reuses the buffer of tile j-1, whose P.V was issued (and, in issue
+        // order, executes) before it.  Two buffers: S0, S1, PV0, S2, PV1, ...:
+        // S_{j+2} reuses the buffer of tile j, so it follows P_j V_j.  The
+        // running tile count carries the buffers across work items.
+        const int n = w.n_tiles;
+        for (int j = 0; j < 2 && j < n && ok; ++j) ok = issue_s(j);
+        for (int j = 0; j < n && ok; ++j) {
+          if (kSB == 3) {
+            if (j + 2 < n) ok = issue_s(j + 2);
+            if (ok) ok = issue_pv(j);
+          } else {
+            ok = issue_pv(j);
+            if (ok && j + 2 < n) ok = issue_s(j + 2);
+          }
         }
+        if (ok) tc::mma_commit(&sh.o_final);
+        g += n;
       }
-      if (ok) tc::mma_commit(&sh.o_final);
       if (!ok) set_abort(sh, p.dev_status);
     }
     __syncwarp();
   } else {
     // ------------------------------------------------------------ softmax warps
-    // Eight warps: warp w reads TMEM lanes 32*(w%4).. (its 32 rows) and key
-    // columns 32*half.. of each tile; the two warps of a row pair exchange
-    // their tile maxima through shared memory every tile.
+    // warp w reads TMEM lanes 32*(w%4).. (its 32 query rows) and all 64 key
+    // columns of each tile
     const int quarter = warp & 3;
-    const int half = (warp - 2) >> 2;
     const int row = quarter * 32 + lane;
-    const int m = mtile * kRowsM + row;
-    const int trow = m / p.G;
     const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
-    constexpr int kDh = D / kSplit;       // Q elements / output columns this warp handles
-    constexpr int kCols = kTileN / kSplit;  // key columns of each tile this warp handles
 
-    // Q row (this warp's D/kSplit elements) into tensor memory as bf16 pairs,
-    // the A operand of S = Q K^T; rows past the block's B*G are zero
-    {
-      const int g = m % p.G;
+    // Q row of work item w into tensor memory as bf16 pairs, the A operand of
+    // S = Q K^T; rows past the block's B*G are zero
+    auto load_q = [&](const TcWork& w) {
+      const int m = w.mtile * kRowsM + row;
       const bool live = m < M;
+      const int trow = live ? m / p.G : 0, g = m % p.G;
       const uint4* qrow = reinterpret_cast<const uint4*>(
           static_cast<const __nv_bfloat16*>(p.q) +
-          (((size_t)r * p.B + (live ? trow : 0)) * p.Hq + kvh * p.G + g) * D + half * kDh);
-      constexpr int kWords = kDh / 2;                        // TMEM columns of this warp
+          (((size_t)w.r * p.B + trow) * p.Hq + w.kvh * p.G + g) * D);
+      constexpr int kWords = D / 2;                          // TMEM columns of a row
       constexpr int kBatch = kWords < 64 ? kWords : 64;      // columns per batch of loads
 #pragma unroll 1
       for (int c0 = 0; c0 < kWords; c0 += kBatch) {
-        uint32_t w[kBatch];
+        uint32_t q[kBatch];
 #pragma unroll
         for (int q4 = 0; q4 < kBatch / 4; ++q4) {
           const uint4 v = live ? qrow[(c0 / 4) + q4] : make_uint4(0u, 0u, 0u, 0u);
-          w[4 * q4] = v.x;
-          w[4 * q4 + 1] = v.y;
-          w[4 * q4 + 2] = v.z;
-          w[4 * q4 + 3] = v.w;
+          q[4 * q4] = v.x;
+          q[4 * q4 + 1] = v.y;
+          q[4 * q4 + 2] = v.z;
+          q[4 * q4 + 3] = v.w;
         }
 #pragma unroll
         for (int c = 0; c < kBatch; c += 16)
-          tmem_st16(tmem_q + lane_off + half * kWords + c0 + c,
-                    *reinterpret_cast<uint32_t(*)[16]>(&w[c]));
+          tmem_st16(tmem_q + lane_off + c0 + c, *reinterpret_cast<uint32_t(*)[16]>(&q[c]));
       }
       tmem_st_wait();
       tc::fence_before_sync();
       tc::mbar_arrive(&sh.q_ready);
-    }
+    };
 
-    float m_run = -INFINITY, l_run = 0.f;  // l_run: this half's share of the row sum
     bool ok = true;
-    for (int j = 0; j < n_tiles; ++j) {
-      const int sb = j % kSB;
-      if (!warp_wait(&sh.s_full[sb], (uint32_t)(j / kSB) & 1u, &sh.abort_flag)) {
-        ok = false;
+    int g = 0;  // running tile count
+    int idx = idx0;
+    TcWork w = tc_work(p, n_mt, idx);
+    load_q(w);
+    for (int k = 0; idx >= 0; ++k) {
+      const int m = w.mtile * kRowsM + row;
+      const int trow = m / p.G;
+      float m_run = -INFINITY, l_run = 0.f;
+      for (int j = 0; j < w.n_tiles; ++j) {
+        const int gg = g + j;
+        const int sb = gg % kSB;
+        if (!warp_wait(&sh.s_full[sb], (uint32_t)(gg / kSB) & 1u, &sh.abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc::fence_after_sync();
+        const uint32_t sbuf = tmem_s + lane_off + sb * kTileN;
+        uint32_t sr[kTileN];
+#pragma unroll
+        for (int c = 0; c < kTileN; c += 16)
+          tc::tmem_ld16(sbuf + c, *reinterpret_cast<uint32_t(*)[16]>(&sr[c]));
+        tc::tmem_ld_wait();
+
+        const bool blk = j >= w.n_pref_here;
+        const int valid = blk ? p.B : min(kTileN, w.P - (w.j0 + j) * kTileN);
+        const bool full = !blk && valid == kTileN;  // prefix tile: no mask at all
+        const int lim = full ? kTileN : ((blk && p.causal) ? min(valid, trow + 1) : valid);
+        // tile maximum of the raw scores (scale >= 0 keeps the order)
+        float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+        for (int c = 0; c < kTileN; ++c)
+          if (full || c < lim) mx[c & 3] = fmaxf(mx[c & 3], __uint_as_float(sr[c]));
+        const float mt = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+        const float m_new = fmaxf(m_run, mt * p.scale_log2);
+        const bool need = (j == 0) || (m_new > m_run + kRescaleThreshold);
+        const bool warp_rescale = __any_sync(0xffffffffu, need);
+        float m_use = m_run;
+        if (warp_rescale) m_use = (j == 0 || m_new > m_run) ? m_new : m_run;
+        const float corr = (j == 0) ? 0.f : tc::ex2(m_run - m_use);
+        const float neg_m = -m_use;
+        float sum0 = 0.f, sum1 = 0.f;
+        uint32_t pk[kTileN / 2];
+        if (full) {
+#pragma unroll
+          for (int c = 0; c < kTileN; c += 2) {
+            const float p0 = tc::ex2(fmaf(__uint_as_float(sr[c]), p.scale_log2, neg_m));
+            const float p1 = tc::ex2(fmaf(__uint_as_float(sr[c + 1]), p.scale_log2, neg_m));
+            sum0 += p0;
+            sum1 += p1;
+            __nv_bfloat162 h2 = __floats2bfloat162_rn(p0, p1);
+            pk[c / 2] = *reinterpret_cast<uint32_t*>(&h2);
+          }
+        } else {
+#pragma unroll
+          for (int c = 0; c < kTileN; c += 2) {
+            const float p0 =
+                c < lim ? tc::ex2(fmaf(__uint_as_float(sr[c]), p.scale_log2, neg_m)) : 0.f;
+            const float p1 =
+                c + 1 < lim ? tc::ex2(fmaf(__uint_as_float(sr[c + 1]), p.scale_log2, neg_m))
+                            : 0.f;
+            sum0 += p0;
+            sum1 += p1;
+            __nv_bfloat162 h2 = __floats2bfloat162_rn(p0, p1);
+            pk[c / 2] = *reinterpret_cast<uint32_t*>(&h2);
+          }
+        }
+        const float sum = sum0 + sum1;
+        l_run = (j == 0) ? sum : l_run * corr + sum;
+        // rescale O when the running max moved (the P.V of the previous tile done)
+        if (warp_rescale && j >= 1) {
+          const int pb = (gg - 1) % kSB;
+          if (!warp_wait(&sh.pv_done[pb], (uint32_t)((gg - 1) / kSB) & 1u, &sh.abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc::fence_after_sync();
+#pragma unroll 1
+          for (int c = 0; c < D; c += 16) {
+            uint32_t o[16];
+            tc::tmem_ld16(tmem_o + lane_off + c, o);
+            tc::tmem_ld_wait();
+#pragma unroll
+            for (int i = 0; i < 16; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * corr);
+            tmem_st16(tmem_o + lane_off + c, o);
+          }
+        }
+        m_run = m_use;
+        // P (bf16 pairs) over the first 32 columns of the S buffer
+#pragma unroll
+        for (int c = 0; c < kTileN / 2; c += 16)
+          tmem_st16(sbuf + c, *reinterpret_cast<uint32_t(*)[16]>(&pk[c]));
+        tmem_st_wait();
+        tc::fence_before_sync();
+        tc::mbar_arrive(&sh.p_full[sb]);
+      }
+      g += w.n_tiles;
+      if (ok && aborted(sh)) ok = false;
+      // the next item's Q can go into tensor memory now: every S product of
+      // this item has completed
+      const int idx_next = ok ? item_of(k + 1) : -1;
+      TcWork wn = w;
+      if (idx_next >= 0) {
+        wn = tc_work(p, n_mt, idx_next);
+        load_q(wn);
+      }
+      // epilogue: O / l (or the split partial) and the log-sum-exp
+      if (ok && !warp_wait(&sh.o_final, (uint32_t)k & 1u, &sh.abort_flag)) ok = false;
+      if (!ok) {
+        set_abort(sh, p.dev_status);
         break;
       }
       tc::fence_after_sync();
-      const uint32_t sbuf = tmem_s + lane_off + sb * kTileN;
-      uint32_t sr[kCols];
-#pragma unroll
-      for (int c = 0; c < kCols; c += 16)
-        tc::tmem_ld16(sbuf + kCols * half + c, *reinterpret_cast<uint32_t(*)[16]>(&sr[c]));
-      tc::tmem_ld_wait();
-
-      int pt;
-      const bool blk = tile_kind(j, pt);
-      const int valid = tile_valid(j);
-      const bool full = !blk && valid == kTileN;  // prefix tile: no mask at all
-      const int lim = full ? kTileN : ((blk && p.causal) ? min(valid, trow + 1) : valid);
-      // tile maximum of the raw scores (scale >= 0 keeps the order)
-      float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-#pragma unroll
-      for (int c = 0; c < kCols; ++c)
-        if (full || kCols * half + c < lim) mx[c & 3] = fmaxf(mx[c & 3], __uint_as_float(sr[c]));
-      float mt = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
-      // the partner has read this slot's previous value before it is overwritten;
-      // this exchange also orders both halves' S reads before either writes P.
-      if (kSplit > 1) {
-        if (j >= 1 && !warp_wait(&sh.xread[quarter], (uint32_t)(j - 1) & 1u, &sh.abort_flag)) {
-          ok = false;
-          break;
-        }
-        sh.xch[half * 128 + row] = mt;
-        tc::fence_before_sync();
-        tc::mbar_arrive(&sh.xbar[quarter]);
-        if (!warp_wait(&sh.xbar[quarter], (uint32_t)j & 1u, &sh.abort_flag)) {
-          ok = false;
-          break;
-        }
-        tc::fence_after_sync();
-        mt = fmaxf(mt, sh.xch[(1 - half) * 128 + row]);
-        tc::mbar_arrive(&sh.xread[quarter]);
-      }
-      const float m_new = fmaxf(m_run, mt * p.scale_log2);
-      const bool need = (j == 0) || (m_new > m_run + kRescaleThreshold);
-      const bool warp_rescale = __any_sync(0xffffffffu, need);
-      float m_use = m_run;
-      if (warp_rescale) m_use = (j == 0 || m_new > m_run) ? m_new : m_run;
-      const float corr = (j == 0) ? 0.f : tc::ex2(m_run - m_use);
-      const float neg_m = -m_use;
-      float sum0 = 0.f, sum1 = 0.f;
-      uint32_t pk[kCols / 2];
-      if (full) {
-#pragma unroll
-        for (int c = 0; c < kCols; c += 2) {
-          const float p0 = tc::ex2(fmaf(__uint_as_float(sr[c]), p.scale_log2, neg_m));
-          const float p1 = tc::ex2(fmaf(__uint_as_float(sr[c + 1]), p.scale_log2, neg_m));
-          sum0 += p0;
-          sum1 += p1;
-          __nv_bfloat162 h2 = __floats2bfloat162_rn(p0, p1);
-          pk[c / 2] = *reinterpret_cast<uint32_t*>(&h2);
-        }
-      } else {
-#pragma unroll
-        for (int c = 0; c < kCols; c += 2) {
-          const int col = kCols * half + c;
-          const float p0 =
-              col < lim ? tc::ex2(fmaf(__uint_as_float(sr[c]), p.scale_log2, neg_m)) : 0.f;
-          const float p1 =
-              col + 1 < lim ? tc::ex2(fmaf(__uint_as_float(sr[c + 1]), p.scale_log2, neg_m)) : 0.f;
-          sum0 += p0;
-          sum1 += p1;
-          __nv_bfloat162 h2 = __floats2bfloat162_rn(p0, p1);
-          pk[c / 2] = *reinterpret_cast<uint32_t*>(&h2);
-        }
-      }
-      const float sum = sum0 + sum1;
-      l_run = (j == 0) ? sum : l_run * corr + sum;
-      // rescale this half's O columns when the running max moved (P.V of tile j-1 done)
-      if (warp_rescale && j >= 1) {
-        const int pb = (j - 1) % kSB;
-        if (!warp_wait(&sh.pv_done[pb], (uint32_t)((j - 1) / kSB) & 1u, &sh.abort_flag)) {
-          ok = false;
-          break;
-        }
-        tc::fence_after_sync();
+      const bool write = m < M;
+      const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
+      const int gq = m % p.G;
+      const size_t orow = (((size_t)w.r * p.B + trow) * p.Hq + w.kvh * p.G + gq);
+      const size_t ws_row = ((size_t)w.item * p.n_split + w.split) * M + m;
 #pragma unroll 1
-        for (int c = half * kDh; c < (half + 1) * kDh; c += 16) {
-          uint32_t o[16];
-          tc::tmem_ld16(tmem_o + lane_off + c, o);
-          tc::tmem_ld_wait();
-#pragma unroll
-          for (int i = 0; i < 16; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * corr);
-          tmem_st16(tmem_o + lane_off + c, o);
-        }
-      }
-      m_run = m_use;
-      // P (bf16 pairs) over this warp's kCols / 2 columns of the S buffer
-#pragma unroll
-      for (int c = 0; c < kCols / 2; c += 16)
-        tmem_st16(sbuf + (kCols / 2) * half + c, *reinterpret_cast<uint32_t(*)[16]>(&pk[c]));
-      tmem_st_wait();
-      tc::fence_before_sync();
-      tc::mbar_arrive(&sh.p_full[sb]);
-    }
-    // row sum = the two halves' shares
-    if (kSplit > 1 && ok &&
-        !warp_wait(&sh.xread[quarter], (uint32_t)(n_tiles - 1) & 1u, &sh.abort_flag))
-      ok = false;
-    if (kSplit > 1 && ok) {
-      sh.xch[half * 128 + row] = l_run;
-      tc::mbar_arrive(&sh.xbar[quarter]);
-      if (!warp_wait(&sh.xbar[quarter], (uint32_t)n_tiles & 1u, &sh.abort_flag)) ok = false;
-      if (ok) l_run += sh.xch[(1 - half) * 128 + row];
-    }
-    if (ok && !warp_wait(&sh.o_final, 0, &sh.abort_flag)) ok = false;
-    if (!ok) set_abort(sh, p.dev_status);
-    tc::fence_after_sync();
-    const bool write = ok && m < M && !aborted(sh);
-    const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
-    const int g = m % p.G;
-    const size_t orow = (((size_t)r * p.B + trow) * p.Hq + kvh * p.G + g);
-    if (ok) {
-#pragma unroll 1
-      for (int c = half * kDh; c < (half + 1) * kDh; c += 16) {
+      for (int c = 0; c < D; c += 16) {
         uint32_t o[16];
         tc::tmem_ld16(tmem_o + lane_off + c, o);
         tc::tmem_ld_wait();
         if (!write) continue;
-        if (p.n_split == 1) {
+        if (!split_mode) {
           uint32_t pkd[8];
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
@@ -705,7 +775,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
           dst[0] = make_uint4(pkd[0], pkd[1], pkd[2], pkd[3]);
           dst[1] = make_uint4(pkd[4], pkd[5], pkd[6], pkd[7]);
         } else {
-          float4* dst = reinterpret_cast<float4*>(p.ws_o + (ws_row0 + m) * D + c);
+          float4* dst = reinterpret_cast<float4*>(p.ws_o + ws_row * D + c);
 #pragma unroll
           for (int i = 0; i < 4; ++i)
             dst[i] = make_float4(__uint_as_float(o[4 * i]) * inv, __uint_as_float(o[4 * i + 1]) * inv,
@@ -713,15 +783,20 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                                  __uint_as_float(o[4 * i + 3]) * inv);
         }
       }
-    }
-    if (write && half == 0) {
-      const float lse = l_run > 0.f ? (m_run + __log2f(l_run)) * 0.6931471805599453f : -INFINITY;
-      if (p.n_split == 1) {
-        if (p.lse) p.lse[orow] = lse;
-      } else {
-        p.ws_lse[ws_row0 + m] = lse;
+      if (write) {
+        const float lse = l_run > 0.f ? (m_run + __log2f(l_run)) * 0.6931471805599453f : -INFINITY;
+        if (!split_mode) {
+          if (p.lse) p.lse[orow] = lse;
+        } else {
+          p.ws_lse[ws_row] = lse;
+        }
       }
+      tc::fence_before_sync();
+      tc::mbar_arrive(&sh.o_free);
+      idx = idx_next;
+      w = wn;
     }
+    if (!ok) set_abort(sh, p.dev_status);
   }
   tc::fence_before_sync();
   __syncthreads();
@@ -730,8 +805,11 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     tc::tmem_dealloc(tmem, C::kTmemCols);
   }
   // a CTA that gave up wrote no partial: its row tile is never merged
-  if (p.n_split > 1 && !aborted(sh))  // the K/V rings are free: merge weights go there
-    finish_split<D>(p, item, r, kvh, mtile, n_mt, &sh.last_split, reinterpret_cast<float*>(Ks));
+  if (split_mode && !aborted(sh)) {  // the K/V rings are free: merge weights go there
+    const TcWork w = tc_work(p, n_mt, idx0);
+    finish_split<D>(p, w.item, w.r, w.kvh, w.mtile, n_mt, &sh.last_split,
+                    reinterpret_cast<float*>(Ks));
+  }
 }
 
 // ------------------------------------------------------------------ host side
@@ -795,16 +873,12 @@ cudaError_t launch_tc_d(const SoftmaxParams& p, const SoftmaxPlan& plan, cudaStr
   cudaError_t err = cudaFuncSetAttribute(softmax_tc_kernel<D>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (err != cudaSuccess) return err;
-  const int M = p.B * p.G;
-  if (p.order) {
-    softmax_order_kernel<<<1, kOrderThreads, 0, stream>>>(p);
-    note_launches(1);
-    err = cudaGetLastError();
-    if (err != cudaSuccess) return err;
-  }
-  const long long n_cta = (long long)((M + kRowsM - 1) / kRowsM) * p.Hkv * p.R * plan.n_split;
-  if (n_cta > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-  softmax_tc_kernel<D><<<(unsigned)n_cta, kThreadsTC, smem, stream>>>(maps, p);
+  if (!p.order || !p.n_valid || !p.bad_mask || plan.num_ctas <= 0) return cudaErrorInvalidValue;
+  softmax_order_kernel<<<1, kOrderThreads, 0, stream>>>(p);
+  note_launches(1);
+  err = cudaGetLastError();
+  if (err != cudaSuccess) return err;
+  softmax_tc_kernel<D><<<(unsigned)plan.num_ctas, kThreadsTC, smem, stream>>>(maps, p);
   note_launches(1);
   return cudaGetLastError();
 }
