@@ -28,12 +28,13 @@
 //
 // Warp roles (224 threads):
 //   warp 0     K producer, warp 6 V producer: one TMA box per page and
-//              64-column chunk (128-byte swizzle) into their own rings.
-//   warp 1     tensor-memory owner and MMA issuer: S_j = Q K_j^T, then
-//              O += P_j V_j; zeroes V rows past the prefix end so poisoned
-//              cache rows never meet a zero probability (0 * NaN).  MMAs from
-//              this one thread execute in issue order, which is what lets an
-//              S buffer be reused once the P.V that reads it was issued.
+//              64-column chunk (128-byte swizzle) into their own rings; the V
+//              producer zeroes the V rows past the prefix end so poisoned
+//              cache rows never meet a zero probability (0 * NaN).
+//   warp 1     tensor-memory owner and MMA issuer (one thread): S_j = Q K_j^T,
+//              then O += P_j V_j.  MMAs from this one thread execute in issue
+//              order, which is what lets an S buffer be reused once the P.V
+//              that reads it was issued.
 //   warps 2-5  softmax, one per TMEM lane quarter: load the Q rows into tensor
 //              memory, then per tile each thread takes one query row and the
 //              tile's 64 key columns; online base-2 softmax with a lazily
@@ -41,7 +42,7 @@
 //              more than 2^8); epilogue divides by the row sum and stores the
 //              output (or a split partial).
 // Every wait is bounded (tc::mbar_wait); a timeout sets FLARE_DEV_WAIT_TIMEOUT,
-// the CTA stops issuing work, writes nothing, frees its TMEM and exits.
+// the CTA stops issuing work, writes nothing more, frees its TMEM and exits.
 #include <cudaTypedefs.h>
 
 #include "common.cuh"
