@@ -132,7 +132,7 @@ def profiled_traffic(kernel, workload):
 
 
 class ClockSampler:
-    """nvidia-smi samples every 200 ms while the timed region runs."""
+    """nvidia-smi samples every 50 ms while the timed region runs."""
 
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -148,7 +148,7 @@ class ClockSampler:
         os.close(fd)
         self.out = open(self.path, "w")
         self.proc = subprocess.Popen(
-            [exe, f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200",
+            [exe, f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "50",
              "-i", str(device_index)], stdout=self.out, stderr=subprocess.DEVNULL)
 
     def stop(self):
@@ -280,35 +280,55 @@ class E2ERunner:
     """The same step through the C ABI with the step's inputs in pinned host
     memory: host->device copies of every per-step input and device->host
     copies of every output happen inside the timed region.  The paged KV pool
-    and the recurrent-state pool are the serving caches and stay resident."""
+    and the recurrent-state pool are the serving caches and stay resident.
+
+    The copies run on their own streams, as a serving loop would issue them:
+    every input goes host->device in the order the step consumes it (the
+    request metadata, then each denoise step's linear and softmax inputs, then
+    the commit's), each denoise step waits only for its own inputs, and its
+    outputs go device->host as soon as they are written."""
 
     def __init__(self, fr: FlareRunner):
         self.fr = fr
         w = fr.w
-        self.h2d = []  # (pinned host, device) pairs
-        self.d2h = []
-        for b in w.denoise:
-            for t in (b.q, b.k, b.v, b.log_decay, b.beta):
-                self.h2d.append((t.cpu().pin_memory(), t))
-        for t in (w.commit.k, w.commit.v, w.commit.log_decay, w.commit.beta):
-            self.h2d.append((t.cpu().pin_memory(), t))
-        for b in w.softmax:
-            for t in (b.q, b.k_blk, b.v_blk):
-                self.h2d.append((t.cpu().pin_memory(), t))
-        for t in (w.page_table, w.prefix_len, w.accept_len, w.state_slot):
-            self.h2d.append((t.cpu().pin_memory(), t))
-        for t in fr.lin_out + fr.sm_out:
-            self.d2h.append((t, torch.empty(t.shape, dtype=t.dtype, pin_memory=True)))
-        self.h2d_bytes = sum(h.numel() * h.element_size() for h, _ in self.h2d)
-        self.d2h_bytes = sum(h.numel() * h.element_size() for _, h in self.d2h)
+        pin = lambda t: (t.cpu().pin_memory(), t)  # noqa: E731
+        self.groups = [[pin(t) for t in (w.page_table, w.prefix_len, w.accept_len, w.state_slot)]]
+        for b, sb in zip(w.denoise, w.softmax):
+            self.groups.append([pin(t) for t in (b.q, b.k, b.v, b.log_decay, b.beta,
+                                                 sb.q, sb.k_blk, sb.v_blk)])
+        self.groups.append([pin(t) for t in (w.commit.k, w.commit.v, w.commit.log_decay,
+                                             w.commit.beta)])
+        self.outs = [[(lo, torch.empty(lo.shape, dtype=lo.dtype, pin_memory=True)),
+                      (so, torch.empty(so.shape, dtype=so.dtype, pin_memory=True))]
+                     for lo, so in zip(fr.lin_out, fr.sm_out)]
+        self.h2d_bytes = sum(h.numel() * h.element_size() for g in self.groups for h, _ in g)
+        self.d2h_bytes = sum(h.numel() * h.element_size() for g in self.outs for _, h in g)
+        self.s_h2d = torch.cuda.Stream()
+        self.s_d2h = torch.cuda.Stream()
+        self.ev_in = [torch.cuda.Event() for _ in self.groups]
+        self.ev_out = [torch.cuda.Event() for _ in self.outs]
 
     def step(self):
-        for h, d in self.h2d:
-            d.copy_(h, non_blocking=True)
-        self.fr.step()
-        for d, h in self.d2h:
-            h.copy_(d, non_blocking=True)
-        torch.cuda.current_stream().synchronize()
+        fr, cs = self.fr, torch.cuda.current_stream()
+        with torch.cuda.stream(self.s_h2d):
+            for g, ev in zip(self.groups, self.ev_in):
+                for h, d in g:
+                    d.copy_(h, non_blocking=True)
+                ev.record(self.s_h2d)
+        cs.wait_event(self.ev_in[0])
+        for i in range(fr.spec.denoise_steps):
+            cs.wait_event(self.ev_in[i + 1])
+            fr.linear(i)
+            fr.softmax(i)
+            self.ev_out[i].record(cs)
+            with torch.cuda.stream(self.s_d2h):
+                self.s_d2h.wait_event(self.ev_out[i])
+                for d, h in self.outs[i]:
+                    h.copy_(d, non_blocking=True)
+        cs.wait_event(self.ev_in[-1])
+        fr.commit()
+        self.s_d2h.synchronize()
+        cs.synchronize()
 
 
 def max_over_ranks(x, distributed, device):
@@ -514,7 +534,7 @@ def run_reference(args, spec):
 def main():
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=40)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(workloads.WORKLOADS))
     ap.add_argument("--impl", default="flare", choices=["flare", "reference"])
