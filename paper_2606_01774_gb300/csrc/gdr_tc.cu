@@ -251,30 +251,35 @@ __global__ void __launch_bounds__(kLinThreads, 2)
   if (!lin_wait(&sh.bar_mma, 0, sh, p.dev_status)) goto done;
   tc::fence_after_sync();
 
-  // ---- A^T (from rows 0..63 of G, fp32) and M2 (rows 64..127, bf16 operand)
+  // ---- A^T (from rows 0..63 of G, fp32) and M2 (rows 64..127, bf16 operand);
+  // all of a row's G values are loaded from tensor memory before any is used
   {
     const int row = tid & 63;
     const float gB = sh.gam2[B - 1];
     const float bt = sh.beta[row], gt = sh.gam2[row];
-#pragma unroll 1
-    for (int c0 = 0; c0 < Bp; c0 += 16) {
-      uint32_t gr[16];
-      tc::tmem_ld16(tmA + lane_off + c0, gr);
-      tc::tmem_ld_wait();
-      float v[16];
+    uint32_t gr[kBmax];
+#pragma unroll
+    for (int c0 = 0; c0 < kBmax; c0 += 16)
+      if (c0 < Bp) tc::tmem_ld16(tmA + lane_off + c0, *reinterpret_cast<uint32_t(*)[16]>(&gr[c0]));
+    tc::tmem_ld_wait();
+#pragma unroll
+    for (int c0 = 0; c0 < kBmax; c0 += 16) {
+      if (c0 >= Bp) break;
       if (tid < 64) {
 #pragma unroll
         for (int e = 0; e < 16; ++e) {
           const int i = c0 + e;
           // A[t][i] = beta_t exp(gamma_t - gamma_i) (k_t . k_i), i < t < B
-          AT[i * kATs + row] =
-              (i < row && row < B) ? bt * tc::ex2(gt - sh.gam2[i]) * __uint_as_float(gr[e]) : 0.f;
+          AT[i * kATs + row] = (i < row && row < B)
+                                   ? bt * tc::ex2(gt - sh.gam2[i]) * __uint_as_float(gr[i])
+                                   : 0.f;
         }
       } else {
+        float v[16];
 #pragma unroll
         for (int e = 0; e < 16; ++e) {
           const int i = c0 + e;
-          v[e] = (i < B && row < B) ? tc::ex2(gB - sh.gam2[i]) * __uint_as_float(gr[e]) : 0.f;
+          v[e] = (i < B && row < B) ? tc::ex2(gB - sh.gam2[i]) * __uint_as_float(gr[i]) : 0.f;
         }
         store16_sw128(M2s, row, c0, v);
       }
@@ -385,26 +390,35 @@ __global__ void __launch_bounds__(kLinThreads, 2)
   }
   if (!lin_wait(&sh.bar_mma, 1, sh, p.dev_status)) goto done;
   tc::fence_after_sync();
+  // out[l][c] = s (Gam_B W^T[c][64+l] + O2^T[c][l]), staged as bf16 [l][c] in the
+  // dead [K;Q] region, then written in 16-byte pieces
   {
     const int c = tid;
     const float GB = sh.Gam[B - 1];
-    __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.out_blockend) +
-                         ((size_t)r * B * p.Hv + j) * DV + c;
-#pragma unroll 1
-    for (int c0 = 0; c0 < Bp; c0 += 16) {
-      uint32_t o2[16], wq[16];
-      tc::tmem_ld16(tmA + lane_off + c0, o2);
-      tc::tmem_ld16(tmW + lane_off + 64 + c0, wq);  // (Q S0)^T[c][l]
-      tc::tmem_ld_wait();
-      if (c < DV) {
+    __nv_bfloat16* stage = reinterpret_cast<__nv_bfloat16*>(KQs);
+    uint32_t o2[kBmax], wq[kBmax];
 #pragma unroll
-        for (int e = 0; e < 16; ++e) {
-          const int l = c0 + e;
-          if (l < B)
-            out[(size_t)l * p.Hv * DV] = __float2bfloat16_rn(
-                p.scale * (GB * __uint_as_float(wq[e]) + __uint_as_float(o2[e])));
-        }
+    for (int c0 = 0; c0 < kBmax; c0 += 16) {
+      if (c0 < Bp) {
+        tc::tmem_ld16(tmA + lane_off + c0, *reinterpret_cast<uint32_t(*)[16]>(&o2[c0]));
+        tc::tmem_ld16(tmW + lane_off + 64 + c0, *reinterpret_cast<uint32_t(*)[16]>(&wq[c0]));
       }
+    }
+    tc::tmem_ld_wait();
+    if (c < DV) {
+#pragma unroll
+      for (int l = 0; l < kBmax; ++l)
+        if (l < B)
+          stage[l * DV + c] = __float2bfloat16_rn(
+              p.scale * (GB * __uint_as_float(wq[l]) + __uint_as_float(o2[l])));
+    }
+    __syncthreads();
+    constexpr int kPieces = DV / 8;  // 16-byte pieces per output row
+    __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.out_blockend);
+    for (int e = tid; e < B * kPieces; e += kLinThreads) {
+      const int l = e / kPieces, pc = e % kPieces;
+      *reinterpret_cast<uint4*>(out + (((size_t)r * B + l) * p.Hv + j) * DV + pc * 8) =
+          *reinterpret_cast<const uint4*>(stage + l * DV + pc * 8);
     }
   }
 
