@@ -89,7 +89,7 @@ struct TcShared {
   uint64_t q_ready;   // a work item's Q rows are in tensor memory (one phase per item)
   uint64_t o_final;   // a work item's last P.V has completed
   uint64_t o_free;    // a work item's O has been read out (the next item may overwrite it)
-  uint64_t v_fix;     // a partial prefix tile's V rows past the prefix end are zeroed
+  uint64_t v_fix[8];  // per V slot: a partial prefix tile's V rows past the prefix end are zeroed
   uint32_t tmem_base;
   int abort_flag;
   int last_split;     // this CTA merges the split partials of its row tile
@@ -430,7 +430,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     tc::mbar_init(&sh.q_ready, kSoftmaxThreads);
     tc::mbar_init(&sh.o_final, 1);
     tc::mbar_init(&sh.o_free, kSoftmaxThreads);
-    tc::mbar_init(&sh.v_fix, 1);
+    for (int s = 0; s < C::kVStages; ++s) tc::mbar_init(&sh.v_fix[s], 1);
     tc::fence_mbar_init();
   }
   if (warp == 1) tc::tmem_alloc(&sh.tmem_base, C::kTmemCols);
@@ -504,7 +504,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 *reinterpret_cast<uint4*>(dst + c * (kTileN * 128) + (valid + e / 8) * 128 +
                                           (e % 8) * 16) = make_uint4(0u, 0u, 0u, 0u);
             tc::fence_async_smem();
-            tc::mbar_arrive(&sh.v_fix);
+            tc::mbar_arrive(&sh.v_fix[st]);
           }
         }
       }
@@ -520,8 +520,8 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
       const uint64_t kdesc0 = tc::sdesc_sw128(tc::smem_u32(Ks), 16, 1024);
       const uint64_t vdesc0 = tc::sdesc_sw128(tc::smem_u32(Vs), kTileN * 128, 1024);
       bool ok = true;
-      int g = 0;     // running tile count
-      int nfix = 0;  // partial tiles seen
+      int g = 0;              // running tile count
+      uint32_t fix_par = 0u;  // per V slot: parity of its next zeroed-partial-tile phase
       for (int k = 0; ok && !aborted(sh); ++k) {
         const int idx = item_of(k);
         if (idx < 0) break;
@@ -540,10 +540,12 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
           if (j == 0 && k > 0 &&
               !tc::mbar_wait(&sh.o_free, (uint32_t)(k - 1) & 1u, &sh.abort_flag))
             return false;
+          // a slot's partial tiles are in order: the next one can only be
+          // loaded once the P.V issued after this wait has freed the slot
           bool ready;
           if (j == w.j_part) {
-            ready = tc::mbar_wait(&sh.v_fix, (uint32_t)nfix & 1u, &sh.abort_flag);
-            ++nfix;
+            ready = tc::mbar_wait(&sh.v_fix[st], (fix_par >> st) & 1u, &sh.abort_flag);
+            fix_par ^= 1u << st;
           } else {
             ready = tc::mbar_wait(&sh.v_full[st], (uint32_t)(gg / C::kVStages) & 1u,
                                   &sh.abort_flag);

@@ -24,6 +24,12 @@ CASES = {
                                                            prefix_hi=70, block_len=7, seed=41),
     "page16_d128": W["small_model_batch256"].replace(num_requests=3, page_size=16,
                                                      prefix_lo=1, prefix_hi=300, seed=42),
+    # more work items than SMs, each a few tiles long and ending inside a page:
+    # every CTA walks several items back to back, each with a zeroed partial tile
+    "many_short_items_d128": W["small_model_batch256"].replace(num_requests=100, prefix_lo=1,
+                                                               prefix_hi=200, seed=43),
+    "many_short_items_d256": W["serving_batch64"].replace(num_requests=80, prefix_lo=1,
+                                                          prefix_hi=300, seed=44),
 }
 
 
