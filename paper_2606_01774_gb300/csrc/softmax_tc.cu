@@ -26,11 +26,11 @@
 // and out once (MMA operand read), and the rings take all of shared memory,
 // since a tile load takes about a microsecond from issue to arrival.
 //
-// Warp roles (224 threads):
+// Warp roles (256 threads):
 //   warp 0     K producer, warp 6 V producer: one TMA box per page and
-//              64-column chunk (128-byte swizzle) into their own rings; the V
-//              producer zeroes the V rows past the prefix end so poisoned
-//              cache rows never meet a zero probability (0 * NaN).
+//              64-column chunk (128-byte swizzle) into their own rings.
+//   warp 7     zeroes the V rows past the prefix end once that tile has landed,
+//              so poisoned cache rows never meet a zero probability (0 * NaN).
 //   warp 1     tensor-memory owner and MMA issuer (one thread): S_j = Q K_j^T,
 //              then O += P_j V_j.  MMAs from this one thread execute in issue
 //              order, which is what lets an S buffer be reused once the P.V
@@ -57,7 +57,8 @@ constexpr int kTileN = 64;     // keys per tile
 constexpr int kRowsM = 128;    // query rows per work item (TMEM lanes)
 constexpr int kSoftmaxThreads = 128;  // warps 2-5, one per TMEM lane quarter
 constexpr int kVWarp = 6;             // V producer
-constexpr int kThreadsTC = 224;       // K producer, MMA issuer, 4 softmax warps, V producer
+constexpr int kFixWarp = 7;           // zeroes the V rows past a prefix end
+constexpr int kThreadsTC = 256;       // K producer, MMA issuer, 4 softmax warps, V producer, fixer
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 
 struct TcMaps {
@@ -93,6 +94,7 @@ struct TcShared {
   uint32_t tmem_base;
   int abort_flag;
   int last_split;     // this CTA merges the split partials of its row tile
+  int v_issued;       // V tiles whose loads the V producer has issued (running count)
 };
 
 // All lanes of the warp wait; the outcome is made warp-uniform so that the
@@ -414,6 +416,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
   if (tid == 0) {
     sh.abort_flag = 0;
     sh.last_split = 0;
+    sh.v_issued = 0;
     for (int s = 0; s < C::kKStages; ++s) {
       tc::mbar_init(&sh.k_full[s], 1);
       tc::mbar_init(&sh.k_empty[s], 1);
@@ -476,6 +479,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
             tc::mbar_expect_tx(full, C::kKVBytes);
             for (int c = 0; c < C::kChunks; ++c)
               tc::tma_load_4d(dst + c * (kTileN * 128), blk_map, full, c * 64, w.kvh, 0, w.r);
+            if (kv) *reinterpret_cast<volatile int*>(&sh.v_issued) = g + 1;
             continue;
           }
           const int tok0 = (w.j0 + j) * kTileN;
@@ -490,26 +494,62 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
               tc::tma_load_4d(dst + c * (kTileN * 128) + bx * box_rows * 128, pool_map, full,
                               c * 64, row0, w.kvh, page);
           }
-          if (kv && j == w.j_part) {
-            // rows past the prefix end hold stale (possibly poisoned) cache
-            // rows; zero them once the load has landed so that a zero
-            // probability never meets a NaN (0 * NaN) in P.V
-            if (!tc::mbar_wait(full, ph, &sh.abort_flag)) {
-              ok = false;
-              break;
-            }
-            const int nrow = kTileN - valid;
-            for (int c = 0; c < C::kChunks; ++c)
-              for (int e = 0; e < nrow * 8; ++e)
-                *reinterpret_cast<uint4*>(dst + c * (kTileN * 128) + (valid + e / 8) * 128 +
-                                          (e % 8) * 16) = make_uint4(0u, 0u, 0u, 0u);
-            tc::fence_async_smem();
-            tc::mbar_arrive(&sh.v_fix[st]);
-          }
+          if (kv) *reinterpret_cast<volatile int*>(&sh.v_issued) = g + 1;
         }
       }
       if (!ok) set_abort(sh, p.dev_status);
     }
+  } else if (warp == kFixWarp) {
+    // ------------------------------------------------------------ V fixer
+    // The last prefix tile of an item ends inside the tile: its V rows past the
+    // prefix end hold stale (possibly poisoned) cache rows.  Once its load has
+    // landed they are zeroed, so that a zero probability never meets a NaN
+    // (0 * NaN) in P.V; the MMA issuer waits for this instead of the load.
+    // A warp of its own, so the V producer never stops to wait for a load.
+    bool ok = true;
+    int g = 0;  // running tile count
+    for (int k = 0; ok && !aborted(sh); ++k) {
+      const int idx = item_of(k);
+      if (idx < 0) break;
+      const TcWork w = tc_work(p, n_mt, idx);
+      if (w.j_part >= 0) {
+        const int gg = g + w.j_part;
+        const int st = gg % C::kVStages;
+        // Parity waits are exact only once the tile's load has been issued:
+        // then the slot's previous load has been consumed, and its next one
+        // needs the P.V that waits for this warp.  Until then, sleep-poll the
+        // producer's count (bounded like every wait).
+        bool issued = true;
+        if (lane == 0) {
+          const uint64_t t0 = tc::globaltimer_ns();
+          while (*reinterpret_cast<volatile int*>(&sh.v_issued) <= gg) {
+            if (aborted(sh) || tc::globaltimer_ns() - t0 > 2000000000ull) {
+              issued = false;
+              break;
+            }
+            __nanosleep(64);
+          }
+        }
+        issued = __shfl_sync(0xffffffffu, issued, 0);
+        if (!issued ||
+            !warp_wait(&sh.v_full[st], (uint32_t)(gg / C::kVStages) & 1u, &sh.abort_flag)) {
+          ok = false;
+          break;
+        }
+        uint8_t* dst = Vs + st * C::kKVBytes;
+        const int valid = w.P - (w.j0 + w.j_part) * kTileN;  // 1 .. kTileN - 1
+        const int n16 = (kTileN - valid) * 8;                 // 16-byte pieces per chunk
+        for (int c = 0; c < C::kChunks; ++c)
+          for (int e = lane; e < n16; e += 32)
+            *reinterpret_cast<uint4*>(dst + c * (kTileN * 128) + (valid + e / 8) * 128 +
+                                      (e % 8) * 16) = make_uint4(0u, 0u, 0u, 0u);
+        tc::fence_async_smem();
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(&sh.v_fix[st]);
+      }
+      g += w.n_tiles;
+    }
+    if (!ok && lane == 0) set_abort(sh, p.dev_status);
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     // One thread waits and issues; operand descriptors advance by adding the
