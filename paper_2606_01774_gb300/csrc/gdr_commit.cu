@@ -75,7 +75,8 @@ __global__ void __launch_bounds__(2 * DV, 2) gdr_commit_kernel(GdrParams p) {
   constexpr int kThreads = 2 * DV;   // DV / 16 warps
   constexpr int kR = DK / 8;         // state rows per thread
   extern __shared__ float smc[];
-  __shared__ float alpha_s[kCBmax], beta_s[kCBmax];
+  // per token: {Gam_t, beta_t, 1/Gam_t (0: fold the decay into the state), Gam after the step}
+  __shared__ float4 tok_s[kCBmax];
 
   const int item = blockIdx.x;
   const int r = item / p.Hv, j = item % p.Hv;
@@ -115,10 +116,49 @@ __global__ void __launch_bounds__(2 * DV, 2) gdr_commit_kernel(GdrParams p) {
     stage_rows<T, DK, kThreads>(Qs, qg, (size_t)p.Hk * DK, steps);
   }
   stage_rows<T, DV, kThreads>(Vs, vg, (size_t)p.Hv * DV, steps);
-  for (int t = threadIdx.x; t < steps; t += kThreads) {
-    const size_t gb = ((size_t)r * B + t) * p.Hv + j;
-    alpha_s[t] = expf(p.log_decay[gb]);
-    beta_s[t] = p.beta[gb];
+  // the decay schedule, once per CTA (warp 0): Gam_t = exp(gamma_t) with
+  // gamma_t = g_1 + ... + g_t while Gam_t stays >= 2^-40 (the common case, one
+  // prefix scan); otherwise thread 0 walks the tokens and folds where needed
+  if (warp == 0) {
+    const size_t gb = (size_t)r * B * p.Hv + j;
+    float g0 = lane < steps ? p.log_decay[gb + (size_t)lane * p.Hv] : 0.f;
+    float g1 = lane + 32 < steps ? p.log_decay[gb + (size_t)(lane + 32) * p.Hv] : 0.f;
+    const float b0 = lane < steps ? p.beta[gb + (size_t)lane * p.Hv] : 0.f;
+    const float b1 = lane + 32 < steps ? p.beta[gb + (size_t)(lane + 32) * p.Hv] : 0.f;
+    const float a0 = expf(g0), a1 = expf(g1);
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float x = __shfl_up_sync(0xffffffffu, g0, o);
+      const float y = __shfl_up_sync(0xffffffffu, g1, o);
+      if (lane >= o) {
+        g0 += x;
+        g1 += y;
+      }
+    }
+    g1 += __shfl_sync(0xffffffffu, g0, 31);
+    constexpr float kMinLog = -27.725887222397812f;  // ln 2^-40
+    const bool fold = __any_sync(0xffffffffu, (lane < steps && g0 < kMinLog) ||
+                                                  (lane + 32 < steps && g1 < kMinLog));
+    if (!fold) {
+      const float e0 = expf(g0), e1 = expf(g1);
+      tok_s[lane] = make_float4(e0, b0, expf(-g0), e0);
+      tok_s[lane + 32] = make_float4(e1, b1, expf(-g1), e1);
+    } else {
+      // alpha and beta through shared memory, then the exact running product
+      tok_s[lane] = make_float4(a0, b0, 0.f, 0.f);
+      tok_s[lane + 32] = make_float4(a1, b1, 0.f, 0.f);
+      __syncwarp();
+      if (lane == 0) {
+        float gam = 1.f;
+        for (int t = 0; t < steps; ++t) {
+          const float4 e = tok_s[t];
+          const float gt = gam * e.x;
+          const bool f = gt < kMinGam;
+          gam = f ? 1.f : gt;
+          tok_s[t] = make_float4(gt, e.y, f ? 0.f : 1.f / gt, gam);
+        }
+      }
+    }
   }
   __syncthreads();
 
@@ -153,16 +193,16 @@ __global__ void __launch_bounds__(2 * DV, 2) gdr_commit_kernel(GdrParams p) {
       d.z += __shfl_xor_sync(0xffffffffu, d.z, o);
       d.w += __shfl_xor_sync(0xffffffffu, d.w, o);
     }
-    const float gt = gam * alpha_s[t];
-    const float bt = beta_s[t];
+    const float4 tp = tok_s[t];
+    const float gt = tp.x, bt = tp.y;
     const float4 v = *reinterpret_cast<const float4*>(Vs + t * DV + c0);
     float4 delta;
     delta.x = bt * (v.x - gt * d.x);
     delta.y = bt * (v.y - gt * d.y);
     delta.z = bt * (v.z - gt * d.z);
     delta.w = bt * (v.w - gt * d.w);
-    if (gt >= kMinGam) {  // uniform across the CTA: the gates are per head
-      const float ig = 1.f / gt;
+    if (tp.z != 0.f) {  // uniform across the CTA: the gates are per head
+      const float ig = tp.z;
       const float4 w = make_float4(delta.x * ig, delta.y * ig, delta.z * ig, delta.w * ig);
 #pragma unroll
       for (int m = 0; m < kR; ++m) {
@@ -171,7 +211,6 @@ __global__ void __launch_bounds__(2 * DV, 2) gdr_commit_kernel(GdrParams p) {
         s[m].z = fmaf(k[m], w.z, s[m].z);
         s[m].w = fmaf(k[m], w.w, s[m].w);
       }
-      gam = gt;
     } else {  // fold the decay into the state
 #pragma unroll
       for (int m = 0; m < kR; ++m) {
@@ -180,8 +219,8 @@ __global__ void __launch_bounds__(2 * DV, 2) gdr_commit_kernel(GdrParams p) {
         s[m].z = fmaf(k[m], delta.z, gt * s[m].z);
         s[m].w = fmaf(k[m], delta.w, gt * s[m].w);
       }
-      gam = 1.f;
     }
+    gam = tp.w;
     if (t + 1 == n) {
 #pragma unroll
       for (int m = 0; m < kR; ++m)

@@ -92,3 +92,22 @@ def test_commit_full_size_sampled():
     got = w.state_pool[w.state_slot.long()[sample]]
     assert_states_close(got, ref["state"], "multistep_batch128")
     assert torch.isfinite(w.state_pool[w.state_slot.long()]).all()
+
+
+@pytest.mark.parametrize("causal", [False, True])
+def test_commit_strong_decay_folds_the_schedule(causal):
+    """Log-gates of -3 per token drive the running decay below 2^-40 inside the
+    block (the kernel then folds the decay into the state); half the heads keep
+    the ordinary gates.  Same oracle, same tolerances."""
+    spec = W["serving_batch64"].replace(num_requests=3, prefix_lo=0, prefix_hi=70,
+                                        accept="uniform", seed=33)
+    w = gen(spec)
+    w.commit.log_decay[:, :, ::2] = -3.0
+    install_states(w)
+    before = w.state_pool.clone()
+    co = run_commit(w, w.state_pool, causal=causal)
+    ref = oracle_commit(w, before, causal=causal)
+    slots = w.state_slot.long()
+    assert_states_close(w.state_pool[slots], ref["state"], "strong decay")
+    if causal:
+        assert_out_close(co, ref["causal"], spec.act_dtype, "strong decay causal")
