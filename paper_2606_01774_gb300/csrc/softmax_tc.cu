@@ -298,15 +298,33 @@ __global__ void __launch_bounds__(kOrderThreads) softmax_order_kernel(SoftmaxPar
       flag(p.dev_status, FLARE_DEV_BAD_PREFIX_LEN);
     }
   }
+  // page ids in use: eight table entries per thread in flight at a time
   const long long n_entries = (long long)p.R * p.max_pages;
-  for (long long i = t; i < n_entries; i += kOrderThreads) {
-    const int r = (int)(i / p.max_pages), pg = (int)(i % p.max_pages);
-    const int P = p.prefix_len[r];
-    if (P < 0 || P > prefix_cap || (long long)pg * p.page_size >= P) continue;  // page unused
-    const int id = p.page_table[i];
-    if (id < 0 || id >= p.num_pages) {
-      atomicOr(&p.bad_mask[r >> 5], 1u << (r & 31));
-      flag(p.dev_status, FLARE_DEV_BAD_PAGE);
+  constexpr int kIn = 8;
+  for (long long i0 = t; i0 < n_entries; i0 += (long long)kIn * kOrderThreads) {
+    int id[kIn], rr[kIn];
+    bool used[kIn];
+#pragma unroll
+    for (int u = 0; u < kIn; ++u) {
+      const long long i = i0 + (long long)u * kOrderThreads;
+      used[u] = false;
+      rr[u] = 0;
+      id[u] = 0;
+      if (i < n_entries) {
+        const int r = (int)(i / p.max_pages);
+        const int pg = (int)(i - (long long)r * p.max_pages);
+        const int P = p.prefix_len[r];
+        used[u] = P >= 0 && P <= prefix_cap && (long long)pg * p.page_size < P;
+        rr[u] = r;
+        id[u] = p.page_table[i];
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kIn; ++u) {
+      if (used[u] && (id[u] < 0 || id[u] >= p.num_pages)) {
+        atomicOr(&p.bad_mask[rr[u] >> 5], 1u << (rr[u] & 31));
+        flag(p.dev_status, FLARE_DEV_BAD_PAGE);
+      }
     }
   }
   __syncthreads();
