@@ -13,6 +13,11 @@ of the paper it follows, is documented in the C file:
   block-end readout (Eq. noisy-block-fwd), commit at the accepted length.
 * :func:`gdr_chunked` -- the same quantities through the chunkwise WY/UT form
   (Eq. chunk-state, Eq. f-blk); used only to pin :func:`gdr_per_token`.
+* :func:`gdr_verify` -- the AR-Trust verify round: token-causal anchor/verify
+  rows, bidirectional draft rows, and the states cached at each verify
+  position (serving appendix, cache-and-scatter).
+* :func:`verify_commit` -- the gather-scatter of the cached state at each
+  request's accepted offset into every layer's state pool.
 * :func:`gather_prefix` -- dense copy of a request's paged prefix.
 * :func:`block_softmax` -- softmax retrieval (Eq. softmax-retrieval) under the
   Diffusion-Trust block mask over the paged prefix plus the block.
@@ -66,7 +71,10 @@ def _load():
         lib.oracle_gdr_chunked.restype = I
         lib.oracle_gather_prefix.argtypes = [I] * 7 + [P, P, P, P]
         lib.oracle_gather_prefix.restype = I
-        lib.oracle_block_softmax.argtypes = [I] * 8 + [D, I, I, P, P, P, P, P, P, P, P, P, I]
+        lib.oracle_gdr_verify.argtypes = [I] * 6 + [D, I, I, P, P, P, I, P, P, I, P, I, P, P,
+                                                    P, P, P, I]
+        lib.oracle_gdr_verify.restype = I
+        lib.oracle_block_softmax.argtypes = [I] * 8 + [D, I, I, P, P, P, P, P, P, P, P, P, P, I]
         lib.oracle_block_softmax.restype = I
         lib.oracle_append_kv.argtypes = [I] * 8 + [P] * 7
         lib.oracle_append_kv.restype = I
@@ -181,6 +189,57 @@ def gdr_chunked(q, k, v, log_decay, beta, state_pool, state_slot, accept_len=Non
     return {"blockend": ob, "state": st}
 
 
+def gdr_verify(q, k, v, log_decay, beta, state_pool, state_slot, verify_len, max_verify, *,
+               scale=None, nthreads=0):
+    """AR-Trust verify round of one gated-delta-rule layer.
+
+    Shapes: q, k [R,L,Hk,dk]; v [R,L,Hv,dv]; log_decay, beta [R,L,Hv];
+    state_pool [slots,Hv,dk,dv]; state_slot, verify_len [R] (K_r, the number
+    of held drafts being verified, 0..min(max_verify, L-1)).
+    Returns fp64 ``out`` [R,L,Hv,dv] (rows t <= K_r: s S_{t+1}^T q_t; later
+    rows: s S_L^T q_t), ``records`` [R,max_verify,Hv,dk,dv] (record t < K_r is
+    S_{t+1}, the state after the anchor and t drafts; the rest stay zero) and
+    ``state`` [R,Hv,dk,dv] (S_{K_r+1}, the live state after every verify
+    token)."""
+    a = _gdr_args(q, k, v, log_decay, beta, state_pool, state_slot, None)
+    R, L, Hv, dk, dv = a["R"], a["B"], a["Hv"], a["dk"], a["dv"]
+    s = 1.0 / np.sqrt(dk) if scale is None else float(scale)
+    vl = _i32(verify_len)
+    out = np.zeros((R, L, Hv, dv))
+    rec = np.zeros((R, max_verify, Hv, dk, dv))
+    st = np.zeros((R, Hv, dk, dv))
+    rc = _load().oracle_gdr_verify(
+        R, L, a["Hk"], Hv, dk, dv, s, int(max_verify), a["dt"], _ptr(a["qa"]), _ptr(a["ka"]),
+        _ptr(a["va"]), a["gdt"], _ptr(a["ga"]), _ptr(a["ba"]), a["sdt"], _ptr(a["sa"]),
+        a["nslots"], _ptr(a["slot"]), _ptr(vl), _ptr(out), _ptr(rec), _ptr(st), int(nthreads))
+    if rc != 0:
+        raise ValueError("oracle_gdr_verify: invalid state slot or verify length")
+    return {"out": out, "records": rec, "state": st}
+
+
+def verify_commit(records, pools, state_slot, accept, verify_len):
+    """Gather-scatter commit of a verify round (serving appendix, path (b)).
+
+    records: per layer [R, max_verify, Hv, dk, dv]; pools: per layer
+    [slots, Hv, dk, dv]; accept[r] in [0, verify_len[r]] is the number of
+    accepted drafts.  Returns copies of the pools where, for every layer and
+    every request with accept[r] < verify_len[r], slot state_slot[r] holds
+    records[r][accept[r]] bit for bit; a request that accepted every draft
+    already has S^(K) in the pool and is left alone.  Raises ValueError on an
+    out-of-range slot, accepted offset or verify length."""
+    slot, acc, vl = _i32(state_slot), _i32(accept), _i32(verify_len)
+    outs = [np.array(p, copy=True) for p in pools]
+    for rec, pool in zip(records, outs):
+        R, max_verify = rec.shape[0], rec.shape[1]
+        for r in range(R):
+            if not (0 <= slot[r] < pool.shape[0] and 0 <= vl[r] <= max_verify
+                    and 0 <= acc[r] <= vl[r]):
+                raise ValueError("verify_commit: invalid slot, accepted offset or verify length")
+            if acc[r] < vl[r]:
+                pool[slot[r]] = rec[r, acc[r]]
+    return outs
+
+
 def gather_prefix(r, pool, page_table, prefix_len, page_size):
     """Dense fp64 copy [P_r, Hkv, D] of request r's paged prefix from one pool."""
     pa, pdt = _arr(pool)
@@ -197,11 +256,13 @@ def gather_prefix(r, pool, page_table, prefix_len, page_size):
 
 
 def block_softmax(q, k_blk, v_blk, k_pool, v_pool, page_table, prefix_len, *, scale=None,
-                  mask_mode=0, nthreads=0):
+                  mask_mode=0, row_type=None, nthreads=0):
     """Block-query softmax attention over paged prefix + block (Eq. softmax-retrieval).
 
     mask_mode 0: every block row sees every block token (denoise pass);
-    mask_mode 1: block row t sees block tokens 0..t (state-update pass).
+    mask_mode 1: block row t sees block tokens 0..t (state-update pass);
+    mask_mode 2 / 3: per-row types, ``row_type`` uint8 [B] (shared) or [R,B]
+    (per request); type 0 rows are token-causal, type 1 rows bidirectional.
     Returns (out [R,B,Hq,D], lse [R,B,Hq]) in fp64."""
     qa, dt = _arr(q)
     kb, _ = _arr(k_blk)
@@ -216,11 +277,19 @@ def block_softmax(q, k_blk, v_blk, k_pool, v_pool, page_table, prefix_len, *, sc
     sc = 1.0 / np.sqrt(D) if scale is None else float(scale)
     out = np.zeros((R, B, Hq, D))
     lse = np.zeros((R, B, Hq))
+    rt = None
+    if mask_mode in (2, 3):
+        if hasattr(row_type, "detach"):
+            row_type = row_type.detach().cpu().numpy()
+        rt = np.ascontiguousarray(np.asarray(row_type, dtype=np.uint8))
+        if rt.shape != ((B,) if mask_mode == 2 else (R, B)):
+            raise ValueError("row_type shape does not match the mask mode")
     rc = _load().oracle_block_softmax(
         R, B, Hq, Hkv, D, p, num_pages, tab.shape[1], sc, int(mask_mode), dt, _ptr(qa), _ptr(kb),
-        _ptr(vb), _ptr(kp), _ptr(vp), _ptr(tab), _ptr(lens), _ptr(out), _ptr(lse), int(nthreads))
+        _ptr(vb), _ptr(kp), _ptr(vp), _ptr(tab), _ptr(lens), _ptr(rt), _ptr(out), _ptr(lse),
+        int(nthreads))
     if rc != 0:
-        raise ValueError("oracle_block_softmax: invalid page id or prefix length")
+        raise ValueError("oracle_block_softmax: invalid page id, prefix length or row type")
     return out, lse
 
 

@@ -22,6 +22,11 @@
  *   commit at accepted length r (serving appendix, "Recovering the recurrent
  *   state at the accept boundary"): the pool slot becomes S^(r) = S_r, and
  *   r = 0 leaves it unchanged.
+ *   AR-Trust verify round (decoding appendix, block layout; serving appendix,
+ *   cache-and-scatter): anchor and verify rows read S_{t+1} token-causally,
+ *   draft rows read S_L, the states after the anchor and each verify token
+ *   are cached, and the commit copies the cached state at the accepted
+ *   offset into the pool.
  *   chunkwise form (Eq. chunk-state / Eq. f-blk with WY-corrected values):
  *   an independent second implementation used only to pin the first.
  *   softmax retrieval over a visible set (Eq. softmax-retrieval) with the
@@ -164,6 +169,97 @@ int oracle_gdr_per_token(int R, int B, int Hk, int Hv, int dk, int dv, double s,
 }
 
 /*
+ * AR-Trust verify round, gated-delta-rule part (decoding appendix, "AR-Trust
+ * sampling": the block is [anchor, d_0 .. d_{K-1}, MASK ...]; serving
+ * appendix, "Recovering the recurrent state at the accept boundary", path (b),
+ * cache-and-scatter).  For request r with K = verify_len[r] the block's rows
+ * 0..K (anchor and verify rows) are token-causal and rows K+1..L-1 (padding and
+ * draft rows) read the whole block.  From S0 = state_pool[state_slot[r]][j]
+ * the gated delta rule (Eq. per-step-fwd) runs over all L block tokens; with
+ * S_n the state after tokens 0..n-1:
+ *   out[r][t][j]        = s S_{t+1}^T q_t   for t <= K   (token-causal rows)
+ *   out[r][t][j]        = s S_L^T q_t       for t >  K   (bidirectional rows)
+ *   records[r][t][j]    = S_{t+1}           for t <  K   (S^(t): the anchor and
+ *                                                          t accepted drafts)
+ *   state_out[r][j]     = S_{K+1}                        (S^(K): every draft accepted)
+ * Shapes: q, k [R,L,Hk,dk]; v [R,L,Hv,dv]; log_decay, beta [R,L,Hv];
+ * state_pool [num_slots,Hv,dk,dv]; state_slot, verify_len [R];
+ * out [R,L,Hv,dv]; records [R,max_verify,Hv,dk,dv] (entries t >= K untouched);
+ * state_out [R,Hv,dk,dv].  Returns -1 for an invalid slot or verify length
+ * (verify_len[r] outside [0, min(max_verify, L-1)]).
+ */
+int oracle_gdr_verify(int R, int L, int Hk, int Hv, int dk, int dv, double s, int max_verify,
+                      int act_dt, const void* q, const void* k, const void* v,
+                      int gate_dt, const void* log_decay, const void* beta,
+                      int state_dt, const void* state_pool, int num_slots,
+                      const int32_t* state_slot, const int32_t* verify_len,
+                      double* out, double* records, double* state_out, int nthreads) {
+  for (int r = 0; r < R; ++r) {
+    if (state_slot[r] < 0 || state_slot[r] >= num_slots) return -1;
+    if (verify_len[r] < 0 || verify_len[r] > max_verify || verify_len[r] > L - 1) return -1;
+  }
+  set_threads(nthreads);
+  const size_t nst = (size_t)dk * dv;
+#pragma omp parallel for schedule(dynamic, 1)
+  for (long item = 0; item < (long)R * Hv; ++item) {
+    const int r = (int)(item / Hv), j = (int)(item % Hv);
+    const int h = (int)(((long)j * Hk) / Hv);
+    const int K = verify_len[r];
+    double* S = (double*)malloc(sizeof(double) * nst);
+    double* u = (double*)malloc(sizeof(double) * dv);
+    double* kt = (double*)malloc(sizeof(double) * dk);
+    double* qt = (double*)malloc(sizeof(double) * dk);
+    const size_t s0 = ((size_t)state_slot[r] * Hv + j) * nst;
+    for (size_t e = 0; e < nst; ++e) S[e] = ld(state_pool, state_dt, s0 + e);
+    for (int t = 0; t < L; ++t) {
+      const size_t kq = (((size_t)r * L + t) * Hk + h) * dk;
+      const size_t vo = (((size_t)r * L + t) * Hv + j) * dv;
+      const size_t gb = ((size_t)r * L + t) * Hv + j;
+      const double alpha = exp(ld(log_decay, gate_dt, gb));
+      const double bt = ld(beta, gate_dt, gb);
+      for (int i = 0; i < dk; ++i) kt[i] = ld(k, act_dt, kq + i);
+      /* S_pre = exp(g_t) S;  u_t = v_t - S_pre^T k_t;  S = S_pre + k_t (beta_t u_t)^T */
+      for (size_t e = 0; e < nst; ++e) S[e] *= alpha;
+      for (int c = 0; c < dv; ++c) u[c] = 0.0;
+      for (int i = 0; i < dk; ++i)
+        for (int c = 0; c < dv; ++c) u[c] += S[i * dv + c] * kt[i];
+      for (int c = 0; c < dv; ++c) u[c] = bt * (ld(v, act_dt, vo + c) - u[c]);
+      for (int i = 0; i < dk; ++i)
+        for (int c = 0; c < dv; ++c) S[i * dv + c] += kt[i] * u[c];
+      /* anchor and verify rows read the state right after their own token */
+      if (t <= K) {
+        for (int i = 0; i < dk; ++i) qt[i] = ld(q, act_dt, kq + i);
+        for (int c = 0; c < dv; ++c) {
+          double acc = 0.0;
+          for (int i = 0; i < dk; ++i) acc += S[i * dv + c] * qt[i];
+          out[vo + c] = s * acc;
+        }
+      }
+      /* cache S^(t) for the verify positions, the live state after the last one */
+      if (t < K)
+        memcpy(records + (((size_t)r * max_verify + t) * Hv + j) * nst, S, sizeof(double) * nst);
+      if (t == K) memcpy(state_out + (size_t)item * nst, S, sizeof(double) * nst);
+    }
+    /* padding and draft rows read the block-end state S_L */
+    for (int t = K + 1; t < L; ++t) {
+      const size_t ql = (((size_t)r * L + t) * Hk + h) * dk;
+      const size_t ol = (((size_t)r * L + t) * Hv + j) * dv;
+      for (int i = 0; i < dk; ++i) qt[i] = ld(q, act_dt, ql + i);
+      for (int c = 0; c < dv; ++c) {
+        double acc = 0.0;
+        for (int i = 0; i < dk; ++i) acc += S[i * dv + c] * qt[i];
+        out[ol + c] = s * acc;
+      }
+    }
+    free(qt);
+    free(kt);
+    free(u);
+    free(S);
+  }
+  return 0;
+}
+
+/*
  * The same quantities computed a second, independent way: the chunkwise
  * (WY / UT) form of the appendix, "Chunkwise-parallel form",
  * "Chunk-corrected values" and Eq. chunk-state, applied to one block.
@@ -292,20 +388,34 @@ int oracle_gather_prefix(int r, int Hkv, int D, int page_size, int num_pages, in
  * h / (Hq / Hkv)) and block row t the visible set is every prefix token
  * j < prefix_len[r] (read through the page table) plus the block tokens i
  * with i < B (mask_mode 0, bidirectional denoise pass) or i <= t
- * (mask_mode 1, token-causal state-update pass).  Two passes in fp64:
+ * (mask_mode 1, token-causal state-update pass).  Mask modes 2 and 3 are the
+ * compact per-row encoding of the serving appendix's dLLM mask modes (AR-Trust
+ * block: anchor and verify rows token-causal, draft rows bidirectional over
+ * the block): row t is token-causal when row_type[t] == 0 and bidirectional
+ * when it is 1, with row_type [B] shared by every request (mode 2) or
+ * [R, B] per request (mode 3).  Every row sees the whole prefix in every mode
+ * (the prefix-tile visibility invariant).  Two passes in fp64:
  *   z_i = scale (q . k_i),  m = max_i z_i,  w_i = exp(z_i - m),
  *   o = sum_i w_i v_i / sum_i w_i,  lse = m + log(sum_i w_i).
  * Shapes: q [R,B,Hq,D]; k_blk, v_blk [R,B,Hkv,D]; pools
  * [num_pages,Hkv,page_size,D]; page_table [R,max_pages]; prefix_len [R];
- * out [R,B,Hq,D]; lse [R,B,Hq] (may be NULL).
+ * out [R,B,Hq,D]; lse [R,B,Hq] (may be NULL); row_type (modes 2 and 3 only)
+ * uint8 [B] or [R,B], each entry 0 or 1.
  */
 int oracle_block_softmax(int R, int B, int Hq, int Hkv, int D, int page_size, int num_pages,
                          int max_pages, double scale, int mask_mode, int act_dt,
                          const void* q, const void* k_blk, const void* v_blk,
                          const void* k_pool, const void* v_pool,
                          const int32_t* page_table, const int32_t* prefix_len,
-                         double* out, double* lse, int nthreads) {
+                         const uint8_t* row_type, double* out, double* lse, int nthreads) {
   if (Hkv <= 0 || Hq % Hkv != 0) return -1;
+  if (mask_mode < 0 || mask_mode > 3) return -1;
+  if (mask_mode >= 2) {
+    if (!row_type) return -1;
+    const long n_types = mask_mode == 2 ? B : (long)R * B;
+    for (long i = 0; i < n_types; ++i)
+      if (row_type[i] > 1) return -1;
+  }
   for (int r = 0; r < R; ++r) {
     const int P = prefix_len[r];
     if (P < 0 || P > max_pages * page_size) return -1;
@@ -323,7 +433,10 @@ int oracle_block_softmax(int R, int B, int Hq, int Hkv, int D, int page_size, in
     const int t = (int)(item % B);
     const int kvh = h / G;
     const int P = prefix_len[r];
-    const int nblk = (mask_mode == 0) ? B : t + 1;
+    int causal_row = mask_mode == 1;
+    if (mask_mode == 2) causal_row = row_type[t] == 0;
+    if (mask_mode == 3) causal_row = row_type[(size_t)r * B + t] == 0;
+    const int nblk = causal_row ? t + 1 : B;
     const int n = P + nblk;
     double* z = (double*)malloc(sizeof(double) * (n > 0 ? n : 1));
     double* qv = (double*)malloc(sizeof(double) * D);
