@@ -13,6 +13,14 @@
  *   flare_block_linear_attn   gated-delta-rule block pass, block-end readout
  *   flare_commit_state        write S^(r) into the state pool
  *   flare_block_softmax_attn  block queries over paged prefix + block
+ *   flare_append_kv           append the finalized block to the paged cache
+ *
+ * and the attention work of an AR-Trust verify round (decoding appendix):
+ *
+ *   flare_verify_linear_attn  token-causal anchor/verify rows, bidirectional
+ *                             draft rows, verify states cached
+ *   flare_verify_commit       restore the state at the accepted offset
+ *   flare_block_softmax_attn  with the per-row ROW_TYPE mask modes
  *
  * Conventions shared by every call
  * --------------------------------
@@ -56,11 +64,24 @@ typedef enum flare_dtype { FLARE_DT_BF16 = 0, FLARE_DT_F32 = 1 } flare_dtype;
 
 /* Softmax block mask (decoding appendix, attention patterns): every block row
  * sees the whole prefix; in the denoise pass (BIDIR) it also sees every block
- * token, in the state-update pass (CAUSAL) the block tokens up to itself. */
+ * token, in the state-update pass (CAUSAL) the block tokens up to itself.
+ * The two ROW_TYPE modes are the compact (B, row_type_1..B) encoding of the
+ * serving appendix's native dLLM mask modes, used by the AR-Trust verify
+ * round (anchor and verify rows token-causal, draft rows bidirectional over
+ * the block): desc->row_type gives one type per block row, shared by the
+ * batch (UNIFORM, [B]) or per request (PER_REQUEST, [R, B]).  Prefix tiles are
+ * unmasked for every row type. */
 typedef enum flare_mask_mode {
   FLARE_MASK_BLOCK_BIDIR = 0,
-  FLARE_MASK_BLOCK_CAUSAL = 1
+  FLARE_MASK_BLOCK_CAUSAL = 1,
+  FLARE_MASK_ROW_TYPE_UNIFORM = 2,
+  FLARE_MASK_ROW_TYPE_PER_REQUEST = 3
 } flare_mask_mode;
+
+/* Row types (uint8) of the ROW_TYPE mask modes.  A value other than these two
+ * reads as FLARE_ROW_BIDIR. */
+#define FLARE_ROW_CAUSAL 0 /* anchor / verify row: block tokens 0..t */
+#define FLARE_ROW_BIDIR 1  /* draft / MASK row: every block token */
 
 /* Device status bits (OR-ed into *dev_status). */
 #define FLARE_DEV_BAD_SLOT 0x1       /* state_slot[r] outside [0, num_state_slots) */
@@ -68,6 +89,8 @@ typedef enum flare_mask_mode {
 #define FLARE_DEV_BAD_PREFIX_LEN 0x4 /* prefix_len[r] < 0 or > max_pages_per_req * page_size */
 #define FLARE_DEV_BAD_ACCEPT_LEN 0x8 /* accept_len[r] outside [0, block_len] */
 #define FLARE_DEV_WAIT_TIMEOUT 0x10  /* an in-kernel pipeline wait gave up (bounded spin) */
+#define FLARE_DEV_BAD_VERIFY_LEN 0x20 /* verify_len[r] outside [0, min(max_verify, block_len-1)],
+                                         or an accepted offset outside [0, verify_len[r]] */
 
 /* Gated-delta-rule layer shape.
  *   num_requests R, block_len B (1..64), num_qk_heads Hk, num_v_heads Hv
@@ -93,7 +116,9 @@ typedef struct flare_linear_desc {
  *   (64, 128 or 256), page_size p (16 or 64 tokens), num_pages in each pool,
  *   max_pages_per_req (columns of the page table), act_dtype of every
  *   activation and pool, scale of the logits (the paper's 1/sqrt(D)),
- *   mask_mode as above. */
+ *   mask_mode as above; row_type is a DEVICE pointer to uint8 row types
+ *   ([B] or [R, B]) for the ROW_TYPE modes and is ignored (may be NULL) in
+ *   the others. */
 typedef struct flare_softmax_desc {
   int32_t num_requests;
   int32_t block_len;
@@ -106,6 +131,7 @@ typedef struct flare_softmax_desc {
   flare_dtype act_dtype;
   float scale;
   flare_mask_mode mask_mode;
+  const uint8_t* row_type;
 } flare_softmax_desc;
 
 /*
@@ -156,6 +182,70 @@ flare_status flare_commit_state(const flare_linear_desc* desc, const void* q, co
                                 int32_t* dev_status, void* stream);
 
 /*
+ * AR-Trust verify round of a gated-delta-rule layer (decoding appendix,
+ * "AR-Trust sampling", block layout; serving appendix, "Recovering the
+ * recurrent state at the accept boundary", path (b) cache-and-scatter).
+ * The block of L = desc->block_len tokens is [anchor, d_0 .. d_{K-1},
+ * MASK ...] with K = verify_len[r] held drafts (0 on a cold start).  For each
+ * request r and value head j the gated delta rule (Eq. per-step-fwd) runs
+ * from S0 = state_pool[state_slot[r]][j] over all L tokens; with S_n the state
+ * after block tokens 0..n-1:
+ *     out[r][t][j]   = scale * S_{t+1}^T q[r][t][h]   t <= K (anchor, verify rows:
+ *                                                     token-causal)
+ *     out[r][t][j]   = scale * S_L^T q[r][t][h]       t >  K (draft rows: the
+ *                                                     whole block)
+ *     verify_states[r][t][j] = S_{t+1}                t <  K (S^(t): the anchor
+ *                                                     and t accepted drafts)
+ *     state_pool[state_slot[r]][j] <- S_{K+1}         (S^(K), written in place)
+ * so the live pool holds the state after every verify token, and
+ * flare_verify_commit restores S^(a) when only a < K drafts are accepted.
+ * Entries t >= K of verify_states are not written.
+ * Precondition: the state_slot entries are distinct within one call.
+ *   q, k           [R, L, Hk, dk]           act_dtype
+ *   v              [R, L, Hv, dv]           act_dtype
+ *   log_decay,beta [R, L, Hv]               fp32
+ *   state_pool     [num_state_slots, Hv, dk, dv] fp32, read and written
+ *   state_slot     [R]                      int32
+ *   verify_len     [R]                      int32 in [0, min(max_verify, L - 1)]
+ *   out            [R, L, Hv, dv]           act_dtype
+ *   verify_states  [R, max_verify, Hv, dk, dv] fp32 (may be NULL if max_verify = 0)
+ *   dev_status     FLARE_DEV_BAD_SLOT | FLARE_DEV_BAD_VERIFY_LEN (the request is
+ *                  skipped: nothing of it is written)
+ */
+flare_status flare_verify_linear_attn(const flare_linear_desc* desc, int32_t max_verify,
+                                      const void* q, const void* k, const void* v,
+                                      const float* log_decay, const float* beta,
+                                      float* state_pool, const int32_t* state_slot,
+                                      const int32_t* verify_len, void* out, float* verify_states,
+                                      int32_t* dev_status, void* stream);
+
+/*
+ * Gather-scatter commit of an AR-Trust verify round across layers (serving
+ * appendix, path (b)): once the verify decision is known, for every layer l
+ * and request r with accepted offset a = accept[r] (drafts accepted, in
+ * [0, verify_len[r]]):
+ *     a <  verify_len[r]:  state_pools[l][state_slot[r]] <- verify_states[l][r][a]
+ *     a == verify_len[r]:  nothing (the pool already holds S^(K))
+ * A bit-for-bit copy, one launch for all layers.
+ *   desc           only num_requests, num_v_heads, head_dim_k, head_dim_v and
+ *                  num_state_slots are used
+ *   num_layers     1 .. 64
+ *   verify_states  HOST array of num_layers DEVICE pointers, each
+ *                  [R, max_verify, Hv, dk, dv] fp32 as written by
+ *                  flare_verify_linear_attn
+ *   state_pools    HOST array of num_layers DEVICE pointers, each
+ *                  [num_state_slots, Hv, dk, dv] fp32
+ *   state_slot, accept, verify_len  [R] int32 (device)
+ *   dev_status     FLARE_DEV_BAD_SLOT | FLARE_DEV_BAD_VERIFY_LEN (the request is
+ *                  skipped)
+ */
+flare_status flare_verify_commit(const flare_linear_desc* desc, int32_t max_verify,
+                                 int32_t num_layers, const float* const* verify_states,
+                                 float* const* state_pools, const int32_t* state_slot,
+                                 const int32_t* accept, const int32_t* verify_len,
+                                 int32_t* dev_status, void* stream);
+
+/*
  * Bytes of device workspace flare_block_softmax_attn needs for `desc`
  * (the longest-first order of the work units and the partial outputs of split
  * prefixes).  May be 0.  Host-only, no GPU work.
@@ -168,7 +258,8 @@ flare_status flare_softmax_workspace_size(const flare_softmax_desc* desc, size_t
  * appendix).  For request r, query head h (kv head h / (Hq / Hkv)) and block
  * row t the visible keys are the prefix tokens j < prefix_len[r], read from
  * page page_table[r][j / p], row j % p of the pools, followed by the block's
- * own keys (all B of them in BIDIR mode, 0..t in CAUSAL mode):
+ * own keys (all B of them in BIDIR mode and for FLARE_ROW_BIDIR rows, 0..t in
+ * CAUSAL mode and for FLARE_ROW_CAUSAL rows):
  *     out[r][t][h] = sum_i softmax_i(scale * q . k_i) v_i
  *     lse[r][t][h] = log sum_i exp(scale * q . k_i)          (natural log)
  * The block's keys/values are not in the pools (they are appended only by the

@@ -36,7 +36,12 @@ flare_status check_softmax(const flare_softmax_desc* d) {
       d->page_size < 1 || d->num_pages < 0 || d->max_pages_per_req < 0 ||
       !valid_dtype(d->act_dtype))
     return FLARE_ERR_INVALID_ARGUMENT;
-  if (d->mask_mode != FLARE_MASK_BLOCK_BIDIR && d->mask_mode != FLARE_MASK_BLOCK_CAUSAL)
+  if (d->mask_mode != FLARE_MASK_BLOCK_BIDIR && d->mask_mode != FLARE_MASK_BLOCK_CAUSAL &&
+      d->mask_mode != FLARE_MASK_ROW_TYPE_UNIFORM &&
+      d->mask_mode != FLARE_MASK_ROW_TYPE_PER_REQUEST)
+    return FLARE_ERR_INVALID_ARGUMENT;
+  if ((d->mask_mode == FLARE_MASK_ROW_TYPE_UNIFORM ||
+       d->mask_mode == FLARE_MASK_ROW_TYPE_PER_REQUEST) && !d->row_type)
     return FLARE_ERR_INVALID_ARGUMENT;
   if (!(d->scale >= 0.f) || !(d->scale < 3.0e38f)) return FLARE_ERR_INVALID_ARGUMENT;
   if (d->num_q_heads % d->num_kv_heads != 0) return FLARE_ERR_INVALID_ARGUMENT;
@@ -69,6 +74,10 @@ SoftmaxParams softmax_params(const flare_softmax_desc* d) {
   p.max_pages = d->max_pages_per_req;
   p.scale_log2 = d->scale * 1.4426950408889634f;
   p.causal = d->mask_mode == FLARE_MASK_BLOCK_CAUSAL;
+  if (d->mask_mode == FLARE_MASK_ROW_TYPE_UNIFORM || d->mask_mode == FLARE_MASK_ROW_TYPE_PER_REQUEST) {
+    p.row_type = d->row_type;
+    p.row_type_stride = d->mask_mode == FLARE_MASK_ROW_TYPE_PER_REQUEST ? d->block_len : 0;
+  }
   return p;
 }
 
@@ -246,6 +255,85 @@ flare_status flare_commit_state(const flare_linear_desc* d, const void* q, const
   p.dev_status = dev_status;
   const cudaError_t e = launch_gdr_commit(p, d->act_dtype == FLARE_DT_BF16,
                                           static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? FLARE_OK : FLARE_ERR_CUDA;
+}
+
+flare_status flare_verify_linear_attn(const flare_linear_desc* d, int32_t max_verify,
+                                      const void* q, const void* k, const void* v,
+                                      const float* log_decay, const float* beta,
+                                      float* state_pool, const int32_t* state_slot,
+                                      const int32_t* verify_len, void* out, float* verify_states,
+                                      int32_t* dev_status, void* stream) {
+  flare_status st = check_linear(d);
+  if (st != FLARE_OK) return st;
+  if (max_verify < 0) return FLARE_ERR_INVALID_ARGUMENT;
+  if (!q || !k || !v || !log_decay || !beta || !state_pool || !state_slot || !verify_len ||
+      !out || !dev_status || (max_verify > 0 && !verify_states))
+    return FLARE_ERR_INVALID_ARGUMENT;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(state_pool) ||
+      !aligned16(out) || !aligned16(verify_states))
+    return FLARE_ERR_INVALID_ARGUMENT;
+  if (d->num_requests == 0) return FLARE_OK;
+  GdrParams p;
+  memset(&p, 0, sizeof p);
+  p.R = d->num_requests;
+  p.B = d->block_len;
+  p.Hk = d->num_qk_heads;
+  p.Hv = d->num_v_heads;
+  p.dk = d->head_dim_k;
+  p.dv = d->head_dim_v;
+  p.nslots = d->num_state_slots;
+  p.scale = d->scale;
+  p.q = q;
+  p.k = k;
+  p.v = v;
+  p.log_decay = log_decay;
+  p.beta = beta;
+  p.state_pool = state_pool;
+  p.state_slot = state_slot;
+  p.out_causal = out;
+  p.write_state = 1;
+  p.verify_len = verify_len;
+  p.max_verify = max_verify;
+  p.verify_states = verify_states;
+  p.dev_status = dev_status;
+  const cudaError_t e = launch_gdr_verify(p, d->act_dtype == FLARE_DT_BF16,
+                                          static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? FLARE_OK : FLARE_ERR_CUDA;
+}
+
+flare_status flare_verify_commit(const flare_linear_desc* d, int32_t max_verify,
+                                 int32_t num_layers, const float* const* verify_states,
+                                 float* const* state_pools, const int32_t* state_slot,
+                                 const int32_t* accept, const int32_t* verify_len,
+                                 int32_t* dev_status, void* stream) {
+  flare_status st = check_linear(d);
+  if (st != FLARE_OK) return st;
+  if (max_verify < 0 || num_layers < 1) return FLARE_ERR_INVALID_ARGUMENT;
+  if (num_layers > kMaxVerifyLayers) return FLARE_ERR_UNSUPPORTED;
+  if (!verify_states || !state_pools || !state_slot || !accept || !verify_len || !dev_status)
+    return FLARE_ERR_INVALID_ARGUMENT;
+  VerifyCommitParams p;
+  memset(&p, 0, sizeof p);
+  for (int l = 0; l < num_layers; ++l) {
+    if (!state_pools[l] || (max_verify > 0 && !verify_states[l]))
+      return FLARE_ERR_INVALID_ARGUMENT;
+    if (!aligned16(state_pools[l]) || !aligned16(verify_states[l]))
+      return FLARE_ERR_INVALID_ARGUMENT;
+    p.records[l] = verify_states[l];
+    p.pools[l] = state_pools[l];
+  }
+  if (d->num_requests == 0 || max_verify == 0) return FLARE_OK;
+  p.R = d->num_requests;
+  p.max_verify = max_verify;
+  p.nslots = d->num_state_slots;
+  p.n_layers = num_layers;
+  p.state_elems = (size_t)d->num_v_heads * d->head_dim_k * d->head_dim_v;
+  p.state_slot = state_slot;
+  p.accept = accept;
+  p.verify_len = verify_len;
+  p.dev_status = dev_status;
+  const cudaError_t e = launch_verify_commit(p, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? FLARE_OK : FLARE_ERR_CUDA;
 }
 

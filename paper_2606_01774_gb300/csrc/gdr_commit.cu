@@ -22,6 +22,14 @@
 // first n = accept_len tokens Gam_n S~ is written back in place; n = 0 leaves
 // the slot untouched.  Exact fp32 arithmetic throughout, which is what the
 // committed state's accuracy needs.
+//
+// The same kernel runs the AR-Trust verify round (decoding appendix, block
+// layout [anchor, d_0 .. d_{K-1}, MASK ...]; serving appendix, cache-and-
+// scatter): all L block tokens are stepped, rows 0..K read the state right
+// after their own token, the states after the anchor and after each of the
+// first K-1 verify tokens are streamed out as S^(0..K-1), the state after
+// token K is written to the pool, and the draft rows read the block-end state
+// once the loop is done.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -70,8 +78,11 @@ __device__ __forceinline__ void stage_rows(float* dst, const T* src, size_t stri
 
 }  // namespace
 
-template <typename T, int DK, int DV, bool CAUSAL>
+// MODE 0: commit; 1: commit with token-causal outputs; 2: AR-Trust verify round.
+template <typename T, int DK, int DV, int MODE>
 __global__ void __launch_bounds__(2 * DV, 2) gdr_commit_kernel(GdrParams p) {
+  constexpr bool CAUSAL = MODE != 0;  // queries staged, readouts written
+  constexpr bool VERIFY = MODE == 2;
   constexpr int kThreads = 2 * DV;   // DV / 16 warps
   constexpr int kR = DK / 8;         // state rows per thread
   extern __shared__ float smc[];
@@ -91,10 +102,20 @@ __global__ void __launch_bounds__(2 * DV, 2) gdr_commit_kernel(GdrParams p) {
     if (threadIdx.x == 0) flag(p.dev_status, FLARE_DEV_BAD_SLOT);
     return;
   }
-  const int n = p.accept_len[r];
-  if (n < 0 || n > B) {
-    if (threadIdx.x == 0) flag(p.dev_status, FLARE_DEV_BAD_ACCEPT_LEN);
-    return;
+  int n, K = 0;
+  if constexpr (VERIFY) {
+    K = p.verify_len[r];
+    if (K < 0 || K > p.max_verify || K > B - 1) {
+      if (threadIdx.x == 0) flag(p.dev_status, FLARE_DEV_BAD_VERIFY_LEN);
+      return;
+    }
+    n = K + 1;  // the live state: after the anchor and every verify token
+  } else {
+    n = p.accept_len[r];
+    if (n < 0 || n > B) {
+      if (threadIdx.x == 0) flag(p.dev_status, FLARE_DEV_BAD_ACCEPT_LEN);
+      return;
+    }
   }
   const int steps = CAUSAL ? B : n;
   if (steps == 0) return;
@@ -162,6 +183,41 @@ __global__ void __launch_bounds__(2 * DV, 2) gdr_commit_kernel(GdrParams p) {
   }
   __syncthreads();
 
+  // out[t] = scale * S^T q_t with S = g * S~ (this thread's 4 columns, the 8
+  // row groups of a warp meeting through shuffles)
+  auto readout = [&](int t, float g) {
+    const float4* q4 = reinterpret_cast<const float4*>(Qs + t * DK + rg * kR);
+    float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int m4 = 0; m4 < kR / 4; ++m4) {
+      const float4 qq = q4[m4];
+      const float qv[4] = {qq.x, qq.y, qq.z, qq.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int m = 4 * m4 + e;
+        o.x = fmaf(s[m].x, qv[e], o.x);
+        o.y = fmaf(s[m].y, qv[e], o.y);
+        o.z = fmaf(s[m].z, qv[e], o.z);
+        o.w = fmaf(s[m].w, qv[e], o.w);
+      }
+    }
+#pragma unroll
+    for (int sh = 4; sh < 32; sh <<= 1) {
+      o.x += __shfl_xor_sync(0xffffffffu, o.x, sh);
+      o.y += __shfl_xor_sync(0xffffffffu, o.y, sh);
+      o.z += __shfl_xor_sync(0xffffffffu, o.z, sh);
+      o.w += __shfl_xor_sync(0xffffffffu, o.w, sh);
+    }
+    if (rg == 0) {
+      T* out = static_cast<T*>(p.out_causal) + (((size_t)r * B + t) * p.Hv + j) * DV + c0;
+      const float sc = p.scale * g;
+      out[0] = from_f32<T>(sc * o.x);
+      out[1] = from_f32<T>(sc * o.y);
+      out[2] = from_f32<T>(sc * o.z);
+      out[3] = from_f32<T>(sc * o.w);
+    }
+  };
+
   float gam = 1.f;  // S = gam * S~
 #pragma unroll 1
   for (int t = 0; t < steps; ++t) {
@@ -221,69 +277,54 @@ __global__ void __launch_bounds__(2 * DV, 2) gdr_commit_kernel(GdrParams p) {
       }
     }
     gam = tp.w;
+    if constexpr (VERIFY) {
+      if (t < K) {  // S^(t), streamed past L2: at most one of them is read back
+        float* rec = p.verify_states +
+                     (((size_t)r * p.max_verify + t) * p.Hv + j) * DK * DV +
+                     (size_t)rg * kR * DV + c0;
+#pragma unroll
+        for (int m = 0; m < kR; ++m)
+          __stcs(reinterpret_cast<float4*>(rec + (size_t)m * DV),
+                 make_float4(gam * s[m].x, gam * s[m].y, gam * s[m].z, gam * s[m].w));
+      }
+    }
     if (t + 1 == n) {
 #pragma unroll
       for (int m = 0; m < kR; ++m)
         *reinterpret_cast<float4*>(Sg + (size_t)m * DV) =
             make_float4(gam * s[m].x, gam * s[m].y, gam * s[m].z, gam * s[m].w);
     }
-    if (CAUSAL) {
-      const float4* q4 = reinterpret_cast<const float4*>(Qs + t * DK + rg * kR);
-      float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-      for (int m4 = 0; m4 < kR / 4; ++m4) {
-        const float4 qq = q4[m4];
-        const float qv[4] = {qq.x, qq.y, qq.z, qq.w};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int m = 4 * m4 + e;
-          o.x = fmaf(s[m].x, qv[e], o.x);
-          o.y = fmaf(s[m].y, qv[e], o.y);
-          o.z = fmaf(s[m].z, qv[e], o.z);
-          o.w = fmaf(s[m].w, qv[e], o.w);
-        }
-      }
-#pragma unroll
-      for (int sh = 4; sh < 32; sh <<= 1) {
-        o.x += __shfl_xor_sync(0xffffffffu, o.x, sh);
-        o.y += __shfl_xor_sync(0xffffffffu, o.y, sh);
-        o.z += __shfl_xor_sync(0xffffffffu, o.z, sh);
-        o.w += __shfl_xor_sync(0xffffffffu, o.w, sh);
-      }
-      if (rg == 0) {
-        T* out = static_cast<T*>(p.out_causal) + (((size_t)r * B + t) * p.Hv + j) * DV + c0;
-        const float sc = p.scale * gam;
-        out[0] = from_f32<T>(sc * o.x);
-        out[1] = from_f32<T>(sc * o.y);
-        out[2] = from_f32<T>(sc * o.z);
-        out[3] = from_f32<T>(sc * o.w);
-      }
-    }
+    if (CAUSAL && (!VERIFY || t <= K)) readout(t, gam);
+  }
+  if constexpr (VERIFY) {
+    // padding and draft rows read the block-end state
+#pragma unroll 1
+    for (int t = K + 1; t < B; ++t) readout(t, gam);
   }
 }
 
 namespace {
 
-template <typename T, int DK, int DV, bool CAUSAL>
+template <typename T, int DK, int DV, int MODE>
 cudaError_t launch_commit_t(const GdrParams& p, cudaStream_t stream) {
   auto smem_for = [](int B) {
-    return sizeof(float) * ((size_t)B * DK * (CAUSAL ? 2 : 1) + (size_t)B * DV);
+    return sizeof(float) * ((size_t)B * DK * (MODE != 0 ? 2 : 1) + (size_t)B * DV);
   };
-  cudaError_t e = cudaFuncSetAttribute(gdr_commit_kernel<T, DK, DV, CAUSAL>,
+  cudaError_t e = cudaFuncSetAttribute(gdr_commit_kernel<T, DK, DV, MODE>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem_for(kCBmax));
   if (e != cudaSuccess) return e;
-  gdr_commit_kernel<T, DK, DV, CAUSAL><<<p.R * p.Hv, 2 * DV, smem_for(p.B), stream>>>(p);
+  gdr_commit_kernel<T, DK, DV, MODE><<<p.R * p.Hv, 2 * DV, smem_for(p.B), stream>>>(p);
   note_launches(1);
   return cudaGetLastError();
 }
 
-template <typename T, bool CAUSAL>
+template <typename T, int MODE>
 cudaError_t launch_commit_c(const GdrParams& p, cudaStream_t stream) {
-  if (p.dk == 128 && p.dv == 128) return launch_commit_t<T, 128, 128, CAUSAL>(p, stream);
-  if (p.dk == 128 && p.dv == 64) return launch_commit_t<T, 128, 64, CAUSAL>(p, stream);
-  if (p.dk == 64 && p.dv == 128) return launch_commit_t<T, 64, 128, CAUSAL>(p, stream);
-  if (p.dk == 64 && p.dv == 64) return launch_commit_t<T, 64, 64, CAUSAL>(p, stream);
+  if (p.dk == 128 && p.dv == 128) return launch_commit_t<T, 128, 128, MODE>(p, stream);
+  if (p.dk == 128 && p.dv == 64) return launch_commit_t<T, 128, 64, MODE>(p, stream);
+  if (p.dk == 64 && p.dv == 128) return launch_commit_t<T, 64, 128, MODE>(p, stream);
+  if (p.dk == 64 && p.dv == 64) return launch_commit_t<T, 64, 64, MODE>(p, stream);
   return cudaErrorInvalidValue;
 }
 
@@ -293,9 +334,14 @@ cudaError_t launch_gdr_commit(const GdrParams& p, bool bf16, cudaStream_t stream
   if (p.R == 0) return cudaSuccess;
   const bool causal = p.out_causal != nullptr;
   if (bf16)
-    return causal ? launch_commit_c<__nv_bfloat16, true>(p, stream)
-                  : launch_commit_c<__nv_bfloat16, false>(p, stream);
-  return causal ? launch_commit_c<float, true>(p, stream) : launch_commit_c<float, false>(p, stream);
+    return causal ? launch_commit_c<__nv_bfloat16, 1>(p, stream)
+                  : launch_commit_c<__nv_bfloat16, 0>(p, stream);
+  return causal ? launch_commit_c<float, 1>(p, stream) : launch_commit_c<float, 0>(p, stream);
+}
+
+cudaError_t launch_gdr_verify(const GdrParams& p, bool bf16, cudaStream_t stream) {
+  if (p.R == 0) return cudaSuccess;
+  return bf16 ? launch_commit_c<__nv_bfloat16, 2>(p, stream) : launch_commit_c<float, 2>(p, stream);
 }
 
 }  // namespace flare

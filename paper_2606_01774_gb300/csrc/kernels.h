@@ -26,6 +26,10 @@ struct GdrParams {
   void* out_blockend;         // [R,B,Hv,dv] or nullptr
   void* out_causal;           // [R,B,Hv,dv] or nullptr
   int write_state;
+  // AR-Trust verify round
+  const int32_t* verify_len;  // [R] or nullptr
+  int max_verify;
+  float* verify_states;       // [R,max_verify,Hv,dk,dv]
   int32_t* dev_status;
 };
 
@@ -33,6 +37,8 @@ struct SoftmaxParams {
   int R, B, Hq, Hkv, G, D, page_size, num_pages, max_pages;
   float scale_log2;  // logit scale * log2(e)
   int causal;
+  const uint8_t* row_type;  // per-row types (0 = token-causal) or nullptr
+  int row_type_stride;      // 0 (one layout for the batch) or B (per request)
   const void* q;      // [R,B,Hq,D]
   const void* k_blk;  // [R,B,Hkv,D]
   const void* v_blk;
@@ -67,6 +73,20 @@ struct SoftmaxPlan {
 size_t gdr_recurrent_smem_bytes(int dk, int dv, int threads);
 bool gdr_denoise_tc_supported(int B, int dk, int dv);
 cudaError_t launch_gdr_commit(const GdrParams& p, bool bf16, cudaStream_t stream);
+cudaError_t launch_gdr_verify(const GdrParams& p, bool bf16, cudaStream_t stream);
+
+constexpr int kMaxVerifyLayers = 64;
+struct VerifyCommitParams {
+  int R, max_verify, nslots, n_layers;
+  size_t state_elems;  // Hv * dk * dv
+  const float* records[kMaxVerifyLayers];
+  float* pools[kMaxVerifyLayers];
+  const int32_t* state_slot;
+  const int32_t* accept;
+  const int32_t* verify_len;
+  int32_t* dev_status;
+};
+cudaError_t launch_verify_commit(const VerifyCommitParams& p, cudaStream_t stream);
 cudaError_t launch_gdr_denoise_tc(const GdrParams& p, cudaStream_t stream);
 cudaError_t launch_gdr_recurrent(const GdrParams& p, bool bf16, cudaStream_t stream);
 

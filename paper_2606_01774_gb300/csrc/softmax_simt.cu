@@ -97,7 +97,9 @@ __global__ void __launch_bounds__(kThreads) softmax_simt_kernel(SoftmaxParams p)
       const int i = warp * 4 + w, m = mt * kRows + i;
       if (m >= M) continue;  // warp-uniform
       const int trow = m / p.G;
-      const bool vis = idx < kv_hi && (!p.causal || idx < P || idx - P <= trow);
+      const bool causal_row =
+          p.row_type ? p.row_type[(size_t)r * p.row_type_stride + trow] == 0 : p.causal != 0;
+      const bool vis = idx < kv_hi && (!causal_row || idx < P || idx - P <= trow);
       float s = -INFINITY;
       if (vis) {
         float a = 0.f;

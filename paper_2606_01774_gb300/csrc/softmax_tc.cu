@@ -708,6 +708,11 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     for (int k = 0; idx >= 0; ++k) {
       const int m = w.mtile * kRowsM + row;
       const int trow = m / p.G;
+      // token-causal block row: the state-update pass, or an anchor / verify
+      // row of the per-row encoding (padding rows past the block read none)
+      const bool causal_row =
+          p.row_type ? (trow < p.B && p.row_type[(size_t)w.r * p.row_type_stride + trow] == 0)
+                     : p.causal != 0;
       float m_run = -INFINITY, l_run = 0.f;
       for (int j = 0; j < w.n_tiles; ++j) {
         const int gg = g + j;
@@ -727,7 +732,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         const bool blk = j >= w.n_pref_here;
         const int valid = blk ? p.B : min(kTileN, w.P - (w.j0 + j) * kTileN);
         const bool full = !blk && valid == kTileN;  // prefix tile: no mask at all
-        const int lim = full ? kTileN : ((blk && p.causal) ? min(valid, trow + 1) : valid);
+        const int lim = full ? kTileN : ((blk && causal_row) ? min(valid, trow + 1) : valid);
         // tile maximum of the raw scores (scale >= 0 keeps the order)
         float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll

@@ -27,12 +27,17 @@ FLARE_DT_BF16 = 0
 FLARE_DT_F32 = 1
 FLARE_MASK_BLOCK_BIDIR = 0
 FLARE_MASK_BLOCK_CAUSAL = 1
+FLARE_MASK_ROW_TYPE_UNIFORM = 2
+FLARE_MASK_ROW_TYPE_PER_REQUEST = 3
+FLARE_ROW_CAUSAL = 0
+FLARE_ROW_BIDIR = 1
 
 FLARE_DEV_BAD_SLOT = 0x1
 FLARE_DEV_BAD_PAGE = 0x2
 FLARE_DEV_BAD_PREFIX_LEN = 0x4
 FLARE_DEV_BAD_ACCEPT_LEN = 0x8
 FLARE_DEV_WAIT_TIMEOUT = 0x10
+FLARE_DEV_BAD_VERIFY_LEN = 0x20
 
 
 class FlareError(RuntimeError):
@@ -56,7 +61,7 @@ class flare_softmax_desc(ctypes.Structure):
                 ("head_dim", ctypes.c_int32), ("page_size", ctypes.c_int32),
                 ("num_pages", ctypes.c_int32), ("max_pages_per_req", ctypes.c_int32),
                 ("act_dtype", ctypes.c_int), ("scale", ctypes.c_float),
-                ("mask_mode", ctypes.c_int)]
+                ("mask_mode", ctypes.c_int), ("row_type", ctypes.c_void_p)]
 
 
 _lib = None
@@ -76,6 +81,8 @@ def load() -> ctypes.CDLL:
     sigs = {
         "flare_block_linear_attn": [lin] + [P] * 10,
         "flare_commit_state": [lin] + [P] * 11,
+        "flare_verify_linear_attn": [lin, I32] + [P] * 12,
+        "flare_verify_commit": [lin, I32, I32] + [P] * 7,
         "flare_softmax_workspace_size": [smx, ctypes.POINTER(S)],
         "flare_block_softmax_attn": [smx] + [P] * 10 + [S, P, P],
         "flare_block_softmax_attn_noalloc": [smx] + [P] * 11,
@@ -142,6 +149,27 @@ def flare_commit_state(desc, q, k, v, log_decay, beta, state_pool, state_slot, a
         _p(state_slot), _p(accept_len), _p(causal_out), _p(dev_status), _stream(stream))
 
 
+def flare_verify_linear_attn(desc, max_verify, q, k, v, log_decay, beta, state_pool,
+                             state_slot, verify_len, out, verify_states, dev_status,
+                             stream=None) -> int:
+    return load().flare_verify_linear_attn(
+        ctypes.byref(desc), int(max_verify), _p(q), _p(k), _p(v), _p(log_decay), _p(beta),
+        _p(state_pool), _p(state_slot), _p(verify_len), _p(out), _p(verify_states),
+        _p(dev_status), _stream(stream))
+
+
+def flare_verify_commit(desc, max_verify, verify_states, state_pools, state_slot, accept,
+                        verify_len, dev_status, stream=None) -> int:
+    """verify_states, state_pools: sequences of per-layer device tensors; their
+    data pointers are passed as host arrays."""
+    n = len(state_pools)
+    recs = (ctypes.c_void_p * n)(*[None if t is None else t.data_ptr() for t in verify_states])
+    pools = (ctypes.c_void_p * n)(*[t.data_ptr() for t in state_pools])
+    return load().flare_verify_commit(
+        ctypes.byref(desc), int(max_verify), n, recs, pools, _p(state_slot), _p(accept),
+        _p(verify_len), _p(dev_status), _stream(stream))
+
+
 def flare_softmax_workspace_size(desc) -> int:
     n = ctypes.c_size_t(0)
     check(load().flare_softmax_workspace_size(ctypes.byref(desc), ctypes.byref(n)),
@@ -199,6 +227,9 @@ def linear_desc(num_requests, block_len, num_qk_heads, num_v_heads, head_dim_k, 
 
 def softmax_desc(num_requests, block_len, num_q_heads, num_kv_heads, head_dim, page_size,
                  num_pages, max_pages_per_req, act_dtype, scale,
-                 mask_mode=FLARE_MASK_BLOCK_BIDIR) -> flare_softmax_desc:
+                 mask_mode=FLARE_MASK_BLOCK_BIDIR, row_type=None) -> flare_softmax_desc:
+    """row_type: uint8 device tensor ([B] or [R,B]) for the ROW_TYPE mask modes;
+    the caller keeps it alive while the descriptor is in use."""
     return flare_softmax_desc(num_requests, block_len, num_q_heads, num_kv_heads, head_dim,
-                              page_size, num_pages, max_pages_per_req, act_dtype, scale, mask_mode)
+                              page_size, num_pages, max_pages_per_req, act_dtype, scale, mask_mode,
+                              None if row_type is None else row_type.data_ptr())

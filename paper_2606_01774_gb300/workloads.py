@@ -48,6 +48,11 @@ class WorkloadSpec:
     state_prefix_tokens: int
     seed: int
     spare_slots: int = 4
+    # AR-Trust verify round: speculation horizon N (0 = not a verify workload).
+    # The block is [anchor, d_0 .. d_{K-1}, MASK ...] of length block_len
+    # (2N - 1 at steady state); K ~ U{0..N-1} held drafts per request (0 is a
+    # cold start) and the accepted offset a ~ U{0..K}.
+    verify_horizon: int = 0
 
     @property
     def torch_dtype(self):
@@ -103,6 +108,15 @@ WORKLOADS = {
         head_dim_v=128, num_q_heads=16, num_kv_heads=2, head_dim=256, page_size=64,
         prefix_lo=1024, prefix_hi=16384, act_dtype="bf16", denoise_steps=8, accept="uniform",
         accept_fixed=0, state_prefix_tokens=512, seed=4),
+    "ar_trust_verify_batch64": WorkloadSpec(
+        name="ar_trust_verify_batch64",
+        description="AR-Trust verify round over serving_batch64's shapes: 64 requests, horizon "
+                    "N=16 (block 2N-1 = 31: anchor, K ~ U{0..15} drafts, MASK rows), prefix "
+                    "~U[512,8192]; cache-and-scatter commit at accepted offsets ~U{0..K}",
+        num_requests=64, block_len=31, num_qk_heads=16, num_v_heads=32, head_dim_k=128,
+        head_dim_v=128, num_q_heads=16, num_kv_heads=2, head_dim=256, page_size=64,
+        prefix_lo=512, prefix_hi=8192, act_dtype="bf16", denoise_steps=1, accept="full",
+        accept_fixed=0, state_prefix_tokens=512, seed=5, verify_horizon=16),
 }
 
 
@@ -139,6 +153,9 @@ class Workload:
     v_pool: torch.Tensor = None
     page_table: torch.Tensor = None  # [R, max_pages] int32, -1 where unused
     prefix_len: torch.Tensor = None  # [R] int32
+    verify_len: torch.Tensor = None  # [R] int32, K held drafts (verify workloads)
+    verify_accept: torch.Tensor = None  # [R] int32 in [0, K], drafts accepted
+    row_type: torch.Tensor = None  # [R, block_len] uint8: 0 for rows 0..K, else 1
 
 
 def _l2n(x: torch.Tensor) -> torch.Tensor:
@@ -223,4 +240,14 @@ def generate(spec: WorkloadSpec, device="cpu", *, softmax=True, linear=True) -> 
             kb = torch.randn(R, B, Hkv, D, **f32).to(dtype)
             vb = torch.randn(R, B, Hkv, D, **f32).to(dtype)
             w.softmax.append(SoftmaxBlock(qs.contiguous(), kb.contiguous(), vb.contiguous()))
+    if spec.verify_horizon:
+        N = spec.verify_horizon
+        if N < 2 or N > B:
+            raise ValueError("verify horizon does not fit the block")
+        K = torch.randint(0, N, (R,), generator=gen, device=device, dtype=torch.int32)
+        u = torch.rand(R, generator=gen, device=device)
+        a = torch.minimum((u * (K + 1).float()).floor().to(torch.int32), K)
+        w.verify_len, w.verify_accept = K.contiguous(), a.contiguous()
+        rows = torch.arange(B, device=device, dtype=torch.int32)
+        w.row_type = (rows[None, :] > K[:, None]).to(torch.uint8).contiguous()
     return w

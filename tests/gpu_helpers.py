@@ -29,11 +29,11 @@ def linear_desc(spec, nslots):
                              act_code(spec), 1.0 / math.sqrt(spec.head_dim_k))
 
 
-def softmax_desc(spec, w, mode=flare.FLARE_MASK_BLOCK_BIDIR):
+def softmax_desc(spec, w, mode=flare.FLARE_MASK_BLOCK_BIDIR, row_type=None):
     return flare.softmax_desc(spec.num_requests, spec.block_len, spec.num_q_heads,
                               spec.num_kv_heads, spec.head_dim, spec.page_size,
                               w.k_pool.shape[0], w.page_table.shape[1], act_code(spec),
-                              1.0 / math.sqrt(spec.head_dim), mode)
+                              1.0 / math.sqrt(spec.head_dim), mode, row_type)
 
 
 def oracle_states(w, requests=None):
@@ -100,10 +100,10 @@ def run_commit(w, pool, causal=False, accept_len=None):
     return co
 
 
-def run_softmax(w, step=0, mode=flare.FLARE_MASK_BLOCK_BIDIR, want_lse=True):
+def run_softmax(w, step=0, mode=flare.FLARE_MASK_BLOCK_BIDIR, want_lse=True, row_type=None):
     spec = w.spec
     sb = w.softmax[step]
-    desc = softmax_desc(spec, w, mode)
+    desc = softmax_desc(spec, w, mode, row_type)
     ws_bytes = flare.flare_softmax_workspace_size(desc)
     ws = torch.empty(max(ws_bytes, 1), dtype=torch.uint8, device=sb.q.device)
     out = torch.empty_like(sb.q)
@@ -147,15 +147,56 @@ def oracle_commit(w, pool_before, requests=None, causal=False, accept_len=None):
     return o
 
 
-def oracle_softmax(w, step=0, requests=None, mode=0):
+def oracle_softmax(w, step=0, requests=None, mode=0, row_type=None):
+    """row_type: [B] (mode 2) or [R,B] (mode 3, rows of `requests` taken here)."""
     spec = w.spec
     req = list(range(spec.num_requests)) if requests is None else list(requests)
     sb = w.softmax[step]
     i = torch.tensor(req, device=sb.q.device)
+    rt = None
+    if mode == 2:
+        rt = row_type.cpu()
+    elif mode == 3:
+        rt = row_type[i].cpu()
     return oracle.block_softmax(sb.q[i].cpu(), sb.k_blk[i].cpu(), sb.v_blk[i].cpu(),
                                 w.k_pool.cpu(), w.v_pool.cpu(), w.page_table[i].cpu(),
                                 w.prefix_len[i].cpu(), scale=1.0 / math.sqrt(spec.head_dim),
-                                mask_mode=mode)
+                                mask_mode=mode, row_type=rt)
+
+
+def run_verify_linear(w, max_verify, verify_len=None, records=None, expect_bits=0):
+    """AR-Trust verify round of the linear layer on w.denoise[0] (updates
+    w.state_pool in place).  Returns (out, records)."""
+    spec = w.spec
+    blk = w.denoise[0]
+    vl = w.verify_len if verify_len is None else verify_len
+    out = torch.empty_like(blk.v)
+    if records is None:
+        records = torch.full((spec.num_requests, max_verify, spec.num_v_heads, spec.head_dim_k,
+                              spec.head_dim_v), float("nan"), device=blk.v.device)
+    st = status_word(blk.v.device)
+    rc = flare.flare_verify_linear_attn(linear_desc(spec, w.state_pool.shape[0]), max_verify,
+                                        blk.q, blk.k, blk.v, blk.log_decay, blk.beta,
+                                        w.state_pool, w.state_slot, vl, out,
+                                        records if max_verify else None, st)
+    flare.check(rc, "flare_verify_linear_attn")
+    rc, bits = flare.flare_read_status(st)
+    assert bits == expect_bits, bits
+    return out, records
+
+
+def oracle_verify(w, pool_before, max_verify, requests=None, verify_len=None):
+    spec = w.spec
+    req = list(range(spec.num_requests)) if requests is None else list(requests)
+    blk = w.denoise[0]
+    vl = w.verify_len if verify_len is None else verify_len
+    i = torch.tensor(req, device=blk.k.device)
+    slots = w.state_slot[i].cpu()
+    pool = pool_before[slots.long()].cpu()
+    return oracle.gdr_verify(blk.q[i].cpu(), blk.k[i].cpu(), blk.v[i].cpu(),
+                             blk.log_decay[i].cpu(), blk.beta[i].cpu(), pool,
+                             np.arange(len(req), dtype=np.int32), vl[i].cpu(), max_verify,
+                             scale=1.0 / math.sqrt(spec.head_dim_k))
 
 
 def rel_fro(a, b):

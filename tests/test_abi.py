@@ -61,3 +61,46 @@ def test_workspace_query_is_host_only(lib):
     assert n >= 0 and n % 256 == 0
     s.num_requests = 0
     assert flare.flare_softmax_workspace_size(s) == 0
+
+
+def _header_param_counts():
+    """Parameter count of every entry point declared in include/flare.h."""
+    import re
+
+    text = re.sub(r"/\*.*?\*/", "", flare.HEADER.read_text(), flags=re.S)
+    counts = {}
+    for m in re.finditer(r"\b(flare_\w+)\s*\(([^;{]*?)\)\s*;", text, re.S):
+        args = m.group(2).strip()
+        counts[m.group(1)] = 0 if args in ("", "void") else args.count(",") + 1
+    return counts
+
+
+def test_binding_signatures_match_the_header(lib):
+    """The ctypes argument lists of the binding have as many entries as the
+    declarations in the header have parameters."""
+    counts = _header_param_counts()
+    assert "flare_verify_linear_attn" in counts and "flare_verify_commit" in counts
+    for name, n in counts.items():
+        fn = getattr(lib, name)
+        if fn.argtypes is not None:
+            assert len(fn.argtypes) == n, (name, len(fn.argtypes), n)
+
+
+def test_verify_entry_points_check_arguments_on_the_host(lib):
+    d = flare.linear_desc(2, 31, 16, 32, 128, 128, 6, flare.FLARE_DT_BF16, 0.088)
+    assert lib.flare_verify_linear_attn(ctypes.byref(d), 15, *([None] * 12)) == \
+        flare.FLARE_ERR_INVALID_ARGUMENT
+    assert lib.flare_verify_linear_attn(ctypes.byref(d), -1, *([None] * 12)) == \
+        flare.FLARE_ERR_INVALID_ARGUMENT
+    assert lib.flare_verify_commit(ctypes.byref(d), 15, 0, *([None] * 7)) == \
+        flare.FLARE_ERR_INVALID_ARGUMENT
+    assert lib.flare_verify_commit(ctypes.byref(d), 15, 65, *([None] * 7)) == \
+        flare.FLARE_ERR_UNSUPPORTED
+    s = flare.softmax_desc(2, 31, 16, 2, 256, 64, 100, 64, flare.FLARE_DT_BF16, 0.0625,
+                           flare.FLARE_MASK_ROW_TYPE_PER_REQUEST, None)
+    n = ctypes.c_size_t(0)
+    assert lib.flare_softmax_workspace_size(ctypes.byref(s), ctypes.byref(n)) == \
+        flare.FLARE_ERR_INVALID_ARGUMENT
+    s.mask_mode = 4
+    assert lib.flare_softmax_workspace_size(ctypes.byref(s), ctypes.byref(n)) == \
+        flare.FLARE_ERR_INVALID_ARGUMENT
