@@ -8,6 +8,11 @@ over fresh block inputs, then one commit of every request's state at its
 accepted length (flare_commit_state).  Metric: block-tokens/s =
 requests x block_len x denoise_steps / step time.
 
+The AR-Trust verify workload (--workload ar_trust_verify_batch64) times the
+verify round instead: flare_verify_linear_attn, flare_block_softmax_attn with
+per-request row types, and flare_verify_commit at the accepted offsets; its
+block-tokens are requests x block_len per round.
+
 Default workload: multistep_batch128 (128 requests, GDN 16 qk / 32 v heads,
 d=128, softmax 16 q / 2 kv heads, D=256, block 64, 8 denoise steps over paged
 prefixes ~U[1024,16384], commit at accepted lengths ~U[1,64]).  Each step
@@ -44,6 +49,7 @@ sys.path.insert(0, ROOT)
 from paper_2606_01774_gb300 import workloads  # noqa: E402
 
 METRIC = "denoise-step attention block-tokens/s"
+VERIFY_METRIC = "AR-Trust verify-round attention block-tokens/s"
 UNIT = "block-tokens/s"
 DEFAULT_WORKLOAD = "multistep_batch128"
 
@@ -100,11 +106,34 @@ def commit_bytes(spec, accept):
             + 2 * R * B * Hv * 4)
 
 
+def verify_linear_bytes(spec, verify_len):
+    """Verify pass: S0 read, live state written, S^(t) written for t < K, plus
+    the block's activations and gates."""
+    st = spec.num_v_heads * spec.head_dim_k * spec.head_dim_v * 4
+    n_rec = int(np.asarray(verify_len).sum())
+    return 2 * spec.num_requests * st + n_rec * st + linear_bytes(spec) - spec.num_requests * st
+
+
+def verify_linear_flops(spec):
+    """fp32 CUDA-core work: per token and head one d_k x d_v product S^T k, one
+    rank-one update and one readout, a multiply-add each."""
+    return 6.0 * spec.num_requests * spec.num_v_heads * spec.block_len * spec.head_dim_k * \
+        spec.head_dim_v
+
+
+def verify_commit_bytes(spec, verify_len, accept):
+    st = spec.num_v_heads * spec.head_dim_k * spec.head_dim_v * 4
+    n = int((np.asarray(accept) < np.asarray(verify_len)).sum())
+    return 2 * n * st
+
+
 # ---------------------------------------------------------------- ncu traffic
 
 
 KERNEL_OF = {"linear": "gdr_denoise_tc_kernel", "softmax": "softmax_tc_kernel",
              "commit": "gdr_commit_kernel"}
+VERIFY_KERNEL_OF = {"linear": "gdr_commit_kernel", "softmax": "softmax_tc_kernel",
+                    "commit": "verify_commit_kernel"}
 
 
 def profiled_traffic(kernel, workload):
@@ -198,10 +227,17 @@ class FlareRunner:
         self.ldesc = flare.linear_desc(s.num_requests, s.block_len, s.num_qk_heads,
                                        s.num_v_heads, s.head_dim_k, s.head_dim_v, nslots,
                                        self.act, 1.0 / math.sqrt(s.head_dim_k))
+        self.verify = s.verify_horizon > 0
+        mode = flare.FLARE_MASK_ROW_TYPE_PER_REQUEST if self.verify else flare.FLARE_MASK_BLOCK_BIDIR
         self.sdesc = flare.softmax_desc(s.num_requests, s.block_len, s.num_q_heads,
                                         s.num_kv_heads, s.head_dim, s.page_size,
                                         self.w.k_pool.shape[0], self.w.page_table.shape[1],
-                                        self.act, 1.0 / math.sqrt(s.head_dim))
+                                        self.act, 1.0 / math.sqrt(s.head_dim), mode,
+                                        self.w.row_type if self.verify else None)
+        if self.verify:
+            self.max_verify = s.verify_horizon - 1
+            self.records = torch.empty(s.num_requests, self.max_verify, s.num_v_heads,
+                                       s.head_dim_k, s.head_dim_v, device=device)
         self.ws_bytes = flare.flare_softmax_workspace_size(self.sdesc)
         self.ws = torch.empty(max(self.ws_bytes, 256), dtype=torch.uint8, device=device)
         self.status = torch.zeros(1, dtype=torch.int32, device=device)
@@ -231,6 +267,14 @@ class FlareRunner:
 
     def linear(self, i, ev=None):
         fl, w, b = self.flare, self.w, self.w.denoise[i]
+        if self.verify:
+            rc = fl.flare_verify_linear_attn(self.ldesc, self.max_verify, b.q, b.k, b.v,
+                                             b.log_decay, b.beta, w.state_pool, w.state_slot,
+                                             w.verify_len, self.lin_out[i], self.records,
+                                             self.status)
+            if rc:
+                fl.check(rc, "flare_verify_linear_attn")
+            return
         rc = fl.flare_block_linear_attn(self.ldesc, b.q, b.k, b.v, b.log_decay, b.beta,
                                         w.state_pool, w.state_slot, self.lin_out[i], self.status)
         if rc:
@@ -246,6 +290,13 @@ class FlareRunner:
 
     def commit(self):
         fl, w, b = self.flare, self.w, self.w.commit
+        if self.verify:
+            rc = fl.flare_verify_commit(self.ldesc, self.max_verify, [self.records],
+                                        [w.state_pool], w.state_slot, w.verify_accept,
+                                        w.verify_len, self.status)
+            if rc:
+                fl.check(rc, "flare_verify_commit")
+            return
         rc = fl.flare_commit_state(self.ldesc, None, b.k, b.v, b.log_decay, b.beta,
                                    w.state_pool, w.state_slot, w.accept_len, None, self.status)
         if rc:
@@ -292,12 +343,18 @@ class E2ERunner:
         self.fr = fr
         w = fr.w
         pin = lambda t: (t.cpu().pin_memory(), t)  # noqa: E731
-        self.groups = [[pin(t) for t in (w.page_table, w.prefix_len, w.accept_len, w.state_slot)]]
+        meta = (w.page_table, w.prefix_len, w.accept_len, w.state_slot)
+        if fr.verify:
+            meta = (w.page_table, w.prefix_len, w.state_slot, w.verify_len, w.row_type)
+        self.groups = [[pin(t) for t in meta]]
         for b, sb in zip(w.denoise, w.softmax):
             self.groups.append([pin(t) for t in (b.q, b.k, b.v, b.log_decay, b.beta,
                                                  sb.q, sb.k_blk, sb.v_blk)])
-        self.groups.append([pin(t) for t in (w.commit.k, w.commit.v, w.commit.log_decay,
-                                             w.commit.beta)])
+        if fr.verify:  # the accept decision, known once the round's logits are sampled
+            self.groups.append([pin(w.verify_accept)])
+        else:
+            self.groups.append([pin(t) for t in (w.commit.k, w.commit.v, w.commit.log_decay,
+                                                 w.commit.beta)])
         self.outs = [[(lo, torch.empty(lo.shape, dtype=lo.dtype, pin_memory=True)),
                       (so, torch.empty(so.shape, dtype=so.dtype, pin_memory=True))]
                      for lo, so in zip(fr.lin_out, fr.sm_out)]
@@ -420,27 +477,50 @@ def run_flare(args, spec, rank, world, local_rank):
                         kernel="flare_block_softmax_attn"),
         "commit": dict(bytes=commit_bytes(s, acc), flops=0.0, kernel="flare_commit_state"),
     }
+    if fr.verify:
+        vl, va = fr.w.verify_len.cpu().numpy(), fr.w.verify_accept.cpu().numpy()
+        kern["linear"] = dict(bytes=verify_linear_bytes(s, vl), flops=verify_linear_flops(s),
+                              kernel="flare_verify_linear_attn", fp32_alu=True)
+        kern["commit"] = dict(bytes=verify_commit_bytes(s, vl, va), flops=0.0,
+                              kernel="flare_verify_commit")
     share = {k: per[k] * (s.denoise_steps if k != "commit" else 1) for k in per}
     dom = max(share, key=share.get)
     kd = kern[dom]
     dur_s = per[dom] / 1e3
     t_hbm = kd["bytes"] / (peaks["hbm_gbs"] * 1e9)
     t_tc = kd["flops"] / (peaks["bf16_tflops_sustained"] * 1e12)
-    if t_tc > t_hbm:
+    if kd.get("fp32_alu"):
+        # CUDA-core fp32: 152 SMs x 128 lanes x 2 flops x the median SM clock
+        mhz = (clk or {}).get("sm_mhz") or 1920.0
+        alu_peak = 152 * 128 * 2 * mhz * 1e6 / 1e12
+        t_tc = kd["flops"] / (alu_peak * 1e12)
+    if kd.get("fp32_alu") and t_tc > t_hbm:
+        roof = {"bound": "alu", "achieved": kd["flops"] / dur_s / 1e12, "peak": alu_peak,
+                "unit": "TFLOP/s"}
+    elif t_tc > t_hbm:
         roof = {"bound": "tensor", "achieved": kd["flops"] / dur_s / 1e12,
                 "peak": peaks["bf16_tflops_sustained"], "unit": "TFLOP/s"}
     else:
         roof = {"bound": "hbm", "achieved": kd["bytes"] / dur_s / 1e9,
                 "peak": peaks["hbm_gbs"], "unit": "GB/s"}
     roof["frac"] = roof["achieved"] / roof["peak"]
-    roof["traffic"] = profiled_traffic(KERNEL_OF[dom], s.name)
+    kernel_of = VERIFY_KERNEL_OF if fr.verify else KERNEL_OF
+    roof["traffic"] = profiled_traffic(kernel_of[dom], s.name)
     roof["kernel"] = kd["kernel"]
-    roof["peak_source"] = f"{peaks['source']} ({'bf16_tflops_sustained' if roof['unit'] == 'TFLOP/s' else 'hbm_gbs'})"
+    roof["peak_source"] = (
+        "fp32 CUDA-core count x median SM clock" if roof["bound"] == "alu" else
+        f"{peaks['source']} ({'bf16_tflops_sustained' if roof['unit'] == 'TFLOP/s' else 'hbm_gbs'})")
     roof["algorithmic_per_launch"] = kd["flops"] if roof["bound"] == "tensor" else kd["bytes"]
     step_bytes = s.denoise_steps * (kern["linear"]["bytes"] + kern["softmax"]["bytes"]) + \
         kern["commit"]["bytes"]
+    if fr.verify:
+        s_extra = {"verify_horizon": s.verify_horizon,
+                   "verify_len_mean": float(fr.w.verify_len.float().mean())}
+    else:
+        s_extra = {}
     line = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "metric": METRIC if not fr.verify else VERIFY_METRIC, "value": value, "unit": UNIT,
+        "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": s.act_dtype, "data": "synthetic",
         "config": {"workload": s.name, "requests": s.num_requests, "block_len": s.block_len,
@@ -448,7 +528,8 @@ def run_flare(args, spec, rank, world, local_rank):
                    "head_dim_k": s.head_dim_k, "softmax_heads": [s.num_q_heads, s.num_kv_heads],
                    "head_dim": s.head_dim, "page_size": s.page_size,
                    "prefix": [s.prefix_lo, s.prefix_hi], "parallelism": f"replicas{world}",
-                   "l2": f"no flush: each step streams {step_bytes / 1e9:.2f} GB > 129 MB L2"},
+                   "l2": f"no flush: each step streams {step_bytes / 1e9:.2f} GB > 129 MB L2",
+                   **s_extra},
         "achieved_hbm_gbs": step_bytes / (ms_step / 1e3) / 1e9,
         "per_call_ms": per,
         "roofline": roof,
@@ -489,25 +570,47 @@ def oracle_sample_rate(spec, n_requests, seed_offset=0, one_head=False):
     pool = S0.astype(np.float32)
     slots = np.arange(R, dtype=np.int32)
     kp, vp = w.k_pool[:, hkv], w.v_pool[:, hkv]
-    t0 = time.perf_counter()
-    oracle.gdr_per_token(b.q[:, :, hk], b.k[:, :, hk], b.v[:, :, hv], b.log_decay[:, :, hv],
-                         b.beta[:, :, hv], pool, slots, None, state=False)
-    t1 = time.perf_counter()
-    oracle.block_softmax(sb.q[:, :, hq], sb.k_blk[:, :, hkv], sb.v_blk[:, :, hkv], kp, vp,
-                         w.page_table, w.prefix_len, scale=1.0 / math.sqrt(sub.head_dim))
-    t2 = time.perf_counter()
-    oracle.gdr_per_token(None, c.k[:, :, hk], c.v[:, :, hv], c.log_decay[:, :, hv],
-                         c.beta[:, :, hv], pool, slots, w.accept_len, blockend=False)
-    t3 = time.perf_counter()
+    if spec.verify_horizon:
+        # AR-Trust verify round: verify pass, per-row-type softmax, commit
+        mv = spec.verify_horizon - 1
+        t0 = time.perf_counter()
+        o = oracle.gdr_verify(b.q[:, :, hk], b.k[:, :, hk], b.v[:, :, hv], b.log_decay[:, :, hv],
+                              b.beta[:, :, hv], pool, slots, w.verify_len, mv)
+        t1 = time.perf_counter()
+        oracle.block_softmax(sb.q[:, :, hq], sb.k_blk[:, :, hkv], sb.v_blk[:, :, hkv], kp, vp,
+                             w.page_table, w.prefix_len, scale=1.0 / math.sqrt(sub.head_dim),
+                             mask_mode=3, row_type=w.row_type)
+        t2 = time.perf_counter()
+        live = pool.astype(np.float64)
+        live[slots] = o["state"]
+        oracle.verify_commit([o["records"]], [live], slots, w.verify_accept, w.verify_len)
+        t3 = time.perf_counter()
+    else:
+        t0 = time.perf_counter()
+        oracle.gdr_per_token(b.q[:, :, hk], b.k[:, :, hk], b.v[:, :, hv], b.log_decay[:, :, hv],
+                             b.beta[:, :, hv], pool, slots, None, state=False)
+        t1 = time.perf_counter()
+        oracle.block_softmax(sb.q[:, :, hq], sb.k_blk[:, :, hkv], sb.v_blk[:, :, hkv], kp, vp,
+                             w.page_table, w.prefix_len, scale=1.0 / math.sqrt(sub.head_dim))
+        t2 = time.perf_counter()
+        oracle.gdr_per_token(None, c.k[:, :, hk], c.v[:, :, hv], c.log_decay[:, :, hv],
+                             c.beta[:, :, hv], pool, slots, w.accept_len, blockend=False)
+        t3 = time.perf_counter()
     f_v = sub.num_v_heads if one_head else 1
     f_q = sub.num_q_heads if one_head else 1
     step_s = spec.denoise_steps * ((t1 - t0) * f_v + (t2 - t1) * f_q) + (t3 - t2) * f_v
     tokens = R * spec.block_len * spec.denoise_steps
     heads = ("q head 0 and v head 0 timed, scaled by the head counts "
              f"({sub.num_q_heads} q, {sub.num_v_heads} v)" if one_head else "all heads")
-    desc = (f"{R} request(s) of {spec.name} drawn on the host with the same recipe "
-            f"(prefix {int(w.prefix_len.sum())} tokens), {heads}: one denoise step "
-            f"(linear + softmax) timed and counted {spec.denoise_steps}x, plus the commit")
+    if spec.verify_horizon:
+        desc = (f"{R} request(s) of {spec.name} drawn on the host with the same recipe "
+                f"(prefix {int(w.prefix_len.sum())} tokens, K = "
+                f"{[int(x) for x in w.verify_len]}), {heads}: the verify pass, the softmax "
+                f"with per-row types and the commit")
+    else:
+        desc = (f"{R} request(s) of {spec.name} drawn on the host with the same recipe "
+                f"(prefix {int(w.prefix_len.sum())} tokens), {heads}: one denoise step "
+                f"(linear + softmax) timed and counted {spec.denoise_steps}x, plus the commit")
     return tokens / step_s, step_s, oracle.max_threads(), desc
 
 
@@ -520,7 +623,8 @@ def run_reference(args, spec):
             secs.append(s)
     value = len(secs) * spec.block_len * spec.denoise_steps / sum(secs)
     return {
-        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "impl": "reference", "metric": METRIC if not spec.verify_horizon else VERIFY_METRIC,
+        "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * float(np.mean(secs)),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic",
