@@ -18,6 +18,8 @@ of the paper it follows, is documented in the C file:
   position (serving appendix, cache-and-scatter).
 * :func:`verify_commit` -- the gather-scatter of the cached state at each
   request's accepted offset into every layer's state pool.
+* :func:`short_conv` -- the two-stream causal ShortConv of a block in its
+  serving form (Eq. short-conv-noisy) and the commit of its W-1-token state.
 * :func:`gather_prefix` -- dense copy of a request's paged prefix.
 * :func:`block_softmax` -- softmax retrieval (Eq. softmax-retrieval) under the
   Diffusion-Trust block mask over the paged prefix plus the block.
@@ -76,6 +78,8 @@ def _load():
         lib.oracle_gdr_verify.restype = I
         lib.oracle_block_softmax.argtypes = [I] * 8 + [D, I, I, P, P, P, P, P, P, P, P, P, P, I]
         lib.oracle_block_softmax.restype = I
+        lib.oracle_short_conv.argtypes = [I] * 6 + [P, P, I, P, I, P, P, P, P, P]
+        lib.oracle_short_conv.restype = I
         lib.oracle_append_kv.argtypes = [I] * 8 + [P] * 7
         lib.oracle_append_kv.restype = I
         lib.oracle_max_threads.argtypes = []
@@ -238,6 +242,42 @@ def verify_commit(records, pools, state_slot, accept, verify_len):
             if acc[r] < vl[r]:
                 pool[slot[r]] = rec[r, acc[r]]
     return outs
+
+
+def short_conv(x, conv_state, state_slot, weight, bias=None, *, silu=True, accept_len=None):
+    """Two-stream causal ShortConv of a block, serving form (Eq. short-conv-noisy).
+
+    Shapes: x [R,B,C]; conv_state [slots, W-1, C] (the last W-1 clean tokens
+    before each request's block, oldest first); state_slot [R]; weight [C,W]
+    (weight[c, i] multiplies lag i); bias [C] or None; accept_len [R] or None.
+    Returns fp64 ``out`` [R,B,C] and, when accept_len is given, ``state``
+    [R, W-1, C], the last W-1 rows of (old state ++ the first accept_len[r]
+    block rows)."""
+    xa, xdt = _arr(x)
+    sa, sdt = _arr(conv_state)
+    if sdt != xdt:
+        raise TypeError("x and conv_state must share an element type")
+    wa, wdt = _arr(weight)
+    ba = None
+    if bias is not None:
+        ba, bdt = _arr(bias)
+        if bdt != wdt:
+            raise TypeError("weight and bias must share an element type")
+    slot = _i32(state_slot)
+    acc = None if accept_len is None else _i32(accept_len)
+    R, B, C = xa.shape
+    W = wa.shape[1]
+    out = np.zeros((R, B, C))
+    st = np.zeros((R, W - 1, C)) if acc is not None else None
+    rc = _load().oracle_short_conv(R, B, C, W, int(bool(silu)), xdt, _ptr(xa), _ptr(sa),
+                                   sa.shape[0], _ptr(slot), wdt, _ptr(wa), _ptr(ba), _ptr(acc),
+                                   _ptr(out), _ptr(st))
+    if rc != 0:
+        raise ValueError("oracle_short_conv: invalid slot, width or accepted length")
+    res = {"out": out}
+    if st is not None:
+        res["state"] = st
+    return res
 
 
 def gather_prefix(r, pool, page_table, prefix_len, page_size):

@@ -27,6 +27,9 @@
  *   draft rows read S_L, the states after the anchor and each verify token
  *   are cached, and the commit copies the cached state at the accepted
  *   offset into the pool.
+ *   two-stream causal ShortConv (Eq. short-conv-noisy): lags inside the block
+ *   read the block, earlier lags the committed W-1-token clean state; the
+ *   state is committed as the last W-1 tokens of (state ++ accepted rows).
  *   chunkwise form (Eq. chunk-state / Eq. f-blk with WY-corrected values):
  *   an independent second implementation used only to pin the first.
  *   softmax retrieval over a visible set (Eq. softmax-retrieval) with the
@@ -355,6 +358,63 @@ int oracle_gdr_chunked(int R, int B, int Hk, int Hv, int dk, int dv, double s,
     free(A);
     free(gam);
     free(S0);
+  }
+  return 0;
+}
+
+/*
+ * Two-stream causal ShortConv of a block (appendix "1D Causal ShortConv:
+ * implementation routes", Eq. short-conv-clean / Eq. short-conv-noisy), in
+ * its serving form.  A depthwise causal convolution of width W over C
+ * channels; for request r and block row l (0-based inside the block) the lag-i
+ * input is the block's own row l - i when it lies inside the block, and
+ * otherwise the committed conv state, i.e. the last W - 1 clean tokens before
+ * the block (the state "is a raw tensor slice" of the clean stream):
+ *     z_{l,i} = x[r][l-i]                      if l - i >= 0
+ *             = conv_state[slot][W-1 + l-i]    otherwise (oldest row first)
+ *     y[r][l][c] = act(bias[c] + sum_{i<W} w[c][i] z_{l,i}[c])
+ * act is the identity (act = 0) or SiLU u / (1 + exp(-u)) (act = 1); bias may
+ * be NULL.  With accept_len non-NULL the state is then committed at length
+ * n = accept_len[r]: state_out[r] = the last W - 1 rows of
+ * (conv_state[slot] ++ x[r][0..n-1]); n = 0 keeps the old state.
+ * Shapes: x [R,B,C]; conv_state [num_slots, W-1, C]; weight [C, W] (w[c][i]
+ * multiplies lag i); bias [C]; out [R,B,C]; state_out [R, W-1, C].
+ * Returns -1 for an invalid slot, width or accepted length.
+ */
+int oracle_short_conv(int R, int B, int C, int W, int act, int act_dt, const void* x,
+                      const void* conv_state, int num_slots, const int32_t* state_slot,
+                      int w_dt, const void* weight, const void* bias,
+                      const int32_t* accept_len, double* out, double* state_out) {
+  if (W < 1 || (act != 0 && act != 1)) return -1;
+  for (int r = 0; r < R; ++r) {
+    if (state_slot[r] < 0 || state_slot[r] >= num_slots) return -1;
+    if (accept_len && (accept_len[r] < 0 || accept_len[r] > B)) return -1;
+  }
+  const int Wm = W - 1;
+  for (int r = 0; r < R; ++r) {
+    const size_t st = (size_t)state_slot[r] * Wm * C;
+    for (int l = 0; l < B; ++l)
+      for (int c = 0; c < C; ++c) {
+        double acc = bias ? ld(bias, w_dt, c) : 0.0;
+        for (int i = 0; i < W; ++i) {
+          const int pos = l - i;
+          const double z = pos >= 0 ? ld(x, act_dt, ((size_t)r * B + pos) * C + c)
+                                     : ld(conv_state, act_dt, st + (size_t)(Wm + pos) * C + c);
+          acc += ld(weight, w_dt, (size_t)c * W + i) * z;
+        }
+        out[((size_t)r * B + l) * C + c] = act ? acc / (1.0 + exp(-acc)) : acc;
+      }
+    if (accept_len && state_out) {
+      const int n = accept_len[r];
+      /* sequence (old state ++ accepted rows); keep its last W - 1 rows */
+      for (int j = 0; j < Wm; ++j) {
+        const int pos = n - Wm + j; /* position in the block, negative = old state */
+        for (int c = 0; c < C; ++c)
+          state_out[((size_t)r * Wm + j) * C + c] =
+              pos >= 0 ? ld(x, act_dt, ((size_t)r * B + pos) * C + c)
+                       : ld(conv_state, act_dt, st + (size_t)(Wm + pos) * C + c);
+      }
+    }
   }
   return 0;
 }
