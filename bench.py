@@ -8,6 +8,10 @@ over fresh block inputs, then one commit of every request's state at its
 accepted length (flare_commit_state).  Metric: block-tokens/s =
 requests x block_len x denoise_steps / step time.
 
+Workloads with a ShortConv (--workload shortconv_serving_batch64) add the GDN
+layer's two-stream causal ShortConv (flare_short_conv) in front of each linear
+call, and its conv-state commit in front of the recurrent-state commit.
+
 The AR-Trust verify workload (--workload ar_trust_verify_batch64) times the
 verify round instead: flare_verify_linear_attn, flare_block_softmax_attn with
 per-request row types, and flare_verify_commit at the accepted offsets; its
@@ -121,6 +125,14 @@ def verify_linear_flops(spec):
         spec.head_dim_v
 
 
+def conv_bytes(spec, commit=False):
+    """ShortConv: block in and out, the conv state read (and written on
+    commit), filter taps and bias."""
+    e = 2 if spec.act_dtype == "bf16" else 4
+    R, B, C, W = spec.num_requests, spec.block_len, spec.conv_channels, spec.conv_width
+    return 2 * R * B * C * e + R * (W - 1) * C * e * (2 if commit else 1) + C * (W + 1) * 4
+
+
 def verify_commit_bytes(spec, verify_len, accept):
     st = spec.num_v_heads * spec.head_dim_k * spec.head_dim_v * 4
     n = int((np.asarray(accept) < np.asarray(verify_len)).sum())
@@ -131,7 +143,8 @@ def verify_commit_bytes(spec, verify_len, accept):
 
 
 KERNEL_OF = {"linear": "gdr_denoise_tc_kernel", "softmax": "softmax_tc_kernel",
-             "commit": "gdr_commit_kernel"}
+             "commit": "gdr_commit_kernel", "shortconv": "short_conv_kernel",
+             "shortconv_commit": "short_conv_kernel"}
 VERIFY_KERNEL_OF = {"linear": "gdr_commit_kernel", "softmax": "softmax_tc_kernel",
                     "commit": "verify_commit_kernel"}
 
@@ -243,6 +256,13 @@ class FlareRunner:
         self.status = torch.zeros(1, dtype=torch.int32, device=device)
         self.lin_out = [torch.empty_like(b.v) for b in self.w.denoise]
         self.sm_out = [torch.empty_like(b.q) for b in self.w.softmax]
+        self.conv = s.conv_width > 0
+        if self.conv:
+            self.cdesc = flare.conv_desc(s.num_requests, s.block_len, s.conv_channels,
+                                         s.conv_width, self.w.conv_state.shape[0], self.act,
+                                         flare.FLARE_ACT_SILU)
+            self.conv_out = [torch.empty_like(x) for x in self.w.conv_x]
+            self.conv_commit_out = torch.empty_like(self.w.conv_commit_x)
         self.prefill_states()
 
     def prefill_states(self):
@@ -302,9 +322,34 @@ class FlareRunner:
         if rc:
             fl.check(rc, "flare_commit_state")
 
+    def shortconv(self, i):
+        """ShortConv of denoise step i's block (i = -1: the state-update pass's
+        block, committing the conv state at the accepted lengths)."""
+        fl, w = self.flare, self.w
+        if i < 0:
+            x, out, acc = w.conv_commit_x, self.conv_commit_out, w.accept_len
+        else:
+            x, out, acc = w.conv_x[i], self.conv_out[i], None
+        rc = fl.flare_short_conv(self.cdesc, x, w.conv_state, w.state_slot, w.conv_weight,
+                                 w.conv_bias, acc, out, self.status)
+        if rc:
+            fl.check(rc, "flare_short_conv")
+
+    def _timed(self, events, key, fn, *args):
+        if events is None:
+            fn(*args)
+            return
+        events.setdefault(key, []).append(torch.cuda.Event(enable_timing=True))
+        events[key][-1].record()
+        fn(*args)
+        events[key].append(torch.cuda.Event(enable_timing=True))
+        events[key][-1].record()
+
     def step(self, events=None):
         """One pass of the hot path; events (if given) bracket each call."""
         for i in range(self.spec.denoise_steps):
+            if self.conv:
+                self._timed(events, "shortconv", self.shortconv, i)
             if events is not None:
                 events["linear"].append(torch.cuda.Event(enable_timing=True))
                 events["linear"][-1].record()
@@ -318,6 +363,8 @@ class FlareRunner:
             if events is not None:
                 events["softmax"].append(torch.cuda.Event(enable_timing=True))
                 events["softmax"][-1].record()
+        if self.conv:
+            self._timed(events, "shortconv_commit", self.shortconv, -1)
         if events is not None:
             events["commit"].append(torch.cuda.Event(enable_timing=True))
             events["commit"][-1].record()
@@ -347,17 +394,21 @@ class E2ERunner:
         if fr.verify:
             meta = (w.page_table, w.prefix_len, w.state_slot, w.verify_len, w.row_type)
         self.groups = [[pin(t) for t in meta]]
-        for b, sb in zip(w.denoise, w.softmax):
-            self.groups.append([pin(t) for t in (b.q, b.k, b.v, b.log_decay, b.beta,
-                                                 sb.q, sb.k_blk, sb.v_blk)])
+        for i, (b, sb) in enumerate(zip(w.denoise, w.softmax)):
+            conv_in = (w.conv_x[i],) if fr.conv else ()
+            self.groups.append([pin(t) for t in conv_in + (b.q, b.k, b.v, b.log_decay, b.beta,
+                                                           sb.q, sb.k_blk, sb.v_blk)])
         if fr.verify:  # the accept decision, known once the round's logits are sampled
             self.groups.append([pin(w.verify_accept)])
         else:
-            self.groups.append([pin(t) for t in (w.commit.k, w.commit.v, w.commit.log_decay,
-                                                 w.commit.beta)])
-        self.outs = [[(lo, torch.empty(lo.shape, dtype=lo.dtype, pin_memory=True)),
-                      (so, torch.empty(so.shape, dtype=so.dtype, pin_memory=True))]
-                     for lo, so in zip(fr.lin_out, fr.sm_out)]
+            conv_in = (w.conv_commit_x,) if fr.conv else ()
+            self.groups.append([pin(t) for t in conv_in + (w.commit.k, w.commit.v,
+                                                           w.commit.log_decay, w.commit.beta)])
+        hbuf = lambda d: (d, torch.empty(d.shape, dtype=d.dtype, pin_memory=True))  # noqa: E731
+        self.outs = [[hbuf(lo), hbuf(so)] for lo, so in zip(fr.lin_out, fr.sm_out)]
+        if fr.conv:
+            for i, co in enumerate(fr.conv_out):
+                self.outs[i].append(hbuf(co))
         self.h2d_bytes = sum(h.numel() * h.element_size() for g in self.groups for h, _ in g)
         self.d2h_bytes = sum(h.numel() * h.element_size() for g in self.outs for _, h in g)
         self.s_h2d = torch.cuda.Stream()
@@ -375,6 +426,8 @@ class E2ERunner:
         cs.wait_event(self.ev_in[0])
         for i in range(fr.spec.denoise_steps):
             cs.wait_event(self.ev_in[i + 1])
+            if fr.conv:
+                fr.shortconv(i)
             fr.linear(i)
             fr.softmax(i)
             self.ev_out[i].record(cs)
@@ -383,6 +436,8 @@ class E2ERunner:
                 for d, h in self.outs[i]:
                     h.copy_(d, non_blocking=True)
         cs.wait_event(self.ev_in[-1])
+        if fr.conv:
+            fr.shortconv(-1)
         fr.commit()
         self.s_d2h.synchronize()
         cs.synchronize()
@@ -427,6 +482,8 @@ def run_flare(args, spec, rank, world, local_rank):
         raise RuntimeError(f"device status {bits:#x} after warm-up")
 
     events = {"linear": [], "softmax": [], "commit": []}
+    if fr.conv:
+        events.update(shortconv=[], shortconv_commit=[])
     clocks = ClockSampler(torch.cuda.current_device()) if rank == 0 else None
     if dist:
         tdist.barrier()
@@ -483,7 +540,12 @@ def run_flare(args, spec, rank, world, local_rank):
                               kernel="flare_verify_linear_attn", fp32_alu=True)
         kern["commit"] = dict(bytes=verify_commit_bytes(s, vl, va), flops=0.0,
                               kernel="flare_verify_commit")
-    share = {k: per[k] * (s.denoise_steps if k != "commit" else 1) for k in per}
+    if fr.conv:
+        kern["shortconv"] = dict(bytes=conv_bytes(s), flops=0.0, kernel="flare_short_conv")
+        kern["shortconv_commit"] = dict(bytes=conv_bytes(s, commit=True), flops=0.0,
+                                        kernel="flare_short_conv")
+    once = ("commit", "shortconv_commit")
+    share = {k: per[k] * (s.denoise_steps if k not in once else 1) for k in per}
     dom = max(share, key=share.get)
     kd = kern[dom]
     dur_s = per[dom] / 1e3
@@ -505,19 +567,23 @@ def run_flare(args, spec, rank, world, local_rank):
                 "peak": peaks["hbm_gbs"], "unit": "GB/s"}
     roof["frac"] = roof["achieved"] / roof["peak"]
     kernel_of = VERIFY_KERNEL_OF if fr.verify else KERNEL_OF
-    roof["traffic"] = profiled_traffic(kernel_of[dom], s.name)
+    roof["traffic"] = profiled_traffic(kernel_of[dom], s.name) if dom in kernel_of else None
     roof["kernel"] = kd["kernel"]
     roof["peak_source"] = (
         "fp32 CUDA-core count x median SM clock" if roof["bound"] == "alu" else
         f"{peaks['source']} ({'bf16_tflops_sustained' if roof['unit'] == 'TFLOP/s' else 'hbm_gbs'})")
     roof["algorithmic_per_launch"] = kd["flops"] if roof["bound"] == "tensor" else kd["bytes"]
-    step_bytes = s.denoise_steps * (kern["linear"]["bytes"] + kern["softmax"]["bytes"]) + \
-        kern["commit"]["bytes"]
+    step_bytes = sum(kd_["bytes"] * (1 if k in once else s.denoise_steps)
+                     for k, kd_ in kern.items())
+    s_extra = {}
     if fr.verify:
         s_extra = {"verify_horizon": s.verify_horizon,
                    "verify_len_mean": float(fr.w.verify_len.float().mean())}
-    else:
-        s_extra = {}
+    if fr.conv:
+        s_extra = {"shortconv": {"width": s.conv_width, "channels": s.conv_channels,
+                                 "activation": "silu"},
+                   "per_call_gbs": {k: kern[k]["bytes"] / (per[k] / 1e3) / 1e9
+                                    for k in ("shortconv", "shortconv_commit")}}
     line = {
         "metric": METRIC if not fr.verify else VERIFY_METRIC, "value": value, "unit": UNIT,
         "n_gpus": world, "steps": args.steps,
@@ -599,6 +665,21 @@ def oracle_sample_rate(spec, n_requests, seed_offset=0, one_head=False):
     f_v = sub.num_v_heads if one_head else 1
     f_q = sub.num_q_heads if one_head else 1
     step_s = spec.denoise_steps * ((t1 - t0) * f_v + (t2 - t1) * f_q) + (t3 - t2) * f_v
+    if spec.conv_width:
+        # the ShortConv of one denoise block and of the committed block; with
+        # one_head, the channels of one v head's share (C / Hv), scaled back
+        C = sub.conv_channels
+        cs = slice(0, C // sub.num_v_heads) if one_head else slice(0, C)
+        f_c = sub.num_v_heads if one_head else 1
+        cpool = w.conv_state[:, :, cs]
+        t4 = time.perf_counter()
+        oracle.short_conv(w.conv_x[0][:, :, cs], cpool, slots_conv(w), w.conv_weight[cs],
+                          w.conv_bias[cs])
+        t5 = time.perf_counter()
+        oracle.short_conv(w.conv_commit_x[:, :, cs], cpool, slots_conv(w), w.conv_weight[cs],
+                          w.conv_bias[cs], accept_len=w.accept_len)
+        t6 = time.perf_counter()
+        step_s += (spec.denoise_steps * (t5 - t4) + (t6 - t5)) * f_c
     tokens = R * spec.block_len * spec.denoise_steps
     heads = ("q head 0 and v head 0 timed, scaled by the head counts "
              f"({sub.num_q_heads} q, {sub.num_v_heads} v)" if one_head else "all heads")
@@ -612,6 +693,10 @@ def oracle_sample_rate(spec, n_requests, seed_offset=0, one_head=False):
                 f"(prefix {int(w.prefix_len.sum())} tokens), {heads}: one denoise step "
                 f"(linear + softmax) timed and counted {spec.denoise_steps}x, plus the commit")
     return tokens / step_s, step_s, oracle.max_threads(), desc
+
+
+def slots_conv(w):
+    return w.state_slot.cpu().numpy().astype(np.int32)
 
 
 def run_reference(args, spec):

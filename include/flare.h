@@ -14,6 +14,7 @@
  *   flare_commit_state        write S^(r) into the state pool
  *   flare_block_softmax_attn  block queries over paged prefix + block
  *   flare_append_kv           append the finalized block to the paged cache
+ *   flare_short_conv          two-stream causal ShortConv of the block, conv-state commit
  *
  * and the attention work of an AR-Trust verify round (decoding appendix):
  *
@@ -25,7 +26,10 @@
  * Conventions shared by every call
  * --------------------------------
  *  - All tensor arguments are DEVICE pointers to contiguous row-major arrays
- *    in the shapes stated per call.  Integer arrays are int32.
+ *    in the shapes stated per call.  Integer arrays are int32.  Activation,
+ *    state, pool, filter and output arrays must start on a 16-byte boundary
+ *    (they are moved in 16-byte pieces); a misaligned one is rejected with
+ *    FLARE_ERR_INVALID_ARGUMENT.
  *  - Ownership: the caller allocates and frees every buffer (inputs, outputs,
  *    pools, workspace, status word).  The library allocates no device memory,
  *    frees nothing and never synchronizes inside a compute call.  Work is
@@ -92,6 +96,9 @@ typedef enum flare_mask_mode {
 #define FLARE_DEV_BAD_VERIFY_LEN 0x20 /* verify_len[r] outside [0, min(max_verify, block_len-1)],
                                          or an accepted offset outside [0, verify_len[r]] */
 
+/* Activation applied after the ShortConv. */
+typedef enum flare_activation { FLARE_ACT_NONE = 0, FLARE_ACT_SILU = 1 } flare_activation;
+
 /* Gated-delta-rule layer shape.
  *   num_requests R, block_len B (1..64), num_qk_heads Hk, num_v_heads Hv
  *   (Hv a multiple of Hk; value head j reads q/k head j / (Hv / Hk)),
@@ -133,6 +140,21 @@ typedef struct flare_softmax_desc {
   flare_mask_mode mask_mode;
   const uint8_t* row_type;
 } flare_softmax_desc;
+
+/* ShortConv shape (the depthwise causal convolution in front of a GDN layer's
+ * q/k/v projections).
+ *   num_requests R, block_len B (>= 1), channels C (a multiple of 8), width W
+ *   (1..4), num_state_slots in the conv-state pool, act_dtype of x, the conv
+ *   state and out, activation after the bias. */
+typedef struct flare_conv_desc {
+  int32_t num_requests;
+  int32_t block_len;
+  int32_t channels;
+  int32_t width;
+  int32_t num_state_slots;
+  flare_dtype act_dtype;
+  flare_activation activation;
+} flare_conv_desc;
 
 /*
  * Denoise pass of a gated-delta-rule layer (Eq. flare-gdn-schedule, noisy
@@ -244,6 +266,35 @@ flare_status flare_verify_commit(const flare_linear_desc* desc, int32_t max_veri
                                  float* const* state_pools, const int32_t* state_slot,
                                  const int32_t* accept, const int32_t* verify_len,
                                  int32_t* dev_status, void* stream);
+
+/*
+ * Two-stream causal ShortConv of a block (appendix "1D Causal ShortConv:
+ * implementation routes", Eq. short-conv-noisy, serving form) and, optionally,
+ * the commit of its conv state.  For request r and block row l the lag-i input
+ * (i < W) is the block's own row l - i when l - i >= 0, and otherwise row
+ * W - 1 + (l - i) of the committed conv state, which holds the last W - 1
+ * clean tokens before the block, oldest first:
+ *     out[r][l][c] = act(bias[c] + sum_i weight[c][i] * z_{l,i}[c])
+ * (act: identity or SiLU u / (1 + e^-u); fp32 arithmetic, one rounding to
+ * act_dtype).  The denoise passes call it with the noisy block and no commit;
+ * the state-update pass (and an AR-Trust round with the anchor plus the
+ * accepted drafts) passes accept_len: after the outputs, each request's slot
+ * becomes the last W - 1 rows of (old state ++ block rows 0..n-1),
+ * n = accept_len[r] in [0, B], a bit copy; n = 0 leaves it unchanged.
+ * Precondition: the state_slot entries are distinct within a committing call.
+ *   x           [R, B, C]                 act_dtype
+ *   conv_state  [num_state_slots, W-1, C] act_dtype (read; written only with accept_len)
+ *   state_slot  [R]                       int32
+ *   weight      [C, W]                    fp32, weight[c][i] multiplies lag i
+ *   bias        [C]                       fp32, nullable
+ *   accept_len  [R]                       int32, nullable (no commit)
+ *   out         [R, B, C]                 act_dtype
+ *   dev_status  FLARE_DEV_BAD_SLOT | FLARE_DEV_BAD_ACCEPT_LEN (the request is skipped)
+ */
+flare_status flare_short_conv(const flare_conv_desc* desc, const void* x, void* conv_state,
+                              const int32_t* state_slot, const float* weight, const float* bias,
+                              const int32_t* accept_len, void* out, int32_t* dev_status,
+                              void* stream);
 
 /*
  * Bytes of device workspace flare_block_softmax_attn needs for `desc`

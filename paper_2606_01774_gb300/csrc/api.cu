@@ -337,6 +337,43 @@ flare_status flare_verify_commit(const flare_linear_desc* d, int32_t max_verify,
   return e == cudaSuccess ? FLARE_OK : FLARE_ERR_CUDA;
 }
 
+flare_status flare_short_conv(const flare_conv_desc* d, const void* x, void* conv_state,
+                              const int32_t* state_slot, const float* weight, const float* bias,
+                              const int32_t* accept_len, void* out, int32_t* dev_status,
+                              void* stream) {
+  if (!d) return FLARE_ERR_INVALID_ARGUMENT;
+  if (d->num_requests < 0 || d->block_len < 1 || d->channels < 1 || d->num_state_slots < 1 ||
+      d->width < 1 || !valid_dtype(d->act_dtype) ||
+      (d->activation != FLARE_ACT_NONE && d->activation != FLARE_ACT_SILU))
+    return FLARE_ERR_INVALID_ARGUMENT;
+  if (d->width > 4 || d->channels % 8 != 0) return FLARE_ERR_UNSUPPORTED;
+  if (!x || !state_slot || !weight || !out || !dev_status || (d->width > 1 && !conv_state))
+    return FLARE_ERR_INVALID_ARGUMENT;
+  if (!aligned16(x) || !aligned16(conv_state) || !aligned16(weight) || !aligned16(bias) ||
+      !aligned16(out))
+    return FLARE_ERR_INVALID_ARGUMENT;
+  if (d->num_requests == 0) return FLARE_OK;
+  ConvParams p;
+  memset(&p, 0, sizeof p);
+  p.R = d->num_requests;
+  p.B = d->block_len;
+  p.C = d->channels;
+  p.W = d->width;
+  p.nslots = d->num_state_slots;
+  p.silu = d->activation == FLARE_ACT_SILU;
+  p.x = x;
+  p.conv_state = conv_state;
+  p.state_slot = state_slot;
+  p.weight = weight;
+  p.bias = bias;
+  p.accept_len = accept_len;
+  p.out = out;
+  p.dev_status = dev_status;
+  const cudaError_t e = launch_short_conv(p, d->act_dtype == FLARE_DT_BF16,
+                                          static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? FLARE_OK : FLARE_ERR_CUDA;
+}
+
 flare_status flare_softmax_workspace_size(const flare_softmax_desc* d, size_t* bytes) {
   flare_status st = check_softmax(d);
   if (st != FLARE_OK) return st;

@@ -87,6 +87,19 @@ struct VerifyCommitParams {
   int32_t* dev_status;
 };
 cudaError_t launch_verify_commit(const VerifyCommitParams& p, cudaStream_t stream);
+
+struct ConvParams {
+  int R, B, C, W, nslots, silu;
+  const void* x;              // [R,B,C]
+  void* conv_state;           // [nslots,W-1,C]
+  const int32_t* state_slot;  // [R]
+  const float* weight;        // [C,W]
+  const float* bias;          // [C] or nullptr
+  const int32_t* accept_len;  // [R] or nullptr (no commit)
+  void* out;                  // [R,B,C]
+  int32_t* dev_status;
+};
+cudaError_t launch_short_conv(const ConvParams& p, bool bf16, cudaStream_t stream);
 cudaError_t launch_gdr_denoise_tc(const GdrParams& p, cudaStream_t stream);
 cudaError_t launch_gdr_recurrent(const GdrParams& p, bool bf16, cudaStream_t stream);
 

@@ -31,6 +31,8 @@ FLARE_MASK_ROW_TYPE_UNIFORM = 2
 FLARE_MASK_ROW_TYPE_PER_REQUEST = 3
 FLARE_ROW_CAUSAL = 0
 FLARE_ROW_BIDIR = 1
+FLARE_ACT_NONE = 0
+FLARE_ACT_SILU = 1
 
 FLARE_DEV_BAD_SLOT = 0x1
 FLARE_DEV_BAD_PAGE = 0x2
@@ -53,6 +55,13 @@ class flare_linear_desc(ctypes.Structure):
                 ("head_dim_k", ctypes.c_int32), ("head_dim_v", ctypes.c_int32),
                 ("num_state_slots", ctypes.c_int32), ("act_dtype", ctypes.c_int),
                 ("scale", ctypes.c_float)]
+
+
+class flare_conv_desc(ctypes.Structure):
+    _fields_ = [("num_requests", ctypes.c_int32), ("block_len", ctypes.c_int32),
+                ("channels", ctypes.c_int32), ("width", ctypes.c_int32),
+                ("num_state_slots", ctypes.c_int32), ("act_dtype", ctypes.c_int),
+                ("activation", ctypes.c_int)]
 
 
 class flare_softmax_desc(ctypes.Structure):
@@ -78,7 +87,9 @@ def load() -> ctypes.CDLL:
     P, S, I32 = ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int32
     lin = ctypes.POINTER(flare_linear_desc)
     smx = ctypes.POINTER(flare_softmax_desc)
+    cnv = ctypes.POINTER(flare_conv_desc)
     sigs = {
+        "flare_short_conv": [cnv] + [P] * 9,
         "flare_block_linear_attn": [lin] + [P] * 10,
         "flare_commit_state": [lin] + [P] * 11,
         "flare_verify_linear_attn": [lin, I32] + [P] * 12,
@@ -170,6 +181,13 @@ def flare_verify_commit(desc, max_verify, verify_states, state_pools, state_slot
         _p(verify_len), _p(dev_status), _stream(stream))
 
 
+def flare_short_conv(desc, x, conv_state, state_slot, weight, bias, accept_len, out,
+                     dev_status, stream=None) -> int:
+    return load().flare_short_conv(
+        ctypes.byref(desc), _p(x), _p(conv_state), _p(state_slot), _p(weight), _p(bias),
+        _p(accept_len), _p(out), _p(dev_status), _stream(stream))
+
+
 def flare_softmax_workspace_size(desc) -> int:
     n = ctypes.c_size_t(0)
     check(load().flare_softmax_workspace_size(ctypes.byref(desc), ctypes.byref(n)),
@@ -223,6 +241,12 @@ def linear_desc(num_requests, block_len, num_qk_heads, num_v_heads, head_dim_k, 
                 num_state_slots, act_dtype, scale) -> flare_linear_desc:
     return flare_linear_desc(num_requests, block_len, num_qk_heads, num_v_heads, head_dim_k,
                              head_dim_v, num_state_slots, act_dtype, scale)
+
+
+def conv_desc(num_requests, block_len, channels, width, num_state_slots, act_dtype,
+              activation=FLARE_ACT_SILU) -> flare_conv_desc:
+    return flare_conv_desc(num_requests, block_len, channels, width, num_state_slots, act_dtype,
+                           activation)
 
 
 def softmax_desc(num_requests, block_len, num_q_heads, num_kv_heads, head_dim, page_size,

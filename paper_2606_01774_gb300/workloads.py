@@ -53,6 +53,13 @@ class WorkloadSpec:
     # (2N - 1 at steady state); K ~ U{0..N-1} held drafts per request (0 is a
     # cold start) and the accepted offset a ~ U{0..K}.
     verify_horizon: int = 0
+    # Two-stream ShortConv in front of the GDN layer (0 = none): width W over
+    # C = 2 Hk dk + Hv dv channels (the q, k and v projections), SiLU.
+    conv_width: int = 0
+
+    @property
+    def conv_channels(self) -> int:
+        return 2 * self.num_qk_heads * self.head_dim_k + self.num_v_heads * self.head_dim_v
 
     @property
     def torch_dtype(self):
@@ -117,6 +124,15 @@ WORKLOADS = {
         head_dim_v=128, num_q_heads=16, num_kv_heads=2, head_dim=256, page_size=64,
         prefix_lo=512, prefix_hi=8192, act_dtype="bf16", denoise_steps=1, accept="full",
         accept_fixed=0, state_prefix_tokens=512, seed=5, verify_horizon=16),
+    "shortconv_serving_batch64": WorkloadSpec(
+        name="shortconv_serving_batch64",
+        description="serving_batch64 with the GDN layer's two-stream ShortConv in front of the "
+                    "linear attention: W=4, SiLU, over the 8192 q/k/v channels, conv state "
+                    "committed with the recurrent state",
+        num_requests=64, block_len=32, num_qk_heads=16, num_v_heads=32, head_dim_k=128,
+        head_dim_v=128, num_q_heads=16, num_kv_heads=2, head_dim=256, page_size=64,
+        prefix_lo=512, prefix_hi=8192, act_dtype="bf16", denoise_steps=1, accept="full",
+        accept_fixed=0, state_prefix_tokens=512, seed=6, conv_width=4),
 }
 
 
@@ -156,6 +172,11 @@ class Workload:
     verify_len: torch.Tensor = None  # [R] int32, K held drafts (verify workloads)
     verify_accept: torch.Tensor = None  # [R] int32 in [0, K], drafts accepted
     row_type: torch.Tensor = None  # [R, block_len] uint8: 0 for rows 0..K, else 1
+    conv_x: list = field(default_factory=list)  # [R,B,C] block inputs of the ShortConv per step
+    conv_commit_x: torch.Tensor = None  # [R,B,C] the finalized block (state-update pass)
+    conv_state: torch.Tensor = None  # [slots, W-1, C]: last W-1 clean tokens per slot
+    conv_weight: torch.Tensor = None  # [C, W] fp32, column i multiplies lag i
+    conv_bias: torch.Tensor = None  # [C] fp32
 
 
 def _l2n(x: torch.Tensor) -> torch.Tensor:
@@ -250,4 +271,18 @@ def generate(spec: WorkloadSpec, device="cpu", *, softmax=True, linear=True) -> 
         w.verify_len, w.verify_accept = K.contiguous(), a.contiguous()
         rows = torch.arange(B, device=device, dtype=torch.int32)
         w.row_type = (rows[None, :] > K[:, None]).to(torch.uint8).contiguous()
+    if spec.conv_width:
+        W, C = spec.conv_width, spec.conv_channels
+        f32 = dict(generator=gen, device=device, dtype=torch.float32)
+        w.conv_x = [torch.randn(R, B, C, **f32).to(dtype).contiguous()
+                    for _ in range(spec.denoise_steps)]
+        w.conv_commit_x = torch.randn(R, B, C, **f32).to(dtype).contiguous()
+        nslots = w.state_pool.shape[0]
+        cs = torch.randn(nslots, W - 1, C, **f32).to(dtype)
+        unused = torch.ones(nslots, dtype=torch.bool, device=device)
+        unused[w.state_slot.long()] = False
+        cs[unused] = float("nan")
+        w.conv_state = cs.contiguous()
+        w.conv_weight = (torch.randn(C, W, **f32) / math.sqrt(W)).contiguous()
+        w.conv_bias = (0.1 * torch.randn(C, **f32)).contiguous()
     return w
