@@ -18,6 +18,9 @@ of the paper it follows, is documented in the C file:
   position (serving appendix, cache-and-scatter).
 * :func:`verify_commit` -- the gather-scatter of the cached state at each
   request's accepted offset into every layer's state pool.
+* :func:`two_stream_fwd` -- the noisy stream of the two-stream training
+  forward (Eq. noisy-block-fwd): noisy blocks seeded with the clean state at
+  their boundary, read at their block end.
 * :func:`short_conv` -- the two-stream causal ShortConv of a block in its
   serving form (Eq. short-conv-noisy) and the commit of its W-1-token state.
 * :func:`gather_prefix` -- dense copy of a request's paged prefix.
@@ -78,6 +81,9 @@ def _load():
         lib.oracle_gdr_verify.restype = I
         lib.oracle_block_softmax.argtypes = [I] * 8 + [D, I, I, P, P, P, P, P, P, P, P, P, P, I]
         lib.oracle_block_softmax.restype = I
+        lib.oracle_two_stream_fwd.argtypes = [I] * 8 + [D, I, P, P, I, P, P, P, P, P, P, P, I, P,
+                                                        P, P, P, I]
+        lib.oracle_two_stream_fwd.restype = I
         lib.oracle_short_conv.argtypes = [I] * 6 + [P, P, I, P, I, P, P, P, P, P]
         lib.oracle_short_conv.restype = I
         lib.oracle_append_kv.argtypes = [I] * 8 + [P] * 7
@@ -179,6 +185,8 @@ def gdr_chunked(q, k, v, log_decay, beta, state_pool, state_slot, accept_len=Non
     """Chunkwise WY/UT form of the same block (Eq. chunk-state, Eq. f-blk).
 
     Returns ``blockend`` and ``state`` like :func:`gdr_per_token`."""
+    if q is None:
+        raise ValueError("gdr_chunked forms the block-end readout and needs q")
     a = _gdr_args(q, k, v, log_decay, beta, state_pool, state_slot, accept_len)
     R, B, Hv, dk, dv = a["R"], a["B"], a["Hv"], a["dk"], a["dv"]
     s = 1.0 / np.sqrt(dk) if scale is None else float(scale)
@@ -242,6 +250,55 @@ def verify_commit(records, pools, state_slot, accept, verify_len):
             if acc[r] < vl[r]:
                 pool[slot[r]] = rec[r, acc[r]]
     return outs
+
+
+def two_stream_fwd(clean, noisy, S_init, block_len, chunk_len, *, chunk_states=None,
+                   record_chunk_states=False, scale=None, nthreads=0):
+    """Noisy stream of the two-stream GDR training forward (Eq. noisy-block-fwd).
+
+    clean = (k [N,L,Hk,dk], v [N,L,Hv,dv], g [N,L,Hv], beta [N,L,Hv]);
+    noisy = (q, k, v, g, beta) with the same shapes (q like k); S_init
+    [N,Hv,dk,dv] is the clean state before position 0.  With chunk_states
+    [N,Hv,L/C,dk,dv] the clean state is reset to them at every chunk start.
+    Returns fp64 ``out`` [N,L,Hv,dv] and, when asked, ``chunk_states`` (the
+    clean state at each chunk start)."""
+    k, v, g, beta = clean
+    qn, kn, vn, gn, bn = noisy
+    ka, kdt = _arr(k)
+    va, vdt = _arr(v)
+    qna, qdt = _arr(qn)
+    kna, kndt = _arr(kn)
+    vna, vndt = _arr(vn)
+    if len({kdt, vdt, qdt, kndt, vndt}) != 1:
+        raise TypeError("activations must share an element type")
+    ga, gdt = _arr(g)
+    ba, bdt = _arr(beta)
+    gna, gndt = _arr(gn)
+    bna, bndt = _arr(bn)
+    if len({gdt, bdt, gndt, bndt}) != 1:
+        raise TypeError("gates must share an element type")
+    sa, sdt = _arr(S_init)
+    ci = None
+    if chunk_states is not None:
+        ci, cdt = _arr(chunk_states)
+        if cdt != sdt:
+            raise TypeError("chunk states and S_init must share an element type")
+    N, L, Hk, dk = ka.shape
+    Hv, dv = va.shape[2], va.shape[3]
+    s = 1.0 / np.sqrt(dk) if scale is None else float(scale)
+    out = np.zeros((N, L, Hv, dv))
+    co = np.zeros((N, Hv, L // chunk_len, dk, dv)) if record_chunk_states else None
+    rc = _load().oracle_two_stream_fwd(
+        N, L, Hk, Hv, dk, dv, int(block_len), int(chunk_len), s, kdt, _ptr(ka), _ptr(va), gdt,
+        _ptr(ga), _ptr(ba), _ptr(qna), _ptr(kna), _ptr(vna), _ptr(gna), _ptr(bna), sdt, _ptr(sa),
+        _ptr(ci), _ptr(out), _ptr(co), int(nthreads))
+    if rc != 0:
+        raise ValueError("oracle_two_stream_fwd: block length must divide the chunk length, "
+                         "and the chunk length the sequence length")
+    res = {"out": out}
+    if co is not None:
+        res["chunk_states"] = co
+    return res
 
 
 def short_conv(x, conv_state, state_slot, weight, bias=None, *, silu=True, accept_len=None):

@@ -27,6 +27,9 @@
  *   draft rows read S_L, the states after the anchor and each verify token
  *   are cached, and the commit copies the cached state at the accepted
  *   offset into the pool.
+ *   two-stream training forward (Eq. noisy-block-fwd): each noisy block is
+ *   seeded with the clean state before it, runs its own tokens and reads its
+ *   block-end state; the clean state advances block by block (Eq. f-blk).
  *   two-stream causal ShortConv (Eq. short-conv-noisy): lags inside the block
  *   read the block, earlier lags the committed W-1-token clean state; the
  *   state is committed as the last W-1 tokens of (state ++ accepted rows).
@@ -358,6 +361,95 @@ int oracle_gdr_chunked(int R, int B, int Hk, int Hv, int dk, int dv, double s,
     free(A);
     free(gam);
     free(S0);
+  }
+  return 0;
+}
+
+/*
+ * Two-stream training forward of a gated-delta-rule layer, noisy stream
+ * (appendix "Two-stream recurrence and block-level chain rule",
+ * Eq. noisy-block-fwd; Route II computes exactly this, "Fused forward
+ * kernel").  For sequence n and value head j the clean recurrence
+ * (Eq. per-step-fwd on the clean tokens) starts from S_init[n][j]; block b
+ * covers positions bB .. bB+B-1 (0-based).  The noisy recurrence of block b
+ * starts from the clean state before the block, S_{bB}, runs the block's B
+ * noisy tokens through Eq. per-step-fwd, and every noisy position of the
+ * block reads the noisy block-end state:
+ *     out[n][l][j] = s S~_{bB+B}^T q~_l      for every l in block b.
+ * The clean state then advances over the block's clean tokens (which is
+ * f_blk of Eq. f-blk).  Between blocks the noisy state is discarded.
+ * chunk_states_out[n][j][c] (nullable) records the clean state at each chunk
+ * start (positions cC); with chunk_states_in (nullable) the clean state is
+ * instead reset to chunk_states_in[n][j][c] at each chunk start, so that the
+ * computation starts from the same (rounded) chunk states a kernel is given.
+ * Shapes: clean k [N,L,Hk,dk], v [N,L,Hv,dv], g, beta [N,L,Hv]; noisy q, k
+ * [N,L,Hk,dk], v [N,L,Hv,dv], g, beta [N,L,Hv]; S_init [N,Hv,dk,dv]; out
+ * [N,L,Hv,dv]; chunk states [N,Hv,L/C,dk,dv].  Requires B | C and C | L.
+ */
+int oracle_two_stream_fwd(int N, int L, int Hk, int Hv, int dk, int dv, int B, int C, double s,
+                          int act_dt, const void* k, const void* v, int gate_dt, const void* g,
+                          const void* beta, const void* qn, const void* kn, const void* vn,
+                          const void* gn, const void* betan, int state_dt, const void* S_init,
+                          const void* chunk_states_in, double* out, double* chunk_states_out,
+                          int nthreads) {
+  if (B < 1 || C < B || C % B != 0 || L % C != 0) return -1;
+  const int n_chunks = L / C;
+  const size_t nst = (size_t)dk * dv;
+  set_threads(nthreads);
+#pragma omp parallel for schedule(dynamic, 1)
+  for (long item = 0; item < (long)N * Hv; ++item) {
+    const int n = (int)(item / Hv), j = (int)(item % Hv);
+    const int h = (int)(((long)j * Hk) / Hv);
+    double* S = (double*)malloc(sizeof(double) * nst);
+    double* Sn = (double*)malloc(sizeof(double) * nst);
+    double* u = (double*)malloc(sizeof(double) * dv);
+    double* kt = (double*)malloc(sizeof(double) * dk);
+    for (size_t e = 0; e < nst; ++e) S[e] = ld(S_init, state_dt, (size_t)item * nst + e);
+    /* one gated-delta-rule step (Eq. per-step-fwd) of state X on token t of a stream */
+#define GDR_STEP(X, KK, VV, GG, BB, t)                                                    \
+  do {                                                                                    \
+    const size_t kq_ = (((size_t)n * L + (t)) * Hk + h) * dk;                             \
+    const size_t vo_ = (((size_t)n * L + (t)) * Hv + j) * dv;                             \
+    const size_t gb_ = ((size_t)n * L + (t)) * Hv + j;                                    \
+    const double alpha_ = exp(ld(GG, gate_dt, gb_)), bt_ = ld(BB, gate_dt, gb_);          \
+    for (int i = 0; i < dk; ++i) kt[i] = ld(KK, act_dt, kq_ + i);                         \
+    for (size_t e = 0; e < nst; ++e) (X)[e] *= alpha_;                                    \
+    for (int c = 0; c < dv; ++c) u[c] = 0.0;                                              \
+    for (int i = 0; i < dk; ++i)                                                          \
+      for (int c = 0; c < dv; ++c) u[c] += (X)[i * dv + c] * kt[i];                       \
+    for (int c = 0; c < dv; ++c) u[c] = bt_ * (ld(VV, act_dt, vo_ + c) - u[c]);           \
+    for (int i = 0; i < dk; ++i)                                                          \
+      for (int c = 0; c < dv; ++c) (X)[i * dv + c] += kt[i] * u[c];                      \
+  } while (0)
+    for (int b = 0; b < L / B; ++b) {
+      const int t0 = b * B;
+      if (t0 % C == 0) {
+        const size_t co = ((size_t)item * n_chunks + t0 / C) * nst;
+        if (chunk_states_in)
+          for (size_t e = 0; e < nst; ++e) S[e] = ld(chunk_states_in, state_dt, co + e);
+        if (chunk_states_out) memcpy(chunk_states_out + co, S, sizeof(double) * nst);
+      }
+      /* noisy block: seeded with the clean state before the block */
+      memcpy(Sn, S, sizeof(double) * nst);
+      for (int t = t0; t < t0 + B; ++t) GDR_STEP(Sn, kn, vn, gn, betan, t);
+      for (int l = t0; l < t0 + B; ++l) {
+        const size_t ql = (((size_t)n * L + l) * Hk + h) * dk;
+        const size_t ol = (((size_t)n * L + l) * Hv + j) * dv;
+        for (int i = 0; i < dk; ++i) kt[i] = ld(qn, act_dt, ql + i);
+        for (int c = 0; c < dv; ++c) {
+          double acc = 0.0;
+          for (int i = 0; i < dk; ++i) acc += Sn[i * dv + c] * kt[i];
+          out[ol + c] = s * acc;
+        }
+      }
+      /* clean stream advances over the block (f_blk) */
+      for (int t = t0; t < t0 + B; ++t) GDR_STEP(S, k, v, g, beta, t);
+    }
+#undef GDR_STEP
+    free(kt);
+    free(u);
+    free(Sn);
+    free(S);
   }
   return 0;
 }
