@@ -23,6 +23,10 @@
  *   flare_verify_commit       restore the state at the accepted offset
  *   flare_block_softmax_attn  with the per-row ROW_TYPE mask modes
  *
+ * and, for training, the fused two-stream forward of a GDN layer:
+ *
+ *   flare_two_stream_fwd      noisy blocks seeded from the on-chip clean state
+ *
  * Conventions shared by every call
  * --------------------------------
  *  - All tensor arguments are DEVICE pointers to contiguous row-major arrays
@@ -155,6 +159,25 @@ typedef struct flare_conv_desc {
   flare_dtype act_dtype;
   flare_activation activation;
 } flare_conv_desc;
+
+/* Two-stream training layer shape (the noisy stream of a GDN layer).
+ *   num_seqs N, seq_len L (a multiple of chunk_len), chunk_len C (64, the
+ *   chunk of the clean chunkwise pass), block_len B (1, 2, 4, 8 or 16; the
+ *   diffusion block), num_qk_heads Hk, num_v_heads Hv (a multiple of Hk),
+ *   head_dim_k = head_dim_v = 128, act_dtype of the activations and the
+ *   output, scale s of the readout. */
+typedef struct flare_two_stream_desc {
+  int32_t num_seqs;
+  int32_t seq_len;
+  int32_t chunk_len;
+  int32_t block_len;
+  int32_t num_qk_heads;
+  int32_t num_v_heads;
+  int32_t head_dim_k;
+  int32_t head_dim_v;
+  flare_dtype act_dtype;
+  float scale;
+} flare_two_stream_desc;
 
 /*
  * Denoise pass of a gated-delta-rule layer (Eq. flare-gdn-schedule, noisy
@@ -295,6 +318,36 @@ flare_status flare_short_conv(const flare_conv_desc* desc, const void* x, void* 
                               const int32_t* state_slot, const float* weight, const float* bias,
                               const int32_t* accept_len, void* out, int32_t* dev_status,
                               void* stream);
+
+/*
+ * Two-stream training forward of a gated-delta-rule layer, noisy stream: the
+ * Route II fused forward (appendix "Two-stream recurrence and block-level
+ * chain rule", Eq. noisy-block-fwd and Eq. f-blk; "Route II: fused
+ * two-stream").  Sequence n is L clean tokens and L noisy tokens over the
+ * same positions, cut into blocks of B.  The noisy recurrence of block b
+ * starts from the clean state before the block, S_{bB}, runs the block's
+ * noisy tokens through the gated delta rule (Eq. per-step-fwd), and every
+ * noisy position of the block reads the noisy block-end state:
+ *     out[n][l][j] = scale * S~_{bB+B}^T q~[n][l][h]     (l in block b)
+ * The clean state S_{bB} comes from chunk_states (the clean state at the
+ * start of each C-token chunk, as the clean chunkwise pass produces it)
+ * advanced over the clean tokens of the chunk's earlier blocks (f_blk), on
+ * chip; no block-boundary state is written.  The clean outputs are the clean
+ * chunkwise pass's and are not formed here.  Value head j reads q/k head
+ * j / (Hv / Hk).
+ *   chunk_states  [N, Hv, L/C, dk, dv]   fp32
+ *   k, v          [N, L, Hk, dk], [N, L, Hv, dv]   clean, act_dtype
+ *   log_decay, beta [N, L, Hv]           clean, fp32
+ *   q_noisy, k_noisy [N, L, Hk, dk], v_noisy [N, L, Hv, dv]   act_dtype
+ *   log_decay_noisy, beta_noisy [N, L, Hv] fp32
+ *   out_noisy     [N, L, Hv, dv]         act_dtype
+ * No device-detected errors (every index is derived from the shape).
+ */
+flare_status flare_two_stream_fwd(const flare_two_stream_desc* desc, const float* chunk_states,
+                                  const void* k, const void* v, const float* log_decay,
+                                  const float* beta, const void* q_noisy, const void* k_noisy,
+                                  const void* v_noisy, const float* log_decay_noisy,
+                                  const float* beta_noisy, void* out_noisy, void* stream);
 
 /*
  * Bytes of device workspace flare_block_softmax_attn needs for `desc`

@@ -374,6 +374,54 @@ flare_status flare_short_conv(const flare_conv_desc* d, const void* x, void* con
   return e == cudaSuccess ? FLARE_OK : FLARE_ERR_CUDA;
 }
 
+flare_status flare_two_stream_fwd(const flare_two_stream_desc* d, const float* chunk_states,
+                                  const void* k, const void* v, const float* log_decay,
+                                  const float* beta, const void* q_noisy, const void* k_noisy,
+                                  const void* v_noisy, const float* log_decay_noisy,
+                                  const float* beta_noisy, void* out_noisy, void* stream) {
+  if (!d) return FLARE_ERR_INVALID_ARGUMENT;
+  if (d->num_seqs < 0 || d->seq_len < 0 || d->chunk_len < 1 || d->block_len < 1 ||
+      d->num_qk_heads < 1 || d->num_v_heads < 1 || d->num_v_heads % d->num_qk_heads != 0 ||
+      !valid_dtype(d->act_dtype))
+    return FLARE_ERR_INVALID_ARGUMENT;
+  if (d->chunk_len != two_stream_chunk_len() || d->seq_len % d->chunk_len != 0)
+    return FLARE_ERR_UNSUPPORTED;
+  const int B = d->block_len;
+  if (B != 1 && B != 2 && B != 4 && B != 8 && B != 16) return FLARE_ERR_UNSUPPORTED;
+  if (d->head_dim_k != 128 || d->head_dim_v != 128) return FLARE_ERR_UNSUPPORTED;
+  if (!chunk_states || !k || !v || !log_decay || !beta || !q_noisy || !k_noisy || !v_noisy ||
+      !log_decay_noisy || !beta_noisy || !out_noisy)
+    return FLARE_ERR_INVALID_ARGUMENT;
+  if (!aligned16(chunk_states) || !aligned16(k) || !aligned16(v) || !aligned16(q_noisy) ||
+      !aligned16(k_noisy) || !aligned16(v_noisy) || !aligned16(out_noisy))
+    return FLARE_ERR_INVALID_ARGUMENT;
+  if (d->num_seqs == 0 || d->seq_len == 0) return FLARE_OK;
+  TwoStreamParams p;
+  memset(&p, 0, sizeof p);
+  p.N = d->num_seqs;
+  p.L = d->seq_len;
+  p.B = B;
+  p.Hk = d->num_qk_heads;
+  p.Hv = d->num_v_heads;
+  p.dk = d->head_dim_k;
+  p.dv = d->head_dim_v;
+  p.scale = d->scale;
+  p.chunk_states = chunk_states;
+  p.k = k;
+  p.v = v;
+  p.g = log_decay;
+  p.beta = beta;
+  p.qn = q_noisy;
+  p.kn = k_noisy;
+  p.vn = v_noisy;
+  p.gn = log_decay_noisy;
+  p.betan = beta_noisy;
+  p.out = out_noisy;
+  const cudaError_t e = launch_two_stream_fwd(p, d->act_dtype == FLARE_DT_BF16,
+                                              static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? FLARE_OK : FLARE_ERR_CUDA;
+}
+
 flare_status flare_softmax_workspace_size(const flare_softmax_desc* d, size_t* bytes) {
   flare_status st = check_softmax(d);
   if (st != FLARE_OK) return st;

@@ -100,6 +100,24 @@ struct ConvParams {
   int32_t* dev_status;
 };
 cudaError_t launch_short_conv(const ConvParams& p, bool bf16, cudaStream_t stream);
+
+struct TwoStreamParams {
+  int N, L, B, Hk, Hv, dk, dv;
+  float scale;
+  const float* chunk_states;  // [N,Hv,L/64,dk,dv]
+  const void* k;              // clean [N,L,Hk,dk]
+  const void* v;              // clean [N,L,Hv,dv]
+  const float* g;             // clean log-gates [N,L,Hv]
+  const float* beta;
+  const void* qn;             // noisy [N,L,Hk,dk]
+  const void* kn;
+  const void* vn;             // noisy [N,L,Hv,dv]
+  const float* gn;
+  const float* betan;
+  void* out;                  // [N,L,Hv,dv]
+};
+int two_stream_chunk_len();
+cudaError_t launch_two_stream_fwd(const TwoStreamParams& p, bool bf16, cudaStream_t stream);
 cudaError_t launch_gdr_denoise_tc(const GdrParams& p, cudaStream_t stream);
 cudaError_t launch_gdr_recurrent(const GdrParams& p, bool bf16, cudaStream_t stream);
 

@@ -64,6 +64,14 @@ class flare_conv_desc(ctypes.Structure):
                 ("activation", ctypes.c_int)]
 
 
+class flare_two_stream_desc(ctypes.Structure):
+    _fields_ = [("num_seqs", ctypes.c_int32), ("seq_len", ctypes.c_int32),
+                ("chunk_len", ctypes.c_int32), ("block_len", ctypes.c_int32),
+                ("num_qk_heads", ctypes.c_int32), ("num_v_heads", ctypes.c_int32),
+                ("head_dim_k", ctypes.c_int32), ("head_dim_v", ctypes.c_int32),
+                ("act_dtype", ctypes.c_int), ("scale", ctypes.c_float)]
+
+
 class flare_softmax_desc(ctypes.Structure):
     _fields_ = [("num_requests", ctypes.c_int32), ("block_len", ctypes.c_int32),
                 ("num_q_heads", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32),
@@ -88,8 +96,10 @@ def load() -> ctypes.CDLL:
     lin = ctypes.POINTER(flare_linear_desc)
     smx = ctypes.POINTER(flare_softmax_desc)
     cnv = ctypes.POINTER(flare_conv_desc)
+    tsd = ctypes.POINTER(flare_two_stream_desc)
     sigs = {
         "flare_short_conv": [cnv] + [P] * 9,
+        "flare_two_stream_fwd": [tsd] + [P] * 12,
         "flare_block_linear_attn": [lin] + [P] * 10,
         "flare_commit_state": [lin] + [P] * 11,
         "flare_verify_linear_attn": [lin, I32] + [P] * 12,
@@ -188,6 +198,14 @@ def flare_short_conv(desc, x, conv_state, state_slot, weight, bias, accept_len, 
         _p(accept_len), _p(out), _p(dev_status), _stream(stream))
 
 
+def flare_two_stream_fwd(desc, chunk_states, k, v, log_decay, beta, q_noisy, k_noisy, v_noisy,
+                         log_decay_noisy, beta_noisy, out_noisy, stream=None) -> int:
+    return load().flare_two_stream_fwd(
+        ctypes.byref(desc), _p(chunk_states), _p(k), _p(v), _p(log_decay), _p(beta), _p(q_noisy),
+        _p(k_noisy), _p(v_noisy), _p(log_decay_noisy), _p(beta_noisy), _p(out_noisy),
+        _stream(stream))
+
+
 def flare_softmax_workspace_size(desc) -> int:
     n = ctypes.c_size_t(0)
     check(load().flare_softmax_workspace_size(ctypes.byref(desc), ctypes.byref(n)),
@@ -247,6 +265,12 @@ def conv_desc(num_requests, block_len, channels, width, num_state_slots, act_dty
               activation=FLARE_ACT_SILU) -> flare_conv_desc:
     return flare_conv_desc(num_requests, block_len, channels, width, num_state_slots, act_dtype,
                            activation)
+
+
+def two_stream_desc(num_seqs, seq_len, chunk_len, block_len, num_qk_heads, num_v_heads,
+                    head_dim_k, head_dim_v, act_dtype, scale) -> flare_two_stream_desc:
+    return flare_two_stream_desc(num_seqs, seq_len, chunk_len, block_len, num_qk_heads,
+                                 num_v_heads, head_dim_k, head_dim_v, act_dtype, scale)
 
 
 def softmax_desc(num_requests, block_len, num_q_heads, num_kv_heads, head_dim, page_size,

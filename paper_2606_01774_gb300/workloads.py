@@ -286,3 +286,68 @@ def generate(spec: WorkloadSpec, device="cpu", *, softmax=True, linear=True) -> 
         w.conv_weight = (torch.randn(C, W, **f32) / math.sqrt(W)).contiguous()
         w.conv_bias = (0.1 * torch.randn(C, **f32)).contiguous()
     return w
+
+
+# ---------------------------------------------------------------- training (two-stream)
+
+
+@dataclass(frozen=True)
+class TwoStreamSpec:
+    """Two-stream training input of one GDN layer: N sequences of L clean and
+    L noisy tokens (the paper's "L = 8192, half clean, half noisy" is
+    L = 4096 here), diffusion block B, chunk C of the clean chunkwise pass."""
+    name: str
+    description: str
+    num_seqs: int
+    seq_len: int
+    block_len: int
+    num_qk_heads: int
+    num_v_heads: int
+    head_dim_k: int
+    head_dim_v: int
+    act_dtype: str
+    seed: int
+    chunk_len: int = 64
+
+    @property
+    def torch_dtype(self):
+        return torch.bfloat16 if self.act_dtype == "bf16" else torch.float32
+
+    def replace(self, **kw) -> "TwoStreamSpec":
+        d = dict(self.__dict__)
+        d.update(kw)
+        return TwoStreamSpec(**d)
+
+
+TWO_STREAM_WORKLOADS = {
+    "two_stream_train_b4": TwoStreamSpec(
+        name="two_stream_train_b4",
+        description="Qwen3.5-2B GDN training shape of the paper's route benchmark: 1 sequence, "
+                    "4096 clean + 4096 noisy tokens, 16 heads, d_k = d_v = 128, block B = 4, "
+                    "chunk 64",
+        num_seqs=1, seq_len=4096, block_len=4, num_qk_heads=16, num_v_heads=16, head_dim_k=128,
+        head_dim_v=128, act_dtype="bf16", seed=7),
+}
+
+
+@dataclass
+class TwoStreamInput:
+    spec: TwoStreamSpec
+    clean: LinearBlock  # q unused (the clean outputs are the clean chunkwise pass's)
+    noisy: LinearBlock
+    S_init: torch.Tensor  # [N, Hv, dk, dv] fp32: the clean state before position 0 (zero)
+
+
+def generate_two_stream(spec: TwoStreamSpec, device="cpu") -> TwoStreamInput:
+    """Clean and noisy token streams with the serving value distributions; the
+    clean state before the sequence is zero (a sequence start).  The clean
+    chunk states are NOT built here: each caller runs the clean recurrence
+    with its own implementation."""
+    device = torch.device(device)
+    gen = torch.Generator(device=device)
+    gen.manual_seed(spec.seed)
+    clean = _linear_block(spec, spec.num_seqs, spec.seq_len, gen, device, spec.torch_dtype)
+    noisy = _linear_block(spec, spec.num_seqs, spec.seq_len, gen, device, spec.torch_dtype)
+    S0 = torch.zeros(spec.num_seqs, spec.num_v_heads, spec.head_dim_k, spec.head_dim_v,
+                     device=device, dtype=torch.float32)
+    return TwoStreamInput(spec, clean, noisy, S0)
