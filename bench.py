@@ -12,6 +12,10 @@ Workloads with a ShortConv (--workload shortconv_serving_batch64) add the GDN
 layer's two-stream causal ShortConv (flare_short_conv) in front of each linear
 call, and its conv-state commit in front of the recurrent-state commit.
 
+The training workload (--workload two_stream_train_b4) times the fused
+two-stream forward of one GDN layer (flare_two_stream_fwd) on the paper's
+route-benchmark shape; its metric is training tokens/s (clean + noisy).
+
 The AR-Trust verify workload (--workload ar_trust_verify_batch64) times the
 verify round instead: flare_verify_linear_attn, flare_block_softmax_attn with
 per-request row types, and flare_verify_commit at the accepted offsets; its
@@ -443,6 +447,202 @@ class E2ERunner:
         cs.synchronize()
 
 
+TWO_STREAM_METRIC = "two-stream GDR training forward tokens/s"
+
+
+class TwoStreamRunner:
+    """One GDN layer's fused two-stream forward on one training batch.  The
+    clean chunk states it consumes (what the clean chunkwise pass hands over)
+    are built once by running the library's own exact commit over the clean
+    tokens chunk by chunk."""
+
+    def __init__(self, spec, device, seed_offset=0):
+        from paper_2606_01774_gb300 import flare
+
+        self.flare = flare
+        self.spec = spec.replace(seed=spec.seed + seed_offset)
+        self.device = device
+        self.x = workloads.generate_two_stream(self.spec, device)
+        s, x = self.spec, self.x
+        self.act = flare.FLARE_DT_BF16 if s.act_dtype == "bf16" else flare.FLARE_DT_F32
+        self.scale = 1.0 / math.sqrt(s.head_dim_k)
+        self.desc = flare.two_stream_desc(s.num_seqs, s.seq_len, s.chunk_len, s.block_len,
+                                          s.num_qk_heads, s.num_v_heads, s.head_dim_k,
+                                          s.head_dim_v, self.act, self.scale)
+        n_chunks = s.seq_len // s.chunk_len
+        self.chunk_states = torch.empty(s.num_seqs, s.num_v_heads, n_chunks, s.head_dim_k,
+                                        s.head_dim_v, device=device)
+        self.out = torch.empty_like(x.noisy.v)
+        self._build_chunk_states()
+
+    def _build_chunk_states(self):
+        fl, s, x = self.flare, self.spec, self.x
+        pool = x.S_init.clone()
+        slot = torch.arange(s.num_seqs, dtype=torch.int32, device=self.device)
+        acc = torch.full((s.num_seqs,), s.chunk_len, dtype=torch.int32, device=self.device)
+        st = torch.zeros(1, dtype=torch.int32, device=self.device)
+        d = fl.linear_desc(s.num_seqs, s.chunk_len, s.num_qk_heads, s.num_v_heads, s.head_dim_k,
+                           s.head_dim_v, s.num_seqs, self.act, self.scale)
+        c = x.clean
+        for ci in range(self.chunk_states.shape[2]):
+            self.chunk_states[:, :, ci] = pool
+            sl = slice(ci * s.chunk_len, (ci + 1) * s.chunk_len)
+            fl.check(fl.flare_commit_state(
+                d, None, c.k[:, sl].contiguous(), c.v[:, sl].contiguous(),
+                c.log_decay[:, sl].contiguous(), c.beta[:, sl].contiguous(), pool, slot, acc,
+                None, st), "chunk states")
+        torch.cuda.synchronize()
+        assert fl.flare_read_status(st) == (fl.FLARE_OK, 0)
+
+    def step(self, events=None):
+        fl, c, n = self.flare, self.x.clean, self.x.noisy
+        if events is not None:
+            events["two_stream"].append(torch.cuda.Event(enable_timing=True))
+            events["two_stream"][-1].record()
+        rc = fl.flare_two_stream_fwd(self.desc, self.chunk_states, c.k, c.v, c.log_decay, c.beta,
+                                     n.q, n.k, n.v, n.log_decay, n.beta, self.out)
+        if rc:
+            fl.check(rc, "flare_two_stream_fwd")
+        if events is not None:
+            events["two_stream"].append(torch.cuda.Event(enable_timing=True))
+            events["two_stream"][-1].record()
+
+    def inputs(self):
+        c, n = self.x.clean, self.x.noisy
+        return [self.chunk_states, c.k, c.v, c.log_decay, c.beta, n.q, n.k, n.v, n.log_decay,
+                n.beta]
+
+    def bytes(self):
+        return sum(t.numel() * t.element_size() for t in self.inputs()) + \
+            self.out.numel() * self.out.element_size()
+
+    def flops(self):
+        """fp32 CUDA-core work per token pair: S^T k (clean), S^T k~, S^T q~ and
+        the clean rank-one update, d_k d_v multiply-adds each."""
+        s = self.spec
+        return 8.0 * s.num_seqs * s.num_v_heads * s.seq_len * s.head_dim_k * s.head_dim_v
+
+
+def run_two_stream(args, spec, rank, world, local_rank):
+    device = torch.device("cuda", local_rank)
+    torch.cuda.set_device(device)
+    from paper_2606_01774_gb300 import flare
+
+    flare.load()
+    tr = TwoStreamRunner(spec, device, seed_offset=rank_seed_offset(rank))
+    dist = world > 1
+    if dist:
+        import torch.distributed as tdist
+    for _ in range(args.warmup):
+        tr.step()
+    torch.cuda.synchronize()
+    events = {"two_stream": []}
+    clocks = ClockSampler(torch.cuda.current_device()) if rank == 0 else None
+    if dist:
+        tdist.barrier()
+    torch.cuda.synchronize()
+    launches0 = flare.flare_launch_count()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for _ in range(args.steps):
+        tr.step(events)
+    t1.record()
+    torch.cuda.synchronize()
+    launches = flare.flare_launch_count() - launches0
+    if dist:
+        tdist.barrier()
+    clk = clocks.stop() if clocks else None
+    ms_step = max_over_ranks(t0.elapsed_time(t1), dist, device) / args.steps
+
+    e2e_ms, h2d, d2h = None, 0, 0
+    if not args.no_e2e:
+        pinned = [(t.cpu().pin_memory(), t) for t in tr.inputs()]
+        hout = torch.empty(tr.out.shape, dtype=tr.out.dtype, pin_memory=True)
+        h2d = sum(h.numel() * h.element_size() for h, _ in pinned)
+        d2h = hout.numel() * hout.element_size()
+
+        def e2e_step():
+            for h, d in pinned:
+                d.copy_(h, non_blocking=True)
+            tr.step()
+            hout.copy_(tr.out, non_blocking=True)
+            torch.cuda.current_stream().synchronize()
+
+        for _ in range(max(1, min(args.warmup, 2))):
+            e2e_step()
+        if dist:
+            tdist.barrier()
+        t_e = time.perf_counter()
+        for _ in range(args.steps):
+            e2e_step()
+        e2e_ms = max_over_ranks((time.perf_counter() - t_e) * 1e3 / args.steps, dist, device)
+    if rank != 0:
+        return None
+    s = tr.spec
+    tokens = 2 * s.num_seqs * s.seq_len
+    per = float(np.mean(_elapsed_pairs(events["two_stream"])))
+    mhz = (clk or {}).get("sm_mhz") or 1920.0
+    alu_peak = 152 * 128 * 2 * mhz * 1e6 / 1e12
+    peaks = load_peaks()
+    t_alu = tr.flops() / (alu_peak * 1e12)
+    t_hbm = tr.bytes() / (peaks["hbm_gbs"] * 1e9)
+    if t_alu > t_hbm:
+        roof = {"bound": "alu", "achieved": tr.flops() / (per / 1e3) / 1e12, "peak": alu_peak,
+                "unit": "TFLOP/s", "peak_source": "fp32 CUDA-core count x median SM clock",
+                "algorithmic_per_launch": tr.flops()}
+    else:
+        roof = {"bound": "hbm", "achieved": tr.bytes() / (per / 1e3) / 1e9,
+                "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "peak_source": f"{peaks['source']} (hbm_gbs)",
+                "algorithmic_per_launch": tr.bytes()}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["traffic"] = profiled_traffic("two_stream_fwd_kernel", s.name)
+    roof["kernel"] = "flare_two_stream_fwd"
+    return {
+        "metric": TWO_STREAM_METRIC, "value": world * tokens / (ms_step / 1e3),
+        "unit": "tokens/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": s.act_dtype, "data": "synthetic",
+        "config": {"workload": s.name, "sequences": s.num_seqs, "clean_tokens": s.seq_len,
+                   "noisy_tokens": s.seq_len, "block_len": s.block_len,
+                   "chunk_len": s.chunk_len, "heads": [s.num_qk_heads, s.num_v_heads],
+                   "head_dim": [s.head_dim_k, s.head_dim_v], "parallelism": f"replicas{world}",
+                   "l2": f"no flush: each step reads {tr.bytes() / 1e6:.0f} MB > 129 MB L2",
+                   "context": "paper, one A100-80GB: Route II forward 17.64 ms at B = 4 "
+                              "(clean chunkwise pass included)"},
+        "per_call_ms": {"two_stream": per},
+        "roofline": roof,
+        "e2e": None if e2e_ms is None else {
+            "value": world * tokens / (e2e_ms / 1e3), "unit": "tokens/s", "ms_per_step": e2e_ms,
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": int(launches),
+        "clocks": clk,
+    }
+
+
+def two_stream_oracle_rate(spec, seed_offset=0):
+    """The fp64 oracle on one head of the same sequence (heads are
+    independent), scaled by the head count."""
+    import oracle
+
+    oracle.build()
+    sub = spec.replace(num_qk_heads=1, num_v_heads=1, seed=spec.seed + seed_offset)
+    x = workloads.generate_two_stream(sub, "cpu")
+    c, n = x.clean, x.noisy
+    t0 = time.perf_counter()
+    res = oracle.two_stream_fwd((c.k, c.v, c.log_decay, c.beta),
+                                (n.q, n.k, n.v, n.log_decay, n.beta), x.S_init, sub.block_len,
+                                sub.chunk_len)
+    secs = (time.perf_counter() - t0) * spec.num_v_heads
+    assert np.isfinite(res["out"]).all()
+    tokens = 2 * spec.num_seqs * spec.seq_len
+    desc = (f"one head of {spec.name} ({spec.seq_len} clean + {spec.seq_len} noisy tokens, "
+            f"drawn on the host with the same recipe), timed and scaled by the "
+            f"{spec.num_v_heads} heads")
+    return tokens / secs, secs, oracle.max_threads(), desc
+
+
 def max_over_ranks(x, distributed, device):
     """Max of a per-rank scalar over all ranks (timing only: no data-path collective)."""
     if not distributed:
@@ -725,7 +925,8 @@ def main():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=40)
     ap.add_argument("--warmup", type=int, default=3)
-    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(workloads.WORKLOADS))
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD,
+                    choices=sorted(workloads.WORKLOADS) + sorted(workloads.TWO_STREAM_WORKLOADS))
     ap.add_argument("--impl", default="flare", choices=["flare", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true",
@@ -734,13 +935,31 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "flare":
         ap.error("--warmup must be >= 3")
-    spec = workloads.WORKLOADS[args.workload]
+    training = args.workload in workloads.TWO_STREAM_WORKLOADS
+    spec = (workloads.TWO_STREAM_WORKLOADS if training else workloads.WORKLOADS)[args.workload]
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
 
     if args.impl == "reference":
         if rank != 0:
+            return 0
+        if training:
+            secs = [two_stream_oracle_rate(spec, i)[1] for i in range(args.warmup + args.steps)]
+            rate, _, threads, desc = two_stream_oracle_rate(spec, 0)
+            secs = secs[args.warmup:]
+            value = len(secs) * 2 * spec.num_seqs * spec.seq_len / sum(secs)
+            print(json.dumps({
+                "impl": "reference", "metric": TWO_STREAM_METRIC, "value": value,
+                "unit": "tokens/s", "n_gpus": args.gpus, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": 1e3 * float(np.mean(secs)),
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+                "data": "synthetic",
+                "config": {"workload": spec.name, "parallelism": "host cores"},
+                "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": threads,
+                                 "kind": "oracle", "sample": "each step: " + desc},
+                "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}}), flush=True)
             return 0
         print(json.dumps(run_reference(args, spec)), flush=True)
         return 0
@@ -750,6 +969,17 @@ def main():
 
         torch.cuda.set_device(local_rank)
         tdist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    if training:
+        line = run_two_stream(args, spec, rank, world, local_rank)
+        if rank == 0:
+            if world == 1 and not args.no_cpu_baseline:
+                rate, secs, threads, desc = two_stream_oracle_rate(spec)
+                line["cpu_baseline"] = {"value": rate, "unit": "tokens/s", "cores": threads,
+                                        "kind": "oracle", "sample": desc, "seconds": secs}
+            print(json.dumps(line), flush=True)
+        if world > 1:
+            tdist.destroy_process_group()
+        return 0
     line = run_flare(args, spec, rank, world, local_rank)
     if rank == 0:
         if world == 1 and not args.no_cpu_baseline:
