@@ -5,7 +5,8 @@
 // from the left, so column c of S evolves on its own (Eq. per-step-fwd):
 //     u_t[c] = v_t[c] - alpha_t (S^T k_t)[c],   delta_t[c] = beta_t u_t[c],
 //     S[:, c] <- alpha_t S[:, c] + k_t delta_t[c].
-// Each thread holds a block of 4 columns x d_k/8 rows of S in registers: lane
+// Each thread holds a block of 4 columns x d_k/8 rows of S in registers (as
+// fp32 pairs, so the multiply-adds run as packed f32x2 instructions): lane
 // = 4 * row_group + column_group, so the 8 row groups of a column sit in one
 // warp and meet with three shuffles, each loaded key value serves 4 columns,
 // and the state moves in 16-byte pieces (a warp covers 16 columns, 8 warps a
@@ -125,9 +126,15 @@ __global__ void __launch_bounds__(2 * DV, 2) gdr_commit_kernel(GdrParams p) {
   float* Vs = Qs + (CAUSAL ? steps * DK : 0);        // [steps][DV]
 
   float* Sg = p.state_pool + ((size_t)slot * p.Hv + j) * DK * DV + (size_t)rg * kR * DV + c0;
-  float4 s[kR];  // S~[rg*kR + m][c0 .. c0+3]
+  // S~[rg*kR + m][c0 .. c0+3] as two fp32 pairs (columns c0, c0+1 and c0+2, c0+3):
+  // the products and updates run as packed f32x2 multiply-adds
+  uint64_t s[kR][2];
 #pragma unroll
-  for (int m = 0; m < kR; ++m) s[m] = *reinterpret_cast<const float4*>(Sg + (size_t)m * DV);
+  for (int m = 0; m < kR; ++m) {
+    const ulonglong2 v = *reinterpret_cast<const ulonglong2*>(Sg + (size_t)m * DV);
+    s[m][0] = v.x;
+    s[m][1] = v.y;
+  }
 
   const T* kg = static_cast<const T*>(p.k) + ((size_t)r * B * p.Hk + h) * DK;
   const T* vg = static_cast<const T*>(p.v) + ((size_t)r * B * p.Hv + j) * DV;
@@ -187,7 +194,7 @@ __global__ void __launch_bounds__(2 * DV, 2) gdr_commit_kernel(GdrParams p) {
   // row groups of a warp meeting through shuffles)
   auto readout = [&](int t, float g) {
     const float4* q4 = reinterpret_cast<const float4*>(Qs + t * DK + rg * kR);
-    float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+    uint64_t o01 = 0, o23 = 0;  // fp32 pairs of zero
 #pragma unroll
     for (int m4 = 0; m4 < kR / 4; ++m4) {
       const float4 qq = q4[m4];
@@ -195,12 +202,14 @@ __global__ void __launch_bounds__(2 * DV, 2) gdr_commit_kernel(GdrParams p) {
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         const int m = 4 * m4 + e;
-        o.x = fmaf(s[m].x, qv[e], o.x);
-        o.y = fmaf(s[m].y, qv[e], o.y);
-        o.z = fmaf(s[m].z, qv[e], o.z);
-        o.w = fmaf(s[m].w, qv[e], o.w);
+        const uint64_t q2 = f2_dup(qv[e]);
+        o01 = f2_fma(s[m][0], q2, o01);
+        o23 = f2_fma(s[m][1], q2, o23);
       }
     }
+    float4 o;
+    f2_split(o01, o.x, o.y);
+    f2_split(o23, o.z, o.w);
 #pragma unroll
     for (int sh = 4; sh < 32; sh <<= 1) {
       o.x += __shfl_xor_sync(0xffffffffu, o.x, sh);
@@ -234,13 +243,19 @@ __global__ void __launch_bounds__(2 * DV, 2) gdr_commit_kernel(GdrParams p) {
       }
     }
     // (S~^T k)[c] over this row group, then over the 8 row groups of the warp
-    float4 d = make_float4(0.f, 0.f, 0.f, 0.f);
+    float4 d;
+    {
+      // two partial sums per pair keep four independent multiply-add chains
+      uint64_t d01[2] = {0, 0}, d23[2] = {0, 0};
 #pragma unroll
-    for (int m = 0; m < kR; ++m) {
-      d.x = fmaf(s[m].x, k[m], d.x);
-      d.y = fmaf(s[m].y, k[m], d.y);
-      d.z = fmaf(s[m].z, k[m], d.z);
-      d.w = fmaf(s[m].w, k[m], d.w);
+      for (int m = 0; m < kR; ++m) {
+        const uint64_t k2 = f2_dup(k[m]);
+        d01[m & 1] = f2_fma(s[m][0], k2, d01[m & 1]);
+        d23[m & 1] = f2_fma(s[m][1], k2, d23[m & 1]);
+      }
+      const uint64_t a01 = f2_add(d01[0], d01[1]), a23 = f2_add(d23[0], d23[1]);
+      f2_split(a01, d.x, d.y);
+      f2_split(a23, d.z, d.w);
     }
 #pragma unroll
     for (int o = 4; o < 32; o <<= 1) {
@@ -259,21 +274,21 @@ __global__ void __launch_bounds__(2 * DV, 2) gdr_commit_kernel(GdrParams p) {
     delta.w = bt * (v.w - gt * d.w);
     if (tp.z != 0.f) {  // uniform across the CTA: the gates are per head
       const float ig = tp.z;
-      const float4 w = make_float4(delta.x * ig, delta.y * ig, delta.z * ig, delta.w * ig);
+      const uint64_t w01 = f2(delta.x * ig, delta.y * ig), w23 = f2(delta.z * ig, delta.w * ig);
 #pragma unroll
       for (int m = 0; m < kR; ++m) {
-        s[m].x = fmaf(k[m], w.x, s[m].x);
-        s[m].y = fmaf(k[m], w.y, s[m].y);
-        s[m].z = fmaf(k[m], w.z, s[m].z);
-        s[m].w = fmaf(k[m], w.w, s[m].w);
+        const uint64_t k2 = f2_dup(k[m]);
+        s[m][0] = f2_fma(k2, w01, s[m][0]);
+        s[m][1] = f2_fma(k2, w23, s[m][1]);
       }
     } else {  // fold the decay into the state
+      const uint64_t g2 = f2_dup(gt);
+      const uint64_t d01 = f2(delta.x, delta.y), d23 = f2(delta.z, delta.w);
 #pragma unroll
       for (int m = 0; m < kR; ++m) {
-        s[m].x = fmaf(k[m], delta.x, gt * s[m].x);
-        s[m].y = fmaf(k[m], delta.y, gt * s[m].y);
-        s[m].z = fmaf(k[m], delta.z, gt * s[m].z);
-        s[m].w = fmaf(k[m], delta.w, gt * s[m].w);
+        const uint64_t k2 = f2_dup(k[m]);
+        s[m][0] = f2_fma(k2, d01, f2_mul(g2, s[m][0]));
+        s[m][1] = f2_fma(k2, d23, f2_mul(g2, s[m][1]));
       }
     }
     gam = tp.w;
@@ -282,17 +297,19 @@ __global__ void __launch_bounds__(2 * DV, 2) gdr_commit_kernel(GdrParams p) {
         float* rec = p.verify_states +
                      (((size_t)r * p.max_verify + t) * p.Hv + j) * DK * DV +
                      (size_t)rg * kR * DV + c0;
+        const uint64_t g2 = f2_dup(gam);
 #pragma unroll
         for (int m = 0; m < kR; ++m)
-          __stcs(reinterpret_cast<float4*>(rec + (size_t)m * DV),
-                 make_float4(gam * s[m].x, gam * s[m].y, gam * s[m].z, gam * s[m].w));
+          __stcs(reinterpret_cast<ulonglong2*>(rec + (size_t)m * DV),
+                 make_ulonglong2(f2_mul(g2, s[m][0]), f2_mul(g2, s[m][1])));
       }
     }
     if (t + 1 == n) {
+      const uint64_t g2 = f2_dup(gam);
 #pragma unroll
       for (int m = 0; m < kR; ++m)
-        *reinterpret_cast<float4*>(Sg + (size_t)m * DV) =
-            make_float4(gam * s[m].x, gam * s[m].y, gam * s[m].z, gam * s[m].w);
+        *reinterpret_cast<ulonglong2*>(Sg + (size_t)m * DV) =
+            make_ulonglong2(f2_mul(g2, s[m][0]), f2_mul(g2, s[m][1]));
     }
     if (CAUSAL && (!VERIFY || t <= K)) readout(t, gam);
   }
