@@ -24,7 +24,8 @@
 // prefixes of every block depend only on the inputs, so they are formed for
 // the whole chunk before the block loop.  The decay of the clean state is
 // applied lazily (S = gam S~, folded back when gam would fall below 2^-40).
-// All arithmetic is fp32; the noisy state is never formed.
+// All arithmetic is fp32 (the state products and updates as packed f32x2
+// multiply-adds on column pairs); the noisy state is never formed.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -120,9 +121,13 @@ __global__ void __launch_bounds__(2 * DV, (B <= 4 && sizeof(T) == 2) ? 2 : 1)
   // the chunk-start clean state, issued before anything else
   const float* Sg = p.chunk_states + (((size_t)n * p.Hv + j) * n_chunks + c) * DK * DV +
                     (size_t)rg * kR * DV + c0;
-  float4 s[kR];
+  uint64_t s[kR][2];  // fp32 pairs: columns c0, c0+1 and c0+2, c0+3
 #pragma unroll
-  for (int m = 0; m < kR; ++m) s[m] = __ldg(reinterpret_cast<const float4*>(Sg + (size_t)m * DV));
+  for (int m = 0; m < kR; ++m) {
+    const ulonglong2 v = __ldg(reinterpret_cast<const ulonglong2*>(Sg + (size_t)m * DV));
+    s[m][0] = v.x;
+    s[m][1] = v.y;
+  }
 
   ts_stage<T, DK, kThreads>(ck, static_cast<const T*>(p.k) + (tok0 * p.Hk + h) * DK,
                             (size_t)p.Hk * DK);
@@ -189,20 +194,22 @@ __global__ void __launch_bounds__(2 * DV, (B <= 4 && sizeof(T) == 2) ? 2 : 1)
 #pragma unroll
         for (int u = 0; u < G; ++u) {
           const T* x = (kind == 0 ? ck : (kind == 1 ? nk : nq)) + (t0 + tg + u) * DK + rg * kR;
-          float a4[4] = {0.f, 0.f, 0.f, 0.f};
+          uint64_t a01 = 0, a23 = 0;  // fp32 pairs of zero
 #pragma unroll
           for (int r0 = 0; r0 < kR; r0 += 16) {
             float xf[16];
             load_vec16<T>(x + r0, xf);
 #pragma unroll
             for (int q = 0; q < 16; ++q) {
-              a4[0] = fmaf(s[r0 + q].x, xf[q], a4[0]);
-              a4[1] = fmaf(s[r0 + q].y, xf[q], a4[1]);
-              a4[2] = fmaf(s[r0 + q].z, xf[q], a4[2]);
-              a4[3] = fmaf(s[r0 + q].w, xf[q], a4[3]);
+              const uint64_t x2 = f2_dup(xf[q]);
+              a01 = f2_fma(s[r0 + q][0], x2, a01);
+              a23 = f2_fma(s[r0 + q][1], x2, a23);
             }
           }
-          acc[kind][u] = make_float4(a4[0], a4[1], a4[2], a4[3]);
+          float4 a4;
+          f2_split(a01, a4.x, a4.y);
+          f2_split(a23, a4.z, a4.w);
+          acc[kind][u] = a4;
         }
 #pragma unroll
       for (int kind = 0; kind < 3; ++kind)
@@ -262,13 +269,11 @@ __global__ void __launch_bounds__(2 * DV, (B <= 4 && sizeof(T) == 2) ? 2 : 1)
       const float gB = __expf(lgc[t0 + B - 1]);
       const bool fold = gam * gB < kTsMinGam;  // uniform: the gates are per head
       if (fold) {
-        const float f = gam * gB;
+        const uint64_t f = f2_dup(gam * gB);
 #pragma unroll
         for (int r = 0; r < kR; ++r) {
-          s[r].x *= f;
-          s[r].y *= f;
-          s[r].z *= f;
-          s[r].w *= f;
+          s[r][0] = f2_mul(f, s[r][0]);
+          s[r][1] = f2_mul(f, s[r][1]);
         }
       }
 #pragma unroll 1
@@ -278,7 +283,7 @@ __global__ void __launch_bounds__(2 * DV, (B <= 4 && sizeof(T) == 2) ? 2 : 1)
         const float coef = fold ? __expf(lgc[t0 + B - 1] - lgc[t0 + i])
                                 : __expf(-lgc[t0 + i]) / gam;
         const float4 dd = *reinterpret_cast<const float4*>(Dl + i * DV + c0);
-        const float4 w = make_float4(dd.x * coef, dd.y * coef, dd.z * coef, dd.w * coef);
+        const uint64_t w01 = f2(dd.x * coef, dd.y * coef), w23 = f2(dd.z * coef, dd.w * coef);
         const T* x = ck + (t0 + i) * DK + rg * kR;
 #pragma unroll
         for (int r0 = 0; r0 < kR; r0 += 16) {
@@ -286,10 +291,9 @@ __global__ void __launch_bounds__(2 * DV, (B <= 4 && sizeof(T) == 2) ? 2 : 1)
           load_vec16<T>(x + r0, xf);
 #pragma unroll
           for (int q = 0; q < 16; ++q) {
-            s[r0 + q].x = fmaf(xf[q], w.x, s[r0 + q].x);
-            s[r0 + q].y = fmaf(xf[q], w.y, s[r0 + q].y);
-            s[r0 + q].z = fmaf(xf[q], w.z, s[r0 + q].z);
-            s[r0 + q].w = fmaf(xf[q], w.w, s[r0 + q].w);
+            const uint64_t x2 = f2_dup(xf[q]);
+            s[r0 + q][0] = f2_fma(x2, w01, s[r0 + q][0]);
+            s[r0 + q][1] = f2_fma(x2, w23, s[r0 + q][1]);
           }
         }
       }
