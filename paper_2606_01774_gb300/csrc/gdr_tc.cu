@@ -57,7 +57,7 @@ struct LinCfg {
   static constexpr int kSmem = kR1 + kR2 + kV + kM2 + kD;
 };
 
-struct LinShared {
+struct alignas(16) LinShared {
   uint64_t bar_kq, bar_v, bar_mma;
   uint32_t tmem_base;
   int abort_flag;
@@ -265,21 +265,26 @@ __global__ void __launch_bounds__(kLinThreads, 2)
 #pragma unroll
     for (int c0 = 0; c0 < kBmax; c0 += 16) {
       if (c0 >= Bp) break;
+      // the chunk's log-gates first: the stores below may alias them for the
+      // compiler, which would otherwise reload one after every store
+      float g2[16];
+#pragma unroll
+      for (int e = 0; e < 16; ++e) g2[e] = sh.gam2[c0 + e];
+      float v[16];
       if (tid < 64) {
 #pragma unroll
         for (int e = 0; e < 16; ++e) {
           const int i = c0 + e;
           // A[t][i] = beta_t exp(gamma_t - gamma_i) (k_t . k_i), i < t < B
-          AT[i * kATs + row] = (i < row && row < B)
-                                   ? bt * tc::ex2(gt - sh.gam2[i]) * __uint_as_float(gr[i])
-                                   : 0.f;
+          v[e] = (i < row && row < B) ? bt * tc::ex2(gt - g2[e]) * __uint_as_float(gr[i]) : 0.f;
         }
+#pragma unroll
+        for (int e = 0; e < 16; ++e) AT[(c0 + e) * kATs + row] = v[e];
       } else {
-        float v[16];
 #pragma unroll
         for (int e = 0; e < 16; ++e) {
           const int i = c0 + e;
-          v[e] = (i < B && row < B) ? tc::ex2(gB - sh.gam2[i]) * __uint_as_float(gr[i]) : 0.f;
+          v[e] = (i < B && row < B) ? tc::ex2(gB - g2[e]) * __uint_as_float(gr[i]) : 0.f;
         }
         store16_sw128(M2s, row, c0, v);
       }
@@ -304,13 +309,23 @@ __global__ void __launch_bounds__(kLinThreads, 2)
       uint32_t w[16];
       tc::tmem_ld16(tmW + lane_off + b0, w);  // (K S0)^T[c][t]
       tc::tmem_ld_wait();
+      // the block's gates as 16-byte broadcast loads (the solve is bound by
+      // shared-memory instruction issue)
+      float bb[16], GG[16];
+#pragma unroll
+      for (int e4 = 0; e4 < 4; ++e4) {
+        const float4 b4 = *reinterpret_cast<const float4*>(&sh.beta[b0 + 4 * e4]);
+        const float4 g4 = *reinterpret_cast<const float4*>(&sh.Gam[b0 + 4 * e4]);
+        bb[4 * e4] = b4.x, bb[4 * e4 + 1] = b4.y, bb[4 * e4 + 2] = b4.z, bb[4 * e4 + 3] = b4.w;
+        GG[4 * e4] = g4.x, GG[4 * e4 + 1] = g4.y, GG[4 * e4 + 2] = g4.z, GG[4 * e4 + 3] = g4.w;
+      }
       float x[16];
 #pragma unroll
       for (int e = 0; e < 16; ++e) {
         const int t = b0 + e;
         const float vt =
             __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(vcol + t * 128));
-        x[e] = (t < B && col_ok) ? sh.beta[t] * (vt - sh.Gam[t] * __uint_as_float(w[e])) : 0.f;
+        x[e] = (t < B && col_ok) ? bb[e] * (vt - GG[e] * __uint_as_float(w[e])) : 0.f;
       }
       if (col_ok) {
         if (b0 > 0) {
@@ -414,11 +429,23 @@ __global__ void __launch_bounds__(kLinThreads, 2)
     }
     __syncthreads();
     constexpr int kPieces = DV / 8;  // 16-byte pieces per output row
+    constexpr int kIt = (kBmax * kPieces + kLinThreads - 1) / kLinThreads;
     __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.out_blockend);
-    for (int e = tid; e < B * kPieces; e += kLinThreads) {
-      const int l = e / kPieces, pc = e % kPieces;
-      *reinterpret_cast<uint4*>(out + (((size_t)r * B + l) * p.Hv + j) * DV + pc * 8) =
-          *reinterpret_cast<const uint4*>(stage + l * DV + pc * 8);
+    uint4 piece[kIt];  // every piece read before the first store
+#pragma unroll
+    for (int it = 0; it < kIt; ++it) {
+      const int e = tid + it * kLinThreads;
+      if (e < B * kPieces)
+        piece[it] = *reinterpret_cast<const uint4*>(stage + (e / kPieces) * DV + (e % kPieces) * 8);
+    }
+#pragma unroll
+    for (int it = 0; it < kIt; ++it) {
+      const int e = tid + it * kLinThreads;
+      if (e < B * kPieces) {
+        const int l = e / kPieces, pc = e % kPieces;
+        *reinterpret_cast<uint4*>(out + (((size_t)r * B + l) * p.Hv + j) * DV + pc * 8) =
+            piece[it];
+      }
     }
   }
 
