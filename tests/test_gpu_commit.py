@@ -94,6 +94,23 @@ def test_commit_full_size_sampled():
     assert torch.isfinite(w.state_pool[w.state_slot.long()]).all()
 
 
+@pytest.mark.parametrize("name", ["serving_batch64", "small_model_batch256"])
+def test_commit_full_size_every_request(name):
+    """Full batch, every request's committed slot against the oracle; the slots
+    no request uses keep their bits."""
+    spec = W[name]
+    w = gen(spec)
+    install_states(w)
+    before = w.state_pool.clone()
+    run_commit(w, w.state_pool)
+    ref = oracle_commit(w, before)
+    got = w.state_pool[w.state_slot.long()]
+    assert_states_close(got, ref["state"], name)
+    used = torch.zeros(w.state_pool.shape[0], dtype=torch.bool, device=w.state_pool.device)
+    used[w.state_slot.long()] = True
+    assert torch.equal(w.state_pool[~used].view(torch.int32), before[~used].view(torch.int32))
+
+
 @pytest.mark.parametrize("causal", [False, True])
 def test_commit_strong_decay_folds_the_schedule(causal):
     """Log-gates of -3 per token drive the running decay below 2^-40 inside the

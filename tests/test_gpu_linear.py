@@ -58,6 +58,18 @@ def test_denoise_full_size_sampled(name):
     assert_out_close(out[sample], ref, spec.act_dtype, name)
 
 
+@pytest.mark.parametrize("name", ["serving_batch64", "small_model_batch256"])
+def test_denoise_full_size_every_request(name):
+    """Full batch in the launch configuration bench.py times, every request and
+    head element by element against the per-token recurrence."""
+    spec = W[name]
+    w = gen(spec)
+    install_states(w)
+    out = run_linear(w, spec.denoise_steps - 1)
+    ref = oracle_linear(w, spec.denoise_steps - 1)
+    assert_out_close(out, ref, spec.act_dtype, name)
+
+
 def test_denoise_is_bidirectional_readout():
     """All block rows read the block-end state: equal queries give equal rows."""
     spec = CASES["serving_batch64_r3"]

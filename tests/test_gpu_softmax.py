@@ -59,6 +59,18 @@ def test_softmax_full_size_sampled(name):
     assert np.abs(lse[sample].double().cpu().numpy() - ref_lse).max() < LSE_ABS
 
 
+@pytest.mark.parametrize("name", ["serving_batch64", "small_model_batch256"])
+def test_softmax_full_size_every_request(name):
+    """Full batch in the launch configuration bench.py times, every request,
+    query head and block row element by element (outputs and log-sum-exp)."""
+    spec = W[name]
+    w = gen(spec)
+    out, lse = run_softmax(w, spec.denoise_steps - 1)
+    ref, ref_lse = oracle_softmax(w, spec.denoise_steps - 1)
+    assert_out_close(out, ref, spec.act_dtype, name)
+    assert np.abs(lse.double().cpu().numpy() - ref_lse).max() < LSE_ABS
+
+
 def test_page_shuffle_is_bit_identical():
     """The same logical prefix stored at another permutation of physical pages
     gives bit-identical outputs (the paging is pure address arithmetic)."""
