@@ -344,7 +344,7 @@ __global__ void __launch_bounds__(kLinThreads, 2)
             acc[nt][2] = hi.x;
             acc[nt][3] = hi.y;
           }
-#pragma unroll 1
+#pragma unroll 2
           for (int i0 = 0; i0 < b0; i0 += 8) {
             // -A[t][i] = -A^T[i][t]
             const float* ar = AT + (i0 + q) * kATs + b0 + g;
@@ -368,17 +368,31 @@ __global__ void __launch_bounds__(kLinThreads, 2)
 #pragma unroll
           for (int e = 0; e < 16; ++e) x[e] = D32[(b0 + e) * kS + c];
         }
-        // diagonal block: x_t -= A[t][i] delta_i for b0 <= i < t
+        // diagonal block: x_t -= A[t][i] delta_i for b0 <= i < t; column i of
+        // the block is loaded one step ahead, so the chain through x waits on
+        // multiply-adds only
+        {
+          const float* ad = AT + b0 * kATs + b0;
+          float4 an[4];
 #pragma unroll
-        for (int e = 0; e < 15; ++e) {
-          const float4* a4 = reinterpret_cast<const float4*>(AT + (b0 + e) * kATs + b0);
+          for (int qq = 0; qq < 4; ++qq) an[qq] = reinterpret_cast<const float4*>(ad)[qq];
 #pragma unroll
-          for (int qq = e / 4; qq < 4; ++qq) {
-            const float4 a = a4[qq];
-            if (4 * qq > e) x[4 * qq] = fmaf(-a.x, x[e], x[4 * qq]);
-            if (4 * qq + 1 > e) x[4 * qq + 1] = fmaf(-a.y, x[e], x[4 * qq + 1]);
-            if (4 * qq + 2 > e) x[4 * qq + 2] = fmaf(-a.z, x[e], x[4 * qq + 2]);
-            if (4 * qq + 3 > e) x[4 * qq + 3] = fmaf(-a.w, x[e], x[4 * qq + 3]);
+          for (int e = 0; e < 15; ++e) {
+            float4 a[4];
+#pragma unroll
+            for (int qq = 0; qq < 4; ++qq) a[qq] = an[qq];
+            if (e + 1 < 15) {
+#pragma unroll
+              for (int qq = (e + 1) / 4; qq < 4; ++qq)
+                an[qq] = reinterpret_cast<const float4*>(ad + (e + 1) * kATs)[qq];
+            }
+#pragma unroll
+            for (int qq = e / 4; qq < 4; ++qq) {
+              if (4 * qq > e) x[4 * qq] = fmaf(-a[qq].x, x[e], x[4 * qq]);
+              if (4 * qq + 1 > e) x[4 * qq + 1] = fmaf(-a[qq].y, x[e], x[4 * qq + 1]);
+              if (4 * qq + 2 > e) x[4 * qq + 2] = fmaf(-a[qq].z, x[e], x[4 * qq + 2]);
+              if (4 * qq + 3 > e) x[4 * qq + 3] = fmaf(-a[qq].w, x[e], x[4 * qq + 3]);
+            }
           }
         }
 #pragma unroll
