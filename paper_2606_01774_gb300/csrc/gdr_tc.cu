@@ -40,21 +40,30 @@ namespace {
 
 constexpr int kLinThreads = 128;
 constexpr int kBmax = 64;
-constexpr int kATs = kBmax + 8;  // row stride of A^T: conflict-free tf32 fragment loads
 
-template <int DK, int DV>
+// Layout for blocks of up to BM rows (BM = 64, or 32 for B <= 32, which fits
+// three CTAs on an SM instead of two).
+template <int DK, int DV, int BM>
 struct LinCfg {
-  static constexpr int kKQ = (DK / 64) * 128 * 128;  // [K;Q]: DK/64 chunks of 128 rows x 128 B
-  static constexpr int kAT = kBmax * kATs * 4;       // A^T fp32 [i][t], row stride kATs
-  static constexpr int kR1 = kKQ > kAT ? kKQ : kAT;  // [K;Q], then A^T
+  static constexpr int kATs = BM + 8;                // row stride of A^T: conflict-free tf32 fragment loads
+  static constexpr int kKQ = (DK / 64) * 2 * BM * 128;  // [K;Q]: DK/64 chunks of 2*BM rows x 128 B
+  static constexpr int kAT = BM * kATs * 4;          // A^T fp32 [i][t], row stride kATs
+  static constexpr int kM2 = BM * 128;               // M2 [l][i] K-major
+  // BM = 32: M2 shares the dead [K;Q] region with A^T (1024-byte aligned)
+  static constexpr bool kM2InR1 = BM < 64;
+  static constexpr int kM2Off = (kAT + 1023) / 1024 * 1024;
+  static constexpr int kR1a = kM2InR1 ? kM2Off + kM2 : kAT;
+  static constexpr int kR1 = kKQ > kR1a ? kKQ : kR1a;  // [K;Q], then A^T (and M2), then the output stage
   static constexpr int kS0 = (DV / 64) * DK * 128;   // S0^T, MN-major: DV/64 chunks of DK rows x 128 B
   static constexpr int kDs = DV + 8;                 // row stride of delta fp32
-  static constexpr int kD32 = kBmax * kDs * 4;       // delta fp32 [t][c]
+  static constexpr int kD32 = BM * kDs * 4;          // delta fp32 [t][c]
   static constexpr int kR2 = kS0 > kD32 ? kS0 : kD32;  // S0^T, then delta
-  static constexpr int kV = (DV / 64) * kBmax * 128;  // V [t][c], DV/64 chunks of 64 rows x 128 B
-  static constexpr int kM2 = kBmax * 128;             // M2 [l][i] K-major
-  static constexpr int kD = 128 * 128;                // delta^T [c][t] K-major
-  static constexpr int kSmem = kR1 + kR2 + kV + kM2 + kD;
+  static constexpr int kV = (DV / 64) * BM * 128;    // V [t][c], DV/64 chunks of BM rows x 128 B
+  static constexpr int kD = 128 * 128;               // delta^T [c][t] K-major
+  static constexpr int kSmem = kR1 + kR2 + kV + (kM2InR1 ? 0 : kM2) + kD;
+  static constexpr int kTmemCols = BM == 64 ? 256 : 128;
+  static constexpr int kWCol = BM == 64 ? 128 : 64;  // W^T columns: [K rows | Q rows], 2*BM
+  static constexpr int kMinBlocks = BM == 64 ? 2 : 3;
 };
 
 struct alignas(16) LinShared {
@@ -120,18 +129,19 @@ __device__ __forceinline__ void store16_sw128(uint8_t* tile, int row, int c0, co
 
 }  // namespace
 
-template <int DK, int DV>
-__global__ void __launch_bounds__(kLinThreads, 2)
+template <int DK, int DV, int BM>
+__global__ void __launch_bounds__(kLinThreads, LinCfg<DK, DV, BM>::kMinBlocks)
     gdr_denoise_tc_kernel(const __grid_constant__ LinMaps maps, GdrParams p) {
-  using C = LinCfg<DK, DV>;
+  using C = LinCfg<DK, DV, BM>;
+  constexpr int kATs = C::kATs;
   extern __shared__ uint8_t smem_raw[];
   __shared__ LinShared sh;
   uint8_t* base = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t* KQs = base;
   uint8_t* S0s = KQs + C::kR1;
   uint8_t* Vs = S0s + C::kR2;
-  uint8_t* M2s = Vs + C::kV;
-  uint8_t* Ds = M2s + C::kM2;
+  uint8_t* M2s = C::kM2InR1 ? KQs + C::kM2Off : Vs + C::kV;
+  uint8_t* Ds = Vs + C::kV + (C::kM2InR1 ? 0 : C::kM2);
   float* AT = reinterpret_cast<float*>(KQs);   // A^T[i][t], once MMA 1/2 have run
   float* D32 = reinterpret_cast<float*>(S0s);  // delta[t][c], once MMA 2 has run
 
@@ -171,24 +181,24 @@ __global__ void __launch_bounds__(kLinThreads, 2)
     tc::mbar_init(&sh.bar_mma, 1);
     tc::fence_mbar_init();
   }
-  if (warp == 0) tc::tmem_alloc(&sh.tmem_base, 256);
+  if (warp == 0) tc::tmem_alloc(&sh.tmem_base, C::kTmemCols);
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = sh.tmem_base;
-  const uint32_t tmA = tmem;        // G, then O2^T                 (64 columns)
-  const uint32_t tmW = tmem + 128;  // W^T = S0^T [K;Q]^T           (128 columns)
+  const uint32_t tmA = tmem;             // G, then O2^T                 (BM columns)
+  const uint32_t tmW = tmem + C::kWCol;  // W^T = S0^T [K;Q]^T           (2*BM columns)
   const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
 
   if (tid == 0) {
-    tc::mbar_expect_tx(&sh.bar_kq, 2 * (DK / 64) * kBmax * 128);
+    tc::mbar_expect_tx(&sh.bar_kq, 2 * (DK / 64) * BM * 128);
     for (int c = 0; c < DK / 64; ++c) {
-      tc::tma_load_4d(KQs + c * 16384, &maps.k, &sh.bar_kq, c * 64, h, 0, r);
-      tc::tma_load_4d(KQs + c * 16384 + 8192, &maps.q, &sh.bar_kq, c * 64, h, 0, r);
+      tc::tma_load_4d(KQs + c * (2 * BM * 128), &maps.k, &sh.bar_kq, c * 64, h, 0, r);
+      tc::tma_load_4d(KQs + c * (2 * BM * 128) + BM * 128, &maps.q, &sh.bar_kq, c * 64, h, 0, r);
     }
-    tc::mbar_expect_tx(&sh.bar_v, (DV / 64) * kBmax * 128);
+    tc::mbar_expect_tx(&sh.bar_v, (DV / 64) * BM * 128);
     for (int c = 0; c < DV / 64; ++c)
-      tc::tma_load_4d(Vs + c * (kBmax * 128), &maps.v, &sh.bar_v, c * 64, j, 0, r);
+      tc::tma_load_4d(Vs + c * (BM * 128), &maps.v, &sh.bar_v, c * 64, j, 0, r);
   }
 
   // S0 (fp32, global) -> bf16 S0^T operand, MN-major 128-byte swizzle:
@@ -237,11 +247,13 @@ __global__ void __launch_bounds__(kLinThreads, 2)
   if (tid == 0) {
     tc::fence_after_sync();
     const uint32_t idG = tc::idesc_bf16(128, Bp, false, false);
-    const uint32_t idW = tc::idesc_bf16(128, 128, true, false);
+    const uint32_t idW = tc::idesc_bf16(128, 2 * BM, true, false);
 #pragma unroll
     for (int kk = 0; kk < DK / 16; ++kk) {
       const int c = kk >> 2, off = (kk & 3) * 32;
-      const uint64_t kq = tc::sdesc_sw128(tc::smem_u32(KQs + c * 16384 + off), 16, 1024);
+      // BM = 32: the A operand's rows past the 2*BM of this chunk read the
+      // next bytes of shared memory; those rows of G are never read
+      const uint64_t kq = tc::sdesc_sw128(tc::smem_u32(KQs + c * (2 * BM * 128) + off), 16, 1024);
       tc::mma_bf16_ss(tmA, kq, kq, idG, kk > 0);
       const uint64_t s0 = tc::sdesc_sw128(tc::smem_u32(S0s + kk * 2048), DK * 128, 1024);
       tc::mma_bf16_ss(tmW, s0, kq, idW, kk > 0);
@@ -251,19 +263,20 @@ __global__ void __launch_bounds__(kLinThreads, 2)
   if (!lin_wait(&sh.bar_mma, 0, sh, p.dev_status)) goto done;
   tc::fence_after_sync();
 
-  // ---- A^T (from rows 0..63 of G, fp32) and M2 (rows 64..127, bf16 operand);
-  // all of a row's G values are loaded from tensor memory before any is used
-  {
-    const int row = tid & 63;
+  // ---- A^T (from rows 0..BM-1 of G, fp32) and M2 (rows BM..2BM-1, bf16
+  // operand); all of a row's G values are loaded from tensor memory before any
+  // is used (BM = 32: warps 2 and 3 hold no rows of G)
+  if (tid < 2 * BM) {
+    const int row = tid & (BM - 1);
     const float gB = sh.gam2[B - 1];
     const float bt = sh.beta[row], gt = sh.gam2[row];
-    uint32_t gr[kBmax];
+    uint32_t gr[BM];
 #pragma unroll
-    for (int c0 = 0; c0 < kBmax; c0 += 16)
+    for (int c0 = 0; c0 < BM; c0 += 16)
       if (c0 < Bp) tc::tmem_ld16(tmA + lane_off + c0, *reinterpret_cast<uint32_t(*)[16]>(&gr[c0]));
     tc::tmem_ld_wait();
 #pragma unroll
-    for (int c0 = 0; c0 < kBmax; c0 += 16) {
+    for (int c0 = 0; c0 < BM; c0 += 16) {
       if (c0 >= Bp) break;
       // the chunk's log-gates first: the stores below may alias them for the
       // compiler, which would otherwise reload one after every store
@@ -271,7 +284,7 @@ __global__ void __launch_bounds__(kLinThreads, 2)
 #pragma unroll
       for (int e = 0; e < 16; ++e) g2[e] = sh.gam2[c0 + e];
       float v[16];
-      if (tid < 64) {
+      if (tid < BM) {
 #pragma unroll
         for (int e = 0; e < 16; ++e) {
           const int i = c0 + e;
@@ -303,7 +316,7 @@ __global__ void __launch_bounds__(kLinThreads, 2)
     const int c = tid;
     const bool col_ok = c < DV;  // warp-uniform
     const int g = lane >> 2, q = lane & 3;
-    const uint8_t* vcol = Vs + ((c & (DV - 1)) >> 6) * (kBmax * 128) + (c & 63) * 2;
+    const uint8_t* vcol = Vs + ((c & (DV - 1)) >> 6) * (BM * 128) + (c & 63) * 2;
 #pragma unroll 1
     for (int b0 = 0; b0 < Bp; b0 += 16) {
       uint32_t w[16];
@@ -419,31 +432,31 @@ __global__ void __launch_bounds__(kLinThreads, 2)
   }
   if (!lin_wait(&sh.bar_mma, 1, sh, p.dev_status)) goto done;
   tc::fence_after_sync();
-  // out[l][c] = s (Gam_B W^T[c][64+l] + O2^T[c][l]), staged as bf16 [l][c] in the
+  // out[l][c] = s (Gam_B W^T[c][BM+l] + O2^T[c][l]), staged as bf16 [l][c] in the
   // dead [K;Q] region, then written in 16-byte pieces
   {
     const int c = tid;
     const float GB = sh.Gam[B - 1];
     __nv_bfloat16* stage = reinterpret_cast<__nv_bfloat16*>(KQs);
-    uint32_t o2[kBmax], wq[kBmax];
+    uint32_t o2[BM], wq[BM];
 #pragma unroll
-    for (int c0 = 0; c0 < kBmax; c0 += 16) {
+    for (int c0 = 0; c0 < BM; c0 += 16) {
       if (c0 < Bp) {
         tc::tmem_ld16(tmA + lane_off + c0, *reinterpret_cast<uint32_t(*)[16]>(&o2[c0]));
-        tc::tmem_ld16(tmW + lane_off + 64 + c0, *reinterpret_cast<uint32_t(*)[16]>(&wq[c0]));
+        tc::tmem_ld16(tmW + lane_off + BM + c0, *reinterpret_cast<uint32_t(*)[16]>(&wq[c0]));
       }
     }
     tc::tmem_ld_wait();
     if (c < DV) {
 #pragma unroll
-      for (int l = 0; l < kBmax; ++l)
+      for (int l = 0; l < BM; ++l)
         if (l < B)
           stage[l * DV + c] = __float2bfloat16_rn(
               p.scale * (GB * __uint_as_float(wq[l]) + __uint_as_float(o2[l])));
     }
     __syncthreads();
     constexpr int kPieces = DV / 8;  // 16-byte pieces per output row
-    constexpr int kIt = (kBmax * kPieces + kLinThreads - 1) / kLinThreads;
+    constexpr int kIt = (BM * kPieces + kLinThreads - 1) / kLinThreads;
     __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.out_blockend);
     uint4 piece[kIt];  // every piece read before the first store
 #pragma unroll
@@ -468,7 +481,7 @@ done:
   __syncthreads();
   if (warp == 0) {
     tc::fence_after_sync();
-    tc::tmem_dealloc(tmem, 256);
+    tc::tmem_dealloc(tmem, C::kTmemCols);
   }
 }
 
@@ -489,12 +502,13 @@ PFN_cuTensorMapEncodeTiled_v12000 lin_encode_fn() {
   return fn;
 }
 
-bool lin_map(CUtensorMap* m, const void* ptr, int d, int H, int B, int R, bool swizzle) {
+bool lin_map(CUtensorMap* m, const void* ptr, int d, int H, int B, int R, int box_rows,
+             bool swizzle) {
   auto fn = lin_encode_fn();
   if (!fn) return false;
   cuuint64_t gd[4] = {(cuuint64_t)d, (cuuint64_t)H, (cuuint64_t)B, (cuuint64_t)R};
   cuuint64_t gs[3] = {(cuuint64_t)d * 2, (cuuint64_t)H * d * 2, (cuuint64_t)B * H * d * 2};
-  cuuint32_t bx[4] = {64, 1, (cuuint32_t)kBmax, 1};
+  cuuint32_t bx[4] = {64, 1, (cuuint32_t)box_rows, 1};
   cuuint32_t es[4] = {1, 1, 1, 1};
   return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(ptr), gd, gs, bx, es,
             CU_TENSOR_MAP_INTERLEAVE_NONE,
@@ -503,21 +517,28 @@ bool lin_map(CUtensorMap* m, const void* ptr, int d, int H, int B, int R, bool s
          CUDA_SUCCESS;
 }
 
-template <int DK, int DV>
-cudaError_t launch_lin_tc(const GdrParams& p, cudaStream_t stream) {
-  using C = LinCfg<DK, DV>;
+template <int DK, int DV, int BM>
+cudaError_t launch_lin_tc_bm(const GdrParams& p, cudaStream_t stream) {
+  using C = LinCfg<DK, DV, BM>;
   LinMaps maps;
-  if (!lin_map(&maps.k, p.k, DK, p.Hk, p.B, p.R, true) ||
-      !lin_map(&maps.q, p.q, DK, p.Hk, p.B, p.R, true) ||
-      !lin_map(&maps.v, p.v, DV, p.Hv, p.B, p.R, false))
+  if (!lin_map(&maps.k, p.k, DK, p.Hk, p.B, p.R, BM, true) ||
+      !lin_map(&maps.q, p.q, DK, p.Hk, p.B, p.R, BM, true) ||
+      !lin_map(&maps.v, p.v, DV, p.Hv, p.B, p.R, BM, false))
     return cudaErrorInvalidValue;
   const int smem = C::kSmem + 1024;
-  cudaError_t e = cudaFuncSetAttribute(gdr_denoise_tc_kernel<DK, DV>,
+  cudaError_t e = cudaFuncSetAttribute(gdr_denoise_tc_kernel<DK, DV, BM>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  gdr_denoise_tc_kernel<DK, DV><<<p.R * p.Hv, kLinThreads, smem, stream>>>(maps, p);
+  gdr_denoise_tc_kernel<DK, DV, BM><<<p.R * p.Hv, kLinThreads, smem, stream>>>(maps, p);
   note_launches(1);
   return cudaGetLastError();
+}
+
+// blocks of up to 32 rows take the smaller layout (three CTAs per SM)
+template <int DK, int DV>
+cudaError_t launch_lin_tc(const GdrParams& p, cudaStream_t stream) {
+  return p.B <= 32 ? launch_lin_tc_bm<DK, DV, 32>(p, stream)
+                   : launch_lin_tc_bm<DK, DV, 64>(p, stream);
 }
 
 }  // namespace
