@@ -473,6 +473,7 @@ class TwoStreamRunner:
         self.chunk_states = torch.empty(s.num_seqs, s.num_v_heads, n_chunks, s.head_dim_k,
                                         s.head_dim_v, device=device)
         self.out = torch.empty_like(x.noisy.v)
+        self.status = torch.zeros(1, dtype=torch.int32, device=device)
         self._build_chunk_states()
 
     def _build_chunk_states(self):
@@ -500,7 +501,7 @@ class TwoStreamRunner:
             events["two_stream"].append(torch.cuda.Event(enable_timing=True))
             events["two_stream"][-1].record()
         rc = fl.flare_two_stream_fwd(self.desc, self.chunk_states, c.k, c.v, c.log_decay, c.beta,
-                                     n.q, n.k, n.v, n.log_decay, n.beta, self.out)
+                                     n.q, n.k, n.v, n.log_decay, n.beta, self.out, self.status)
         if rc:
             fl.check(rc, "flare_two_stream_fwd")
         if events is not None:
@@ -577,19 +578,32 @@ def run_two_stream(args, spec, rank, world, local_rank):
         for _ in range(args.steps):
             e2e_step()
         e2e_ms = max_over_ranks((time.perf_counter() - t_e) * 1e3 / args.steps, dist, device)
+    st, bits = tr.flare.flare_read_status(tr.status)
+    if st != tr.flare.FLARE_OK or bits:
+        raise RuntimeError(f"two-stream device status {bits:#x}")
     if rank != 0:
         return None
     s = tr.spec
     tokens = 2 * s.num_seqs * s.seq_len
     per = float(np.mean(_elapsed_pairs(events["two_stream"])))
-    mhz = (clk or {}).get("sm_mhz") or 1920.0
-    alu_peak = 152 * 128 * 2 * mhz * 1e6 / 1e12
     peaks = load_peaks()
-    t_alu = tr.flops() / (alu_peak * 1e12)
+    tc_path = s.act_dtype == "bf16" and s.head_dim_k == 128 and s.head_dim_v == 128
+    if tc_path:
+        # bf16 activations: the state products and updates run as tf32 tensor-core
+        # MMAs; peak = the measured bf16 burst rate x the nominal tf32 / bf16 ratio
+        peak = peaks["bf16_tflops"] * 1.1 / 2.25
+        peak_source = f"{peaks['source']} bf16_tflops x nominal tf32/bf16 (1.1 / 2.25)"
+        bound = "tensor"
+    else:
+        mhz = (clk or {}).get("sm_mhz") or 1920.0
+        peak = 152 * 128 * 2 * mhz * 1e6 / 1e12
+        peak_source = "fp32 CUDA-core count x median SM clock"
+        bound = "alu"
+    t_cmp = tr.flops() / (peak * 1e12)
     t_hbm = tr.bytes() / (peaks["hbm_gbs"] * 1e9)
-    if t_alu > t_hbm:
-        roof = {"bound": "alu", "achieved": tr.flops() / (per / 1e3) / 1e12, "peak": alu_peak,
-                "unit": "TFLOP/s", "peak_source": "fp32 CUDA-core count x median SM clock",
+    if t_cmp > t_hbm:
+        roof = {"bound": bound, "achieved": tr.flops() / (per / 1e3) / 1e12, "peak": peak,
+                "unit": "TFLOP/s", "peak_source": peak_source,
                 "algorithmic_per_launch": tr.flops()}
     else:
         roof = {"bound": "hbm", "achieved": tr.bytes() / (per / 1e3) / 1e9,
@@ -597,7 +611,8 @@ def run_two_stream(args, spec, rank, world, local_rank):
                 "peak_source": f"{peaks['source']} (hbm_gbs)",
                 "algorithmic_per_launch": tr.bytes()}
     roof["frac"] = roof["achieved"] / roof["peak"]
-    roof["traffic"] = profiled_traffic("two_stream_fwd_kernel", s.name)
+    roof["traffic"] = profiled_traffic("two_stream_tc_kernel" if tc_path else "two_stream_fwd_kernel",
+                                       s.name)
     roof["kernel"] = "flare_two_stream_fwd"
     return {
         "metric": TWO_STREAM_METRIC, "value": world * tokens / (ms_step / 1e3),

@@ -341,13 +341,17 @@ flare_status flare_short_conv(const flare_conv_desc* desc, const void* x, void* 
  *   q_noisy, k_noisy [N, L, Hk, dk], v_noisy [N, L, Hv, dv]   act_dtype
  *   log_decay_noisy, beta_noisy [N, L, Hv] fp32
  *   out_noisy     [N, L, Hv, dv]         act_dtype
- * No device-detected errors (every index is derived from the shape).
+ *   dev_status    int32 status word (bits OR-ed in, never cleared)
+ * Every index is derived from the shape, so the only device-detected error is
+ * FLARE_DEV_WAIT_TIMEOUT (a tensor-core pipeline wait that gave up; the
+ * outputs of the affected chunk are then incomplete).
  */
 flare_status flare_two_stream_fwd(const flare_two_stream_desc* desc, const float* chunk_states,
                                   const void* k, const void* v, const float* log_decay,
                                   const float* beta, const void* q_noisy, const void* k_noisy,
                                   const void* v_noisy, const float* log_decay_noisy,
-                                  const float* beta_noisy, void* out_noisy, void* stream);
+                                  const float* beta_noisy, void* out_noisy, int32_t* dev_status,
+                                  void* stream);
 
 /*
  * Bytes of device workspace flare_block_softmax_attn needs for `desc`

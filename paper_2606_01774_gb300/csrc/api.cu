@@ -378,7 +378,8 @@ flare_status flare_two_stream_fwd(const flare_two_stream_desc* d, const float* c
                                   const void* k, const void* v, const float* log_decay,
                                   const float* beta, const void* q_noisy, const void* k_noisy,
                                   const void* v_noisy, const float* log_decay_noisy,
-                                  const float* beta_noisy, void* out_noisy, void* stream) {
+                                  const float* beta_noisy, void* out_noisy, int32_t* dev_status,
+                                  void* stream) {
   if (!d) return FLARE_ERR_INVALID_ARGUMENT;
   if (d->num_seqs < 0 || d->seq_len < 0 || d->chunk_len < 1 || d->block_len < 1 ||
       d->num_qk_heads < 1 || d->num_v_heads < 1 || d->num_v_heads % d->num_qk_heads != 0 ||
@@ -390,7 +391,7 @@ flare_status flare_two_stream_fwd(const flare_two_stream_desc* d, const float* c
   if (B != 1 && B != 2 && B != 4 && B != 8 && B != 16) return FLARE_ERR_UNSUPPORTED;
   if (d->head_dim_k != 128 || d->head_dim_v != 128) return FLARE_ERR_UNSUPPORTED;
   if (!chunk_states || !k || !v || !log_decay || !beta || !q_noisy || !k_noisy || !v_noisy ||
-      !log_decay_noisy || !beta_noisy || !out_noisy)
+      !log_decay_noisy || !beta_noisy || !out_noisy || !dev_status)
     return FLARE_ERR_INVALID_ARGUMENT;
   if (!aligned16(chunk_states) || !aligned16(k) || !aligned16(v) || !aligned16(q_noisy) ||
       !aligned16(k_noisy) || !aligned16(v_noisy) || !aligned16(out_noisy))
@@ -417,6 +418,7 @@ flare_status flare_two_stream_fwd(const flare_two_stream_desc* d, const float* c
   p.gn = log_decay_noisy;
   p.betan = beta_noisy;
   p.out = out_noisy;
+  p.dev_status = dev_status;
   const cudaError_t e = launch_two_stream_fwd(p, d->act_dtype == FLARE_DT_BF16,
                                               static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? FLARE_OK : FLARE_ERR_CUDA;

@@ -99,7 +99,7 @@ def load() -> ctypes.CDLL:
     tsd = ctypes.POINTER(flare_two_stream_desc)
     sigs = {
         "flare_short_conv": [cnv] + [P] * 9,
-        "flare_two_stream_fwd": [tsd] + [P] * 12,
+        "flare_two_stream_fwd": [tsd] + [P] * 13,
         "flare_block_linear_attn": [lin] + [P] * 10,
         "flare_commit_state": [lin] + [P] * 11,
         "flare_verify_linear_attn": [lin, I32] + [P] * 12,
@@ -199,11 +199,11 @@ def flare_short_conv(desc, x, conv_state, state_slot, weight, bias, accept_len, 
 
 
 def flare_two_stream_fwd(desc, chunk_states, k, v, log_decay, beta, q_noisy, k_noisy, v_noisy,
-                         log_decay_noisy, beta_noisy, out_noisy, stream=None) -> int:
+                         log_decay_noisy, beta_noisy, out_noisy, dev_status, stream=None) -> int:
     return load().flare_two_stream_fwd(
         ctypes.byref(desc), _p(chunk_states), _p(k), _p(v), _p(log_decay), _p(beta), _p(q_noisy),
         _p(k_noisy), _p(v_noisy), _p(log_decay_noisy), _p(beta_noisy), _p(out_noisy),
-        _stream(stream))
+        _p(dev_status), _stream(stream))
 
 
 def flare_softmax_workspace_size(desc) -> int:

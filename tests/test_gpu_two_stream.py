@@ -56,10 +56,12 @@ def _run(x, cs):
                               1.0 / math.sqrt(sp.head_dim_k))
     out = torch.empty_like(x.noisy.v)
     c, nz = x.clean, x.noisy
+    st = torch.zeros(1, dtype=torch.int32, device=out.device)
     rc = flare.flare_two_stream_fwd(d, cs, c.k, c.v, c.log_decay, c.beta, nz.q, nz.k, nz.v,
-                                    nz.log_decay, nz.beta, out)
+                                    nz.log_decay, nz.beta, out, st)
     flare.check(rc, "flare_two_stream_fwd")
     torch.cuda.synchronize()
+    assert flare.flare_read_status(st) == (flare.FLARE_OK, 0)
     return out
 
 
@@ -111,7 +113,8 @@ def test_two_stream_host_checks():
     cs = torch.zeros(sp.num_seqs, sp.num_v_heads, sp.seq_len // 64, 128, 128, device="cuda")
     out = torch.empty_like(x.noisy.v)
     c, nz = x.clean, x.noisy
-    args = (cs, c.k, c.v, c.log_decay, c.beta, nz.q, nz.k, nz.v, nz.log_decay, nz.beta, out)
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    args = (cs, c.k, c.v, c.log_decay, c.beta, nz.q, nz.k, nz.v, nz.log_decay, nz.beta, out, st)
     assert flare.flare_two_stream_fwd(d, *args) == flare.FLARE_ERR_UNSUPPORTED
     d.block_len = 4
     d.chunk_len = 32
