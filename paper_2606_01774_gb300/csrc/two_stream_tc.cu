@@ -228,19 +228,15 @@ __global__ void __launch_bounds__(kTcThreads, B <= 4 ? 2 : 1)
     __syncthreads();
     if (tid == 0) {
       tc::fence_after_sync();
-      // the previous block's update is in S~ before S~ is read again
-      if (m > 0 && !tc::mbar_wait(&bar_upd, (uint32_t)(m - 1) & 1u, &abort_flag)) {
-        abort_flag = 1;
-        flag(p.dev_status, FLARE_DEV_WAIT_TIMEOUT);
-      } else {
+      // MMAs issued by one thread execute in issue order: this product reads
+      // S~ after the previous block's update has written it
 #pragma unroll
-        for (int kk = 0; kk < DK / 8; ++kk) {
-          const uint64_t b = tc::sdesc_sw128(
-              tc::smem_u32(Xs + (kk >> 2) * (N1 * 128) + (kk & 3) * 32), 16, 1024);
-          tc::mma_tf32_ts(tmY, tmS + kk * 8, b, id_p1, kk > 0);
-        }
-        tc::mma_commit(&bar_p1);
+      for (int kk = 0; kk < DK / 8; ++kk) {
+        const uint64_t b = tc::sdesc_sw128(
+            tc::smem_u32(Xs + (kk >> 2) * (N1 * 128) + (kk & 3) * 32), 16, 1024);
+        tc::mma_tf32_ts(tmY, tmS + kk * 8, b, id_p1, kk > 0);
       }
+      tc::mma_commit(&bar_p1);
     }
     if (!tc2_wait(&bar_p1, (uint32_t)m & 1u, &abort_flag, p.dev_status)) break;
     tc::fence_after_sync();
@@ -251,7 +247,8 @@ __global__ void __launch_bounds__(kTcThreads, B <= 4 ? 2 : 1)
       tc::tmem_ld16(tmY + lane_off + q * 16, *reinterpret_cast<uint32_t(*)[16]>(&y[q * 16]));
     tc::tmem_ld_wait();
     // the block's keys transposed, the update's B operand (row i, element t);
-    // the previous update has completed (the product above followed it)
+    // the previous update has completed (the product above followed it in
+    // issue order), so its operands may be overwritten
     for (int e = tid; e < 128 * B; e += kTcThreads) {
       const int i = e / B, t = e % B;
       const float kv = __bfloat162float(ck[(t0 + t) * DK + i]);
