@@ -1,6 +1,8 @@
 // Two-stream training forward of a gated-delta-rule layer, noisy stream
 // (appendix "Two-stream recurrence and block-level chain rule",
-// Eq. noisy-block-fwd; the Route II fused forward).
+// Eq. noisy-block-fwd; the Route II fused forward), CUDA-core form in exact
+// fp32.  It serves fp32 activations; bf16 activations (d_k = d_v = 128) take
+// the tensor-core kernel in two_stream_tc.cu.
 //
 // One CTA per (sequence, value head, chunk of 64 tokens).  The clean state
 // S_[c] at the chunk start (from the clean chunkwise pass) is loaded into
