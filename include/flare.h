@@ -334,7 +334,9 @@ flare_status flare_short_conv(const flare_conv_desc* desc, const void* x, void* 
  * advanced over the clean tokens of the chunk's earlier blocks (f_blk), on
  * chip; no block-boundary state is written.  The clean outputs are the clean
  * chunkwise pass's and are not formed here.  Value head j reads q/k head
- * j / (Hv / Hk).
+ * j / (Hv / Hk).  Arithmetic: bf16 activations run the state's products and
+ * updates as tf32 tensor-core products with fp32 accumulation (the state
+ * itself stays fp32); fp32 activations run exact fp32.
  *   chunk_states  [N, Hv, L/C, dk, dv]   fp32
  *   k, v          [N, L, Hk, dk], [N, L, Hv, dv]   clean, act_dtype
  *   log_decay, beta [N, L, Hv]           clean, fp32
