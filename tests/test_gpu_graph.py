@@ -1,7 +1,8 @@
 """The library's compute calls are graph-capturable (no allocation, no host
 synchronization, every launch on the caller's stream): a whole denoise step
-and commit, and a whole AR-Trust verify round, captured once into a CUDA graph
-and replayed give the same bits as the same calls issued one by one."""
+and commit, a whole AR-Trust verify round, the two-stream training forward and
+a ShortConv denoise + commit, captured once into a CUDA graph and replayed,
+give the same bits as the same calls issued one by one."""
 import math
 
 import pytest
@@ -88,4 +89,77 @@ def test_step_replays_bit_identically_from_a_graph(name):
         torch.cuda.synchronize()
         for a, r in zip(outs + [w.state_pool], ref):
             assert torch.equal(a.view(torch.uint8), r.view(torch.uint8))
+    assert flare.flare_read_status(st) == (flare.FLARE_OK, 0)
+
+
+def _replays_like_eager(run, outs, states=()):
+    """Issues `run` once eagerly, then captures it into a CUDA graph and
+    replays it twice from the same starting states: the outputs and states
+    must come back bit for bit."""
+    starts = [s.clone() for s in states]
+    run()
+    torch.cuda.synchronize()
+    ref = [t.clone() for t in list(outs) + list(states)]
+    for s, s0 in zip(states, starts):
+        s.copy_(s0)
+    side = torch.cuda.Stream()
+    with torch.cuda.stream(side):
+        g = torch.cuda.CUDAGraph()
+        launches0 = flare.flare_launch_count()
+        with torch.cuda.graph(g, stream=side):
+            run()
+        captured = flare.flare_launch_count() - launches0
+    torch.cuda.synchronize()
+    assert captured >= 1
+    for _ in range(2):
+        for s, s0 in zip(states, starts):
+            s.copy_(s0)
+        for o in outs:
+            o.zero_()
+        g.replay()
+        torch.cuda.synchronize()
+        for a, r in zip(list(outs) + list(states), ref):
+            assert torch.equal(a.view(torch.uint8), r.view(torch.uint8))
+
+
+def test_two_stream_replays_bit_identically_from_a_graph():
+    sp = workloads.TWO_STREAM_WORKLOADS["two_stream_train_b4"].replace(
+        num_seqs=1, seq_len=256, num_qk_heads=2, num_v_heads=4, seed=31)
+    x = workloads.generate_two_stream(sp, "cuda")
+    gen_ = torch.Generator(device="cuda")
+    gen_.manual_seed(5)
+    cs = 0.05 * torch.randn(sp.num_seqs, sp.num_v_heads, sp.seq_len // sp.chunk_len, 128, 128,
+                            generator=gen_, device="cuda")
+    d = flare.two_stream_desc(sp.num_seqs, sp.seq_len, sp.chunk_len, sp.block_len,
+                              sp.num_qk_heads, sp.num_v_heads, 128, 128, flare.FLARE_DT_BF16,
+                              1.0 / math.sqrt(128))
+    out = torch.empty_like(x.noisy.v)
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    c, nz = x.clean, x.noisy
+
+    def run():
+        flare.check(flare.flare_two_stream_fwd(d, cs, c.k, c.v, c.log_decay, c.beta, nz.q, nz.k,
+                                               nz.v, nz.log_decay, nz.beta, out, st))
+
+    _replays_like_eager(run, [out])
+    assert flare.flare_read_status(st) == (flare.FLARE_OK, 0)
+
+
+def test_shortconv_denoise_and_commit_replay_bit_identically_from_a_graph():
+    spec = W["shortconv_serving_batch64"].replace(num_requests=6, prefix_lo=64, prefix_hi=128)
+    w = gen(spec)
+    act = flare.FLARE_DT_BF16
+    d = flare.conv_desc(spec.num_requests, spec.block_len, spec.conv_channels, spec.conv_width,
+                        w.conv_state.shape[0], act, flare.FLARE_ACT_SILU)
+    x0, x1 = w.conv_x[0], w.conv_commit_x
+    out0, out1 = torch.empty_like(x0), torch.empty_like(x1)
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+
+    def run():
+        flare.check(flare.flare_short_conv(d, x0, w.conv_state, w.state_slot, w.conv_weight,
+                                           w.conv_bias, None, out0, st))
+        flare.check(flare.flare_short_conv(d, x1, w.conv_state, w.state_slot, w.conv_weight,
+                                           w.conv_bias, w.accept_len, out1, st))
+
+    _replays_like_eager(run, [out0, out1], [w.conv_state])
     assert flare.flare_read_status(st) == (flare.FLARE_OK, 0)
