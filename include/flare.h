@@ -464,6 +464,15 @@ flare_status flare_debug_gather_prefix(const flare_softmax_desc* desc, const voi
                                        void* v_out, int32_t* dev_status, void* stream);
 
 /*
+ * Test helper for failure detection: one CTA waits on a pipeline barrier that
+ * nothing ever completes, through the bounded wait every pipelined kernel
+ * uses, gives up after limit_ns nanoseconds (1 us .. 1 s; else
+ * FLARE_ERR_INVALID_ARGUMENT) and sets FLARE_DEV_WAIT_TIMEOUT in dev_status.
+ * The context stays usable afterwards.
+ */
+flare_status flare_debug_wait_timeout(int32_t* dev_status, uint64_t limit_ns, void* stream);
+
+/*
  * Waits for `stream`, copies the status word to *bits_out (nullable) and
  * returns FLARE_ERR_DEVICE_STATUS if any bit is set, FLARE_ERR_CUDA if the
  * stream reported an error, else FLARE_OK.  This is the one call that

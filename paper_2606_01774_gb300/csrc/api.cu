@@ -529,6 +529,14 @@ flare_status flare_debug_gather_prefix(const flare_softmax_desc* d, const void* 
   return e == cudaSuccess ? FLARE_OK : FLARE_ERR_CUDA;
 }
 
+flare_status flare_debug_wait_timeout(int32_t* dev_status, uint64_t limit_ns, void* stream) {
+  if (!dev_status || limit_ns < 1000ull || limit_ns > 1000000000ull)
+    return FLARE_ERR_INVALID_ARGUMENT;
+  const cudaError_t e =
+      launch_debug_wait_timeout(dev_status, limit_ns, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? FLARE_OK : FLARE_ERR_CUDA;
+}
+
 uint64_t flare_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
 flare_status flare_read_status(const int32_t* dev_status, void* stream, int32_t* bits_out) {

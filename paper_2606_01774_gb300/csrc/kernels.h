@@ -136,6 +136,7 @@ cudaError_t launch_softmax_combine(const SoftmaxParams& p, bool bf16, cudaStream
 bool softmax_tc_supported(int B, int Hq, int Hkv, int D, int page_size);
 cudaError_t launch_append_kv(const SoftmaxParams& p, const int32_t* append_len, void* k_pool,
                              void* v_pool, int elem_bytes, cudaStream_t stream);
+cudaError_t launch_debug_wait_timeout(int32_t* status, uint64_t limit_ns, cudaStream_t stream);
 cudaError_t launch_gather_prefix(const SoftmaxParams& p, int request, void* k_out, void* v_out,
                                  bool bf16, cudaStream_t stream);
 

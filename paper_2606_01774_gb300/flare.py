@@ -109,6 +109,7 @@ def load() -> ctypes.CDLL:
         "flare_block_softmax_attn_noalloc": [smx] + [P] * 11,
         "flare_append_kv": [smx] + [P] * 9,
         "flare_debug_gather_prefix": [smx, P, P, P, P, I32, P, P, P, P],
+        "flare_debug_wait_timeout": [P, ctypes.c_uint64, P],
         "flare_read_status": [P, P, ctypes.POINTER(I32)],
     }
     for name, args in sigs.items():
@@ -243,6 +244,10 @@ def flare_debug_gather_prefix(desc, k_pool, v_pool, page_table, prefix_len, requ
     return load().flare_debug_gather_prefix(
         ctypes.byref(desc), _p(k_pool), _p(v_pool), _p(page_table), _p(prefix_len),
         int(request), _p(k_out), _p(v_out), _p(dev_status), _stream(stream))
+
+
+def flare_debug_wait_timeout(dev_status, limit_ns, stream=None) -> int:
+    return load().flare_debug_wait_timeout(_p(dev_status), int(limit_ns), _stream(stream))
 
 
 def flare_read_status(dev_status, stream=None):

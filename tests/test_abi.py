@@ -53,6 +53,14 @@ def test_host_argument_checks_need_no_gpu(lib):
     assert lib.flare_softmax_workspace_size(ctypes.byref(s), ctypes.byref(n)) == \
         flare.FLARE_ERR_UNSUPPORTED
     assert lib.flare_read_status(None, None, None) == flare.FLARE_ERR_INVALID_ARGUMENT
+    # the bounded-wait test entry rejects a missing status word and limits
+    # outside 1 us .. 1 s before launching anything
+    word = ctypes.c_int32(0)
+    assert lib.flare_debug_wait_timeout(None, 1_000_000, None) == flare.FLARE_ERR_INVALID_ARGUMENT
+    assert lib.flare_debug_wait_timeout(ctypes.byref(word), 999, None) == \
+        flare.FLARE_ERR_INVALID_ARGUMENT
+    assert lib.flare_debug_wait_timeout(ctypes.byref(word), 2_000_000_000, None) == \
+        flare.FLARE_ERR_INVALID_ARGUMENT
 
 
 def test_workspace_query_is_host_only(lib):

@@ -17,6 +17,34 @@ def _st():
     return torch.zeros(1, dtype=torch.int32, device="cuda")
 
 
+def test_bounded_wait_gives_up_and_reports():
+    """A pipeline wait on a barrier that nothing ever completes gives up after
+    its limit (the same bounded wait every pipelined kernel uses) and reports
+    FLARE_DEV_WAIT_TIMEOUT; the context stays usable."""
+    import time
+
+    st = _st()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    flare.check(flare.flare_debug_wait_timeout(st, 20_000_000), "flare_debug_wait_timeout")
+    rc, bits = flare.flare_read_status(st)
+    elapsed = time.perf_counter() - t0
+    assert rc == flare.FLARE_ERR_DEVICE_STATUS and bits == flare.FLARE_DEV_WAIT_TIMEOUT
+    assert elapsed >= 0.02
+    # the context is intact: an ordinary call afterwards runs clean
+    spec = reduced(W["serving_batch64"], 2, 64, 200)
+    w = gen(spec)
+    install_states(w)
+    b = w.denoise[0]
+    out = torch.empty_like(b.v)
+    st2 = _st()
+    flare.check(flare.flare_block_linear_attn(linear_desc(spec, w.state_pool.shape[0]), b.q, b.k,
+                                              b.v, b.log_decay, b.beta, w.state_pool,
+                                              w.state_slot, out, st2), "flare_block_linear_attn")
+    assert flare.flare_read_status(st2) == (flare.FLARE_OK, 0)
+    assert torch.isfinite(out.float()).all()
+
+
 def test_bad_state_slot_sets_bit_and_skips_request():
     spec = reduced(W["small_model_batch256"], 3)
     w = gen(spec)
