@@ -387,7 +387,7 @@ class E2ERunner:
     The copies run on their own streams, as a serving loop would issue them:
     every input goes host->device in the order the step consumes it (the
     request metadata, then each denoise step's linear and softmax inputs, then
-    the commit's), each denoise step waits only for its own inputs, and its
+    the commit's), each layer call waits only for its own inputs, and its
     outputs go device->host as soon as they are written."""
 
     def __init__(self, fr: FlareRunner):
@@ -397,11 +397,13 @@ class E2ERunner:
         meta = (w.page_table, w.prefix_len, w.accept_len, w.state_slot)
         if fr.verify:
             meta = (w.page_table, w.prefix_len, w.state_slot, w.verify_len, w.row_type)
+        # groups in consumption order: the metadata, then per denoise step the
+        # linear layer's inputs and the softmax layer's, then the commit's
         self.groups = [[pin(t) for t in meta]]
         for i, (b, sb) in enumerate(zip(w.denoise, w.softmax)):
             conv_in = (w.conv_x[i],) if fr.conv else ()
-            self.groups.append([pin(t) for t in conv_in + (b.q, b.k, b.v, b.log_decay, b.beta,
-                                                           sb.q, sb.k_blk, sb.v_blk)])
+            self.groups.append([pin(t) for t in conv_in + (b.q, b.k, b.v, b.log_decay, b.beta)])
+            self.groups.append([pin(t) for t in (sb.q, sb.k_blk, sb.v_blk)])
         if fr.verify:  # the accept decision, known once the round's logits are sampled
             self.groups.append([pin(w.verify_accept)])
         else:
@@ -409,10 +411,12 @@ class E2ERunner:
             self.groups.append([pin(t) for t in conv_in + (w.commit.k, w.commit.v,
                                                            w.commit.log_decay, w.commit.beta)])
         hbuf = lambda d: (d, torch.empty(d.shape, dtype=d.dtype, pin_memory=True))  # noqa: E731
-        self.outs = [[hbuf(lo), hbuf(so)] for lo, so in zip(fr.lin_out, fr.sm_out)]
-        if fr.conv:
-            for i, co in enumerate(fr.conv_out):
-                self.outs[i].append(hbuf(co))
+        # per denoise step: the linear layer's outputs (and the ShortConv's),
+        # then the softmax layer's
+        self.outs = []
+        for i, (lo, so) in enumerate(zip(fr.lin_out, fr.sm_out)):
+            self.outs.append([hbuf(lo)] + ([hbuf(fr.conv_out[i])] if fr.conv else []))
+            self.outs.append([hbuf(so)])
         self.h2d_bytes = sum(h.numel() * h.element_size() for g in self.groups for h, _ in g)
         self.d2h_bytes = sum(h.numel() * h.element_size() for g in self.outs for _, h in g)
         self.s_h2d = torch.cuda.Stream()
@@ -428,17 +432,23 @@ class E2ERunner:
                     d.copy_(h, non_blocking=True)
                 ev.record(self.s_h2d)
         cs.wait_event(self.ev_in[0])
+
+        def send_back(k):  # outputs of group k go to the host as soon as written
+            self.ev_out[k].record(cs)
+            with torch.cuda.stream(self.s_d2h):
+                self.s_d2h.wait_event(self.ev_out[k])
+                for d, h in self.outs[k]:
+                    h.copy_(d, non_blocking=True)
+
         for i in range(fr.spec.denoise_steps):
-            cs.wait_event(self.ev_in[i + 1])
+            cs.wait_event(self.ev_in[1 + 2 * i])  # this step's linear inputs
             if fr.conv:
                 fr.shortconv(i)
             fr.linear(i)
+            send_back(2 * i)
+            cs.wait_event(self.ev_in[2 + 2 * i])  # this step's softmax inputs
             fr.softmax(i)
-            self.ev_out[i].record(cs)
-            with torch.cuda.stream(self.s_d2h):
-                self.s_d2h.wait_event(self.ev_out[i])
-                for d, h in self.outs[i]:
-                    h.copy_(d, non_blocking=True)
+            send_back(2 * i + 1)
         cs.wait_event(self.ev_in[-1])
         if fr.conv:
             fr.shortconv(-1)
