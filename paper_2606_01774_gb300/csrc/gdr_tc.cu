@@ -16,18 +16,19 @@
 // independently of the others (the update acts on S from the left), so thread
 // c owns everything about column c from the first MMA to its output.
 //
-//   MMA 1   G   = [K;Q] K^T          M=128 (64 k rows, 64 q rows), N=Bp, K=dk
-//   MMA 2   W^T = S0^T [K;Q]^T       M=128 (c),  N=128, K=dk   (S0^T is MN-major)
+//   MMA 1   G   = [K;Q] K^T          M=128 (BM k rows, BM q rows), N=Bp, K=dk
+//   MMA 2   W^T = S0^T [K;Q]^T       M=128 (c),  N=2BM, K=dk   (S0^T is MN-major)
 //   solve   (I + A) delta = X        unit lower triangular, 16 rows at a time:
 //                                    off-diagonal terms on warp-level tf32 MMA,
 //                                    diagonal blocks by fp32 forward substitution
 //   MMA 4   O2^T = delta^T M2^T      M=128 (c),  N=Bp,  K=Bp, M2[l][i] = exp(gamma_B-gamma_i) q_l.k_i
-//   out[l][c] = s (Gam_B W^T[c][64+l] + O2^T[c][l])
+//   out[l][c] = s (Gam_B W^T[c][BM+l] + O2^T[c][l])
 //
-// Bp = B rounded up to 16.  Inputs bf16, state fp32 read once and rounded to
-// bf16 for the MMA, all accumulation fp32.  One CTA per (request, value
-// head); 128 threads; 107 KiB shared memory and 256 TMEM
-// columns, so two CTAs share an SM.
+// Bp = B rounded up to 16; BM = 32 for B <= 32, else 64 (the K/Q/V tiles hold
+// BM rows).  Inputs bf16, state fp32 read once and rounded to bf16 for the
+// MMA, all accumulation fp32.  One CTA per (request, value head), 128
+// threads: BM = 64 takes 106 KiB of shared memory and 256 TMEM columns (two
+// CTAs per SM), BM = 32 73 KiB and 128 columns (three CTAs per SM).
 #include <cudaTypedefs.h>
 
 #include "common.cuh"
