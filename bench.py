@@ -647,24 +647,24 @@ def run_two_stream(args, spec, rank, world, local_rank):
 
 
 def two_stream_oracle_rate(spec, seed_offset=0):
-    """The fp64 oracle on one head of the same sequence (heads are
-    independent), scaled by the head count."""
+    """The fp64 oracle on the whole training sequence (every head), drawn on
+    the host with the same recipe, wall-timed."""
     import oracle
 
     oracle.build()
-    sub = spec.replace(num_qk_heads=1, num_v_heads=1, seed=spec.seed + seed_offset)
+    sub = spec.replace(seed=spec.seed + seed_offset)
     x = workloads.generate_two_stream(sub, "cpu")
     c, n = x.clean, x.noisy
     t0 = time.perf_counter()
     res = oracle.two_stream_fwd((c.k, c.v, c.log_decay, c.beta),
                                 (n.q, n.k, n.v, n.log_decay, n.beta), x.S_init, sub.block_len,
                                 sub.chunk_len)
-    secs = (time.perf_counter() - t0) * spec.num_v_heads
+    secs = time.perf_counter() - t0
     assert np.isfinite(res["out"]).all()
     tokens = 2 * spec.num_seqs * spec.seq_len
-    desc = (f"one head of {spec.name} ({spec.seq_len} clean + {spec.seq_len} noisy tokens, "
-            f"drawn on the host with the same recipe), timed and scaled by the "
-            f"{spec.num_v_heads} heads")
+    desc = (f"{spec.name} ({spec.seq_len} clean + {spec.seq_len} noisy tokens, "
+            f"{spec.num_v_heads} heads, drawn on the host with the same recipe), wall time "
+            f"measured; the oracle's loop runs over (sequence, head) items")
     return tokens / secs, secs, oracle.max_threads(), desc
 
 
@@ -688,68 +688,38 @@ def _elapsed_pairs(evs):
     return [evs[i].elapsed_time(evs[i + 1]) for i in range(0, len(evs), 2)]
 
 
-def run_flare(args, spec, rank, world, local_rank):
-    device = torch.device("cuda", local_rank)
-    torch.cuda.set_device(device)
-    from paper_2606_01774_gb300 import flare
+SUSTAINED_AFTER_S = 2.0  # timed regions at least this long use the sustained tensor peak
 
-    flare.load()
-    fr = FlareRunner(spec, device, seed_offset=rank_seed_offset(rank))
-    dist = world > 1
-    if dist:
-        import torch.distributed as tdist
 
-    for _ in range(args.warmup):
+def tensor_peak(peaks, timed_s):
+    """The measured bf16 peak that applies to a kernel timed inside a region of
+    timed_s seconds: the burst figure for short regions, the sustained
+    (power-capped) one for regions of seconds."""
+    key = "bf16_tflops_sustained" if timed_s >= SUSTAINED_AFTER_S else "bf16_tflops"
+    return peaks[key], key
+
+
+def _warm_up(fr, warmup, clocks_rank0=False):
+    """Untimed warm-up steps; returns the per-call event lists to fill and the
+    clock sampler (rank 0) started just before the timed region."""
+    flare = fr.flare
+    for _ in range(warmup):
         fr.step()
     torch.cuda.synchronize()
     st, bits = flare.flare_read_status(fr.status)
     if st != flare.FLARE_OK:
         raise RuntimeError(f"device status {bits:#x} after warm-up")
-
     events = {"linear": [], "softmax": [], "commit": []}
     if fr.conv:
         events.update(shortconv=[], shortconv_commit=[])
-    clocks = ClockSampler(torch.cuda.current_device()) if rank == 0 else None
-    if dist:
-        tdist.barrier()
-    torch.cuda.synchronize()
-    launches0 = flare.flare_launch_count()
-    t0 = torch.cuda.Event(enable_timing=True)
-    t1 = torch.cuda.Event(enable_timing=True)
-    t0.record()
-    for _ in range(args.steps):
-        fr.step(events)
-    t1.record()
-    torch.cuda.synchronize()
-    launches = flare.flare_launch_count() - launches0
-    if dist:
-        tdist.barrier()
-    clk = clocks.stop() if clocks else None
-    ms = max_over_ranks(t0.elapsed_time(t1), dist, device)
-    ms_step = ms / args.steps
+    clocks = ClockSampler(torch.cuda.current_device()) if clocks_rank0 else None
+    return events, clocks
 
-    # end-to-end through host buffers
-    e2e, e2e_ms = None, None
-    if not args.no_e2e:
-        e2e = E2ERunner(fr)
-        for _ in range(max(1, min(args.warmup, 2))):
-            e2e.step()
-        if dist:
-            tdist.barrier()
-        t_e = time.perf_counter()
-        for _ in range(args.steps):
-            e2e.step()
-        e2e_ms = max_over_ranks((time.perf_counter() - t_e) * 1e3 / args.steps, dist, device)
-    st, bits = flare.flare_read_status(fr.status)
-    if st != flare.FLARE_OK:
-        raise RuntimeError(f"device status {bits:#x} after timing")
 
-    if rank != 0:
-        return None
+def summarise(fr, per, timed_s, clk):
+    """Algorithmic bytes and flops of each call, the step's achieved HBM
+    bandwidth and the roofline of the dominant kernel."""
     s = fr.spec
-    tokens = s.num_requests * s.block_len * s.denoise_steps
-    value = world * tokens / (ms_step / 1e3)
-    per = {k: float(np.mean(_elapsed_pairs(v))) for k, v in events.items()}
     prefix_sum = int(fr.w.prefix_len.sum().item())
     acc = fr.w.accept_len.cpu().numpy()
     peaks = load_peaks()
@@ -774,8 +744,9 @@ def run_flare(args, spec, rank, world, local_rank):
     dom = max(share, key=share.get)
     kd = kern[dom]
     dur_s = per[dom] / 1e3
+    tc_peak, tc_key = tensor_peak(peaks, timed_s)
     t_hbm = kd["bytes"] / (peaks["hbm_gbs"] * 1e9)
-    t_tc = kd["flops"] / (peaks["bf16_tflops_sustained"] * 1e12)
+    t_tc = kd["flops"] / (tc_peak * 1e12)
     if kd.get("fp32_alu"):
         # CUDA-core fp32: 152 SMs x 128 lanes x 2 flops x the median SM clock
         mhz = (clk or {}).get("sm_mhz") or 1920.0
@@ -784,31 +755,131 @@ def run_flare(args, spec, rank, world, local_rank):
     if kd.get("fp32_alu") and t_tc > t_hbm:
         roof = {"bound": "alu", "achieved": kd["flops"] / dur_s / 1e12, "peak": alu_peak,
                 "unit": "TFLOP/s"}
+        peak_source = "fp32 CUDA-core count x median SM clock"
     elif t_tc > t_hbm:
-        roof = {"bound": "tensor", "achieved": kd["flops"] / dur_s / 1e12,
-                "peak": peaks["bf16_tflops_sustained"], "unit": "TFLOP/s"}
+        roof = {"bound": "tensor", "achieved": kd["flops"] / dur_s / 1e12, "peak": tc_peak,
+                "unit": "TFLOP/s"}
+        peak_source = f"{peaks['source']} ({tc_key}; timed region {timed_s:.2f} s)"
     else:
         roof = {"bound": "hbm", "achieved": kd["bytes"] / dur_s / 1e9,
                 "peak": peaks["hbm_gbs"], "unit": "GB/s"}
+        peak_source = f"{peaks['source']} (hbm_gbs)"
     roof["frac"] = roof["achieved"] / roof["peak"]
     kernel_of = VERIFY_KERNEL_OF if fr.verify else KERNEL_OF
     roof["traffic"] = profiled_traffic(kernel_of[dom], s.name) if dom in kernel_of else None
     roof["kernel"] = kd["kernel"]
-    roof["peak_source"] = (
-        "fp32 CUDA-core count x median SM clock" if roof["bound"] == "alu" else
-        f"{peaks['source']} ({'bf16_tflops_sustained' if roof['unit'] == 'TFLOP/s' else 'hbm_gbs'})")
+    roof["peak_source"] = peak_source
     roof["algorithmic_per_launch"] = kd["flops"] if roof["bound"] == "tensor" else kd["bytes"]
     step_bytes = sum(kd_["bytes"] * (1 if k in once else s.denoise_steps)
                      for k, kd_ in kern.items())
+    per_call_gbs = {k: kern[k]["bytes"] / (per[k] / 1e3) / 1e9 for k in per}
+    return kern, roof, step_bytes, per_call_gbs
+
+
+def run_steps(fr, steps, warmup, dist=False, device=None, clocks_rank0=False):
+    """Times `steps` steps of a FlareRunner; returns (per-call mean ms, total
+    ms, launches, clock record)."""
+    flare = fr.flare
+    events, clocks = _warm_up(fr, warmup, clocks_rank0)
+    if dist:
+        import torch.distributed as tdist
+
+        tdist.barrier()
+    torch.cuda.synchronize()
+    launches0 = flare.flare_launch_count()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for _ in range(steps):
+        fr.step(events)
+    t1.record()
+    torch.cuda.synchronize()
+    launches = flare.flare_launch_count() - launches0
+    if dist:
+        tdist.barrier()
+    clk = clocks.stop() if clocks else None
+    ms = max_over_ranks(t0.elapsed_time(t1), dist, device)
+    per = {k: float(np.mean(_elapsed_pairs(v))) for k, v in events.items()}
+    return per, ms, launches, clk
+
+
+PER_CONFIG_WORKLOADS = ("serving_batch64", "small_model_batch256")
+
+
+def run_per_config(steps, warmup, device, names=PER_CONFIG_WORKLOADS):
+    """The other batched workloads, timed in the same process after the
+    headline one: ms per step, per-call ms and GB/s, the step's achieved HBM
+    bandwidth and the dominant kernel's roofline."""
+    out = {}
+    for name in names:
+        fr = FlareRunner(workloads.WORKLOADS[name], device)
+        per, ms, launches, _ = run_steps(fr, steps, warmup)
+        ms_step = ms / steps
+        kern, roof, step_bytes, gbs = summarise(fr, per, ms / 1e3, None)
+        s = fr.spec
+        peaks = load_peaks()
+        st, bits = fr.flare.flare_read_status(fr.status)
+        if st != fr.flare.FLARE_OK:
+            raise RuntimeError(f"{name}: device status {bits:#x}")
+        out[name] = {
+            "value": s.num_requests * s.block_len * s.denoise_steps / (ms_step / 1e3),
+            "unit": UNIT, "ms_per_step": ms_step, "steps": steps,
+            "achieved_hbm_gbs": step_bytes / (ms_step / 1e3) / 1e9,
+            "step_hbm_frac": step_bytes / (ms_step / 1e3) / 1e9 / peaks["hbm_gbs"],
+            "step_bytes": step_bytes, "per_call_ms": per, "per_call_gbs": gbs,
+            "per_call_hbm_frac": {k: v / peaks["hbm_gbs"] for k, v in gbs.items()},
+            "roofline": roof, "gpu_launches": int(launches),
+        }
+        del fr
+        torch.cuda.synchronize()
+        torch.cuda.empty_cache()
+    return out
+
+
+def run_flare(args, spec, rank, world, local_rank):
+    device = torch.device("cuda", local_rank)
+    torch.cuda.set_device(device)
+    from paper_2606_01774_gb300 import flare
+
+    flare.load()
+    fr = FlareRunner(spec, device, seed_offset=rank_seed_offset(rank))
+    dist = world > 1
+    if dist:
+        import torch.distributed as tdist
+
+    per, ms, launches, clk = run_steps(fr, args.steps, args.warmup, dist, device,
+                                       clocks_rank0=rank == 0)
+    ms_step = ms / args.steps
+
+    # end-to-end through host buffers
+    e2e, e2e_ms = None, None
+    if not args.no_e2e:
+        e2e = E2ERunner(fr)
+        for _ in range(max(1, min(args.warmup, 2))):
+            e2e.step()
+        if dist:
+            tdist.barrier()
+        t_e = time.perf_counter()
+        for _ in range(args.steps):
+            e2e.step()
+        e2e_ms = max_over_ranks((time.perf_counter() - t_e) * 1e3 / args.steps, dist, device)
+    st, bits = flare.flare_read_status(fr.status)
+    if st != flare.FLARE_OK:
+        raise RuntimeError(f"device status {bits:#x} after timing")
+
+    if rank != 0:
+        return None
+    s = fr.spec
+    tokens = s.num_requests * s.block_len * s.denoise_steps
+    value = world * tokens / (ms_step / 1e3)
+    kern, roof, step_bytes, per_call_gbs = summarise(fr, per, ms / 1e3, clk)
     s_extra = {}
     if fr.verify:
         s_extra = {"verify_horizon": s.verify_horizon,
                    "verify_len_mean": float(fr.w.verify_len.float().mean())}
     if fr.conv:
         s_extra = {"shortconv": {"width": s.conv_width, "channels": s.conv_channels,
-                                 "activation": "silu"},
-                   "per_call_gbs": {k: kern[k]["bytes"] / (per[k] / 1e3) / 1e9
-                                    for k in ("shortconv", "shortconv_commit")}}
+                                 "activation": "silu"}}
     line = {
         "metric": METRIC if not fr.verify else VERIFY_METRIC, "value": value, "unit": UNIT,
         "n_gpus": world, "steps": args.steps,
@@ -823,6 +894,7 @@ def run_flare(args, spec, rank, world, local_rank):
                    **s_extra},
         "achieved_hbm_gbs": step_bytes / (ms_step / 1e3) / 1e9,
         "per_call_ms": per,
+        "per_call_gbs": per_call_gbs,
         "roofline": roof,
         "e2e": None if e2e is None else {
             "value": world * tokens / (e2e_ms / 1e3), "unit": UNIT, "ms_per_step": e2e_ms,
@@ -830,94 +902,74 @@ def run_flare(args, spec, rank, world, local_rank):
         "gpu_launches": int(launches),
         "clocks": clk,
     }
+    if world == 1 and not args.no_per_config and s.name == DEFAULT_WORKLOAD:
+        del e2e
+        del fr
+        torch.cuda.empty_cache()
+        line["per_config"] = run_per_config(args.steps, args.warmup, device)
     return line
 
 
 # ---------------------------------------------------------------- oracle (CPU) arm
 
 
-def oracle_sample_rate(spec, n_requests, seed_offset=0, one_head=False):
+def oracle_sample_rate(spec, n_requests, seed_offset=0):
     """Times the fp64 oracle on a bounded sample of the workload (drawn on the
-    host with the same recipe): the first n_requests, one denoise step (linear
-    + softmax) and the commit.  With one_head, only q head 0 (and its kv head)
-    and v head 0 (and its q/k head) are computed and the time is scaled by the
-    head counts, heads being independent.  Returns (block-tokens/s, seconds
-    per bench step, threads, sample description)."""
+    host with the same recipe): the first n_requests with every head, the
+    workload's whole step for them (each denoise step's linear and softmax
+    layer calls, with the ShortConv where the workload has one, then the
+    commit), timed end to end with the wall clock.  Returns (block-tokens/s,
+    measured seconds, threads, sample description)."""
     import oracle
 
     oracle.build()
-    sub = spec.replace(num_requests=n_requests, denoise_steps=1, seed=spec.seed + seed_offset)
+    sub = spec.replace(num_requests=n_requests, seed=spec.seed + seed_offset)
     w = workloads.generate(sub, "cpu")
     R, Hv, dk, dv = sub.num_requests, sub.num_v_heads, sub.head_dim_k, sub.head_dim_v
-    b, c, sb, sp = w.denoise[0], w.commit, w.softmax[0], w.state_prefix
-    hv = slice(0, 1) if one_head else slice(0, Hv)
-    hk = slice(0, 1) if one_head else slice(0, sub.num_qk_heads)
-    hq = slice(0, 1) if one_head else slice(0, sub.num_q_heads)
-    hkv = slice(0, 1) if one_head else slice(0, sub.num_kv_heads)
-    nv = hv.stop - hv.start
-    S0 = oracle.gdr_per_token(None, sp.k[:, :, hk], sp.v[:, :, hv], sp.log_decay[:, :, hv],
-                              sp.beta[:, :, hv], np.zeros((1, nv, dk, dv), np.float32),
+    c, sp = w.commit, w.state_prefix
+    S0 = oracle.gdr_per_token(None, sp.k, sp.v, sp.log_decay, sp.beta,
+                              np.zeros((1, Hv, dk, dv), np.float32),
                               np.zeros(R, np.int32), None, blockend=False)["state"]
     pool = S0.astype(np.float32)
     slots = np.arange(R, dtype=np.int32)
-    kp, vp = w.k_pool[:, hkv], w.v_pool[:, hkv]
+    scale = 1.0 / math.sqrt(sub.head_dim)
+    t0 = time.perf_counter()
     if spec.verify_horizon:
         # AR-Trust verify round: verify pass, per-row-type softmax, commit
         mv = spec.verify_horizon - 1
-        t0 = time.perf_counter()
-        o = oracle.gdr_verify(b.q[:, :, hk], b.k[:, :, hk], b.v[:, :, hv], b.log_decay[:, :, hv],
-                              b.beta[:, :, hv], pool, slots, w.verify_len, mv)
-        t1 = time.perf_counter()
-        oracle.block_softmax(sb.q[:, :, hq], sb.k_blk[:, :, hkv], sb.v_blk[:, :, hkv], kp, vp,
-                             w.page_table, w.prefix_len, scale=1.0 / math.sqrt(sub.head_dim),
-                             mask_mode=3, row_type=w.row_type)
-        t2 = time.perf_counter()
+        b, sb = w.denoise[0], w.softmax[0]
+        o = oracle.gdr_verify(b.q, b.k, b.v, b.log_decay, b.beta, pool, slots, w.verify_len, mv)
+        oracle.block_softmax(sb.q, sb.k_blk, sb.v_blk, w.k_pool, w.v_pool, w.page_table,
+                             w.prefix_len, scale=scale, mask_mode=3, row_type=w.row_type)
         live = pool.astype(np.float64)
         live[slots] = o["state"]
         oracle.verify_commit([o["records"]], [live], slots, w.verify_accept, w.verify_len)
-        t3 = time.perf_counter()
     else:
-        t0 = time.perf_counter()
-        oracle.gdr_per_token(b.q[:, :, hk], b.k[:, :, hk], b.v[:, :, hv], b.log_decay[:, :, hv],
-                             b.beta[:, :, hv], pool, slots, None, state=False)
-        t1 = time.perf_counter()
-        oracle.block_softmax(sb.q[:, :, hq], sb.k_blk[:, :, hkv], sb.v_blk[:, :, hkv], kp, vp,
-                             w.page_table, w.prefix_len, scale=1.0 / math.sqrt(sub.head_dim))
-        t2 = time.perf_counter()
-        oracle.gdr_per_token(None, c.k[:, :, hk], c.v[:, :, hv], c.log_decay[:, :, hv],
-                             c.beta[:, :, hv], pool, slots, w.accept_len, blockend=False)
-        t3 = time.perf_counter()
-    f_v = sub.num_v_heads if one_head else 1
-    f_q = sub.num_q_heads if one_head else 1
-    step_s = spec.denoise_steps * ((t1 - t0) * f_v + (t2 - t1) * f_q) + (t3 - t2) * f_v
-    if spec.conv_width:
-        # the ShortConv of one denoise block and of the committed block; with
-        # one_head, the channels of one v head's share (C / Hv), scaled back
-        C = sub.conv_channels
-        cs = slice(0, C // sub.num_v_heads) if one_head else slice(0, C)
-        f_c = sub.num_v_heads if one_head else 1
-        cpool = w.conv_state[:, :, cs]
-        t4 = time.perf_counter()
-        oracle.short_conv(w.conv_x[0][:, :, cs], cpool, slots_conv(w), w.conv_weight[cs],
-                          w.conv_bias[cs])
-        t5 = time.perf_counter()
-        oracle.short_conv(w.conv_commit_x[:, :, cs], cpool, slots_conv(w), w.conv_weight[cs],
-                          w.conv_bias[cs], accept_len=w.accept_len)
-        t6 = time.perf_counter()
-        step_s += (spec.denoise_steps * (t5 - t4) + (t6 - t5)) * f_c
+        for i in range(sub.denoise_steps):
+            b, sb = w.denoise[i], w.softmax[i]
+            if spec.conv_width:
+                oracle.short_conv(w.conv_x[i], w.conv_state, slots_conv(w), w.conv_weight,
+                                  w.conv_bias)
+            oracle.gdr_per_token(b.q, b.k, b.v, b.log_decay, b.beta, pool, slots, None,
+                                 state=False)
+            oracle.block_softmax(sb.q, sb.k_blk, sb.v_blk, w.k_pool, w.v_pool, w.page_table,
+                                 w.prefix_len, scale=scale)
+        if spec.conv_width:
+            oracle.short_conv(w.conv_commit_x, w.conv_state, slots_conv(w), w.conv_weight,
+                              w.conv_bias, accept_len=w.accept_len)
+        oracle.gdr_per_token(None, c.k, c.v, c.log_decay, c.beta, pool, slots, w.accept_len,
+                             blockend=False)
+    secs = time.perf_counter() - t0
     tokens = R * spec.block_len * spec.denoise_steps
-    heads = ("q head 0 and v head 0 timed, scaled by the head counts "
-             f"({sub.num_q_heads} q, {sub.num_v_heads} v)" if one_head else "all heads")
-    if spec.verify_horizon:
-        desc = (f"{R} request(s) of {spec.name} drawn on the host with the same recipe "
-                f"(prefix {int(w.prefix_len.sum())} tokens, K = "
-                f"{[int(x) for x in w.verify_len]}), {heads}: the verify pass, the softmax "
-                f"with per-row types and the commit")
-    else:
-        desc = (f"{R} request(s) of {spec.name} drawn on the host with the same recipe "
-                f"(prefix {int(w.prefix_len.sum())} tokens), {heads}: one denoise step "
-                f"(linear + softmax) timed and counted {spec.denoise_steps}x, plus the commit")
-    return tokens / step_s, step_s, oracle.max_threads(), desc
+    what = ("the verify pass, the softmax with per-row types and the commit"
+            if spec.verify_horizon else
+            f"{spec.denoise_steps} denoise step(s) (linear + softmax"
+            + (" + ShortConv" if spec.conv_width else "") + ") and the commit")
+    desc = (f"{R} request(s) of {spec.name} drawn on the host with the same recipe "
+            f"(prefix {int(w.prefix_len.sum())} tokens), all heads: {what}, wall time "
+            f"measured; the oracle's loops run over (request, head) and (request, head, row) "
+            f"items, at least {R * min(Hv, sub.num_q_heads * sub.block_len)} per call")
+    return tokens / secs, secs, oracle.max_threads(), desc
 
 
 def slots_conv(w):
@@ -925,22 +977,27 @@ def slots_conv(w):
 
 
 def run_reference(args, spec):
+    """The oracle arm: every step is one request of the workload (a fresh
+    seeded draw per step), its whole step on the host cores, wall-timed."""
     secs = []
-    threads, desc = None, None
+    threads, desc, prefix = None, None, []
     for i in range(args.warmup + args.steps):
-        _, s, threads, desc = oracle_sample_rate(spec, 1, seed_offset=i, one_head=True)
+        _, sec, threads, desc = oracle_sample_rate(spec, 1, seed_offset=i)
         if i >= args.warmup:
-            secs.append(s)
-    value = len(secs) * spec.block_len * spec.denoise_steps / sum(secs)
+            secs.append(sec)
+    tokens = spec.block_len * spec.denoise_steps
+    value = len(secs) * tokens / sum(secs)
     return {
         "impl": "reference", "metric": METRIC if not spec.verify_horizon else VERIFY_METRIC,
         "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * float(np.mean(secs)),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic",
-        "config": {"workload": spec.name, "requests_per_step": 1, "parallelism": "host cores"},
+        "config": {"workload": spec.name, "requests_per_step": 1,
+                   "block_tokens_per_step": tokens, "parallelism": "host cores"},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
-                         "sample": "each step: " + desc},
+                         "sample": "each step: " + desc,
+                         "seconds_timed": float(sum(secs))},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
 
@@ -957,6 +1014,8 @@ def main():
     ap.add_argument("--no-e2e", action="store_true",
                     help="skip the host-buffer end-to-end measurement (profiling runs)")
     ap.add_argument("--cpu-sample-requests", type=int, default=2)
+    ap.add_argument("--no-per-config", action="store_true",
+                    help="skip timing the other batched workloads after the headline one")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "flare":
         ap.error("--warmup must be >= 3")
@@ -1000,7 +1059,8 @@ def main():
             if world == 1 and not args.no_cpu_baseline:
                 rate, secs, threads, desc = two_stream_oracle_rate(spec)
                 line["cpu_baseline"] = {"value": rate, "unit": "tokens/s", "cores": threads,
-                                        "kind": "oracle", "sample": desc, "seconds": secs}
+                                        "kind": "oracle", "sample": desc,
+                                        "seconds_measured": secs}
             print(json.dumps(line), flush=True)
         if world > 1:
             tdist.destroy_process_group()
@@ -1010,7 +1070,7 @@ def main():
         if world == 1 and not args.no_cpu_baseline:
             rate, secs, threads, desc = oracle_sample_rate(spec, args.cpu_sample_requests)
             line["cpu_baseline"] = {"value": rate, "unit": UNIT, "cores": threads,
-                                    "kind": "oracle", "sample": desc, "seconds": secs}
+                                    "kind": "oracle", "sample": desc, "seconds_measured": secs}
         print(json.dumps(line), flush=True)
     if world > 1:
         tdist.destroy_process_group()

@@ -436,8 +436,15 @@ flare_status flare_append_kv(const flare_softmax_desc* desc, const void* k_blk, 
  *  - This call allocates nothing (no cudaMalloc, cudaFree or allocating
  *    library routine).
  *  - The first call on each device looks up the array's device address
- *    (cudaGetSymbolAddress, current device); make that first call before any
- *    stream capture.
+ *    (cudaGetSymbolAddress, current device) and caches it.  With CUDA's
+ *    default lazy module loading that lookup is also when the array's memory
+ *    is committed on the device, so make the first call (a warm-up call will
+ *    do) at start-up: before the engine reserves its memory pool, and before
+ *    any stream capture.  CUDA_MODULE_LOADING=EAGER commits it when the
+ *    library is loaded instead.
+ *  - The cached address belongs to the device's current context: after
+ *    cudaDeviceReset (or anything else that destroys the primary context)
+ *    this entry point must not be called again in the process.
  *  - If the shape needs more scratch than FLARE_NOALLOC_SCRATCH_BYTES
  *    (flare_softmax_workspace_size reports the need), the call returns
  *    FLARE_ERR_UNSUPPORTED and launches nothing.

@@ -14,6 +14,11 @@
 // loads it holds its FLARE_NOALLOC_SCRATCH_BYTES.  In host code the array's
 // name is only a host-side stand-in, so its device address is looked up with
 // cudaGetSymbolAddress once per device (with that device current) and cached.
+// Under CUDA's default lazy module loading, that first lookup is what commits
+// the array on the device, so a caller makes its first call at start-up,
+// before its own memory pool takes the device and before any stream capture.
+// The cached address is tied to the device's primary context and goes stale
+// if that context is destroyed (cudaDeviceReset).
 // Every call shares the array: calls that overlap on the GPU (other streams,
 // other host threads) race on it.  Nothing in it needs to start at zero: each
 // call writes every partial it later reads.
