@@ -253,8 +253,13 @@ flare_status flare_commit_state(const flare_linear_desc* d, const void* q, const
   p.out_causal = causal_out;
   p.write_state = 1;
   p.dev_status = dev_status;
-  const cudaError_t e = launch_gdr_commit(p, d->act_dtype == FLARE_DT_BF16,
-                                          static_cast<cudaStream_t>(stream));
+  const bool bf16 = d->act_dtype == FLARE_DT_BF16;
+  // bf16 blocks of the 128 x 128 state without token-causal outputs take the
+  // tensor-core chunkwise commit, the rest the register recurrence
+  const cudaError_t e =
+      (bf16 && !causal_out && gdr_commit_tc_supported(p.B, p.dk, p.dv))
+          ? launch_gdr_commit_tc(p, static_cast<cudaStream_t>(stream))
+          : launch_gdr_commit(p, bf16, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? FLARE_OK : FLARE_ERR_CUDA;
 }
 
