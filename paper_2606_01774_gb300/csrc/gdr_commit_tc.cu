@@ -63,11 +63,14 @@ struct CtCfg {
   static constexpr int kATs = BM + 4;              // row stride of A^T (floats)
   static constexpr int kAT = BM * kATs * 4;        // A^T[i][t] = A[t][i]
   static constexpr int kV = 2 * BM * 128;          // values: 2 chunks of BM rows x 128 B
-  // the values, once read into registers, make room for A^T
-  static constexpr int kR = kAT > kV ? kAT : kV;
-  // the keys come first: the Gram MMA's A operand reads 128 rows from each
-  // 64-row chunk, the second chunk's surplus rows land in the state buffer
-  static constexpr int kSmem = kK + kS0 + kR;
+  // the values, once read into registers, make room for A^T; at least 8 KiB,
+  // since the Gram MMA's A operand reads 128 rows from each 64-row key chunk
+  // and the second chunk's surplus rows land here
+  static constexpr int kR0 = kAT > kV ? kAT : kV;
+  static constexpr int kR = kR0 > 8192 ? kR0 : 8192;
+  // tensor-memory columns of each bf16 part of delta'^T (whole 16-column stores)
+  static constexpr int kDP = BM / 2 < 16 ? 16 : BM / 2;
+  static constexpr int kSmem = kS0 + kK + kR;  // state, keys, values / A^T
 };
 
 struct CtMaps {
@@ -141,9 +144,9 @@ __global__ void __launch_bounds__(kCtThreads, 2)
   extern __shared__ uint8_t smem_raw[];
   __shared__ CtShared sh;
   uint8_t* base = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  uint8_t* Ks = base;
-  float* S0s = reinterpret_cast<float*>(base + C::kK);
-  uint8_t* Rs = base + C::kK + C::kS0;  // the values, then A^T
+  float* S0s = reinterpret_cast<float*>(base);
+  uint8_t* Ks = base + C::kS0;
+  uint8_t* Rs = Ks + C::kK;  // the values, then A^T
   float* AT = reinterpret_cast<float*>(Rs);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -168,7 +171,7 @@ __global__ void __launch_bounds__(kCtThreads, 2)
   tc::fence_after_sync();
   const uint32_t tmem = sh.tmem_base;
   const uint32_t tmS = tmem;             // S0^T hi [0,64) and lo [64,128); then D
-  const uint32_t tmW = tmem + 128;       // W^T; then delta'^T hi [0,BM/2) and lo [BM/2,BM)
+  const uint32_t tmW = tmem + 128;       // W^T; then delta'^T hi [0,kDP) and lo [kDP,2kDP)
   const uint32_t tmG = tmem + 128 + BM;  // G (rows t on lanes t)
   const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
 
@@ -319,36 +322,45 @@ __global__ void __launch_bounds__(kCtThreads, 2)
         tc::tmem_st16(tmS + lane_off + i0, d);
       }
     }
-    // A^T from the Gram rows t < B (warps 0 .. BM/32-1)
-    if (tid < BM) {
+    // A^T from the Gram rows t < BM (the warps holding those lanes); rows of
+    // A at or past n are zero, so the solve below may run all BM steps
+    if (warp < (BM + 31) / 32) {
       const int t = tid;
       uint32_t gr[BM];
 #pragma unroll
       for (int c0 = 0; c0 < BM; c0 += 16)
         tc::tmem_ld16(tmG + lane_off + c0, *reinterpret_cast<uint32_t(*)[16]>(&gr[c0]));
       tc::tmem_ld_wait();
-      const float bt = sh.beta[t], gt = sh.gam2[t];
-      const bool live = t < n;
+      if (t < BM) {
+        const float bt = sh.beta[t], gt = sh.gam2[t];
+        const bool live = t < n;
 #pragma unroll
-      for (int i = 0; i < BM; ++i)
-        AT[i * kATs + t] =
-            (live && i < t) ? bt * tc::ex2(gt - sh.gam2[i]) * __uint_as_float(gr[i]) : 0.f;
+        for (int i = 0; i < BM; ++i)
+          AT[i * kATs + t] =
+              (live && i < t) ? bt * tc::ex2(gt - sh.gam2[i]) * __uint_as_float(gr[i]) : 0.f;
+      }
     }
     // X = diag(beta) (V - diag(Gam) W) for this thread's column
     float x[BM];
 #pragma unroll
     for (int c0 = 0; c0 < BM; c0 += 16) {
       uint32_t w[16];
-      tc::tmem_ld16(tmW + lane_off + c0, w);
+      tc::tmem_ld16(tmW + lane_off + c0, w);  // columns past Bp: stale, used by no kept row
       tc::tmem_ld_wait();
 #pragma unroll
-      for (int e = 0; e < 16; ++e) {
-        const int t = c0 + e;
-        x[t] = sh.beta[t] * (__uint_as_float(vraw[t] << 16) - sh.Gam[t] * __uint_as_float(w[e]));
+      for (int e4 = 0; e4 < 4; ++e4) {
+        const float4 b4 = *reinterpret_cast<const float4*>(&sh.beta[c0 + 4 * e4]);
+        const float4 g4 = *reinterpret_cast<const float4*>(&sh.Gam[c0 + 4 * e4]);
+        const float bb[4] = {b4.x, b4.y, b4.z, b4.w}, gg[4] = {g4.x, g4.y, g4.z, g4.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int t = c0 + 4 * e4 + e;
+          x[t] = bb[e] * (__uint_as_float(vraw[t] << 16) - gg[e] * __uint_as_float(w[4 * e4 + e]));
+        }
       }
     }
     tc::fence_before_sync();
-    __syncthreads();  // A^T published; the state buffer and W^T, G read
+    __syncthreads();  // A^T published; the state buffer, W^T and G read
     // the next item's state streams in while this one is solved and stored
     if (tid == 0 && it_next >= 0) {
       issue_s0(it_next, slot_next);
@@ -357,37 +369,39 @@ __global__ void __launch_bounds__(kCtThreads, 2)
     }
 
     // (I + A) delta = X, right-looking: once delta_t is final it leaves the
-    // remaining rows (A^T row t as 16-byte broadcast loads)
+    // remaining rows (A^T row t as 16-byte broadcast loads).  Rows t >= n
+    // only touch rows past n (A^T is zero there), which nothing keeps.
 #pragma unroll
     for (int t = 0; t < BM; ++t) {
-      if (t < n) {
-        const float dt = x[t];
-        const float* ar = AT + t * kATs;
+      const float dt = x[t];
+      const float* ar = AT + t * kATs;
 #pragma unroll
-        for (int u4 = (t + 1) / 4; u4 < BM / 4; ++u4) {
-          const float4 a = *reinterpret_cast<const float4*>(ar + 4 * u4);
-          if (4 * u4 + 0 > t) x[4 * u4 + 0] = fmaf(-a.x, dt, x[4 * u4 + 0]);
-          if (4 * u4 + 1 > t) x[4 * u4 + 1] = fmaf(-a.y, dt, x[4 * u4 + 1]);
-          if (4 * u4 + 2 > t) x[4 * u4 + 2] = fmaf(-a.z, dt, x[4 * u4 + 2]);
-          if (4 * u4 + 3 > t) x[4 * u4 + 3] = fmaf(-a.w, dt, x[4 * u4 + 3]);
-        }
+      for (int u4 = (t + 1) / 4; u4 < BM / 4; ++u4) {
+        const float4 a = *reinterpret_cast<const float4*>(ar + 4 * u4);
+        if (4 * u4 + 0 > t) x[4 * u4 + 0] = fmaf(-a.x, dt, x[4 * u4 + 0]);
+        if (4 * u4 + 1 > t) x[4 * u4 + 1] = fmaf(-a.y, dt, x[4 * u4 + 1]);
+        if (4 * u4 + 2 > t) x[4 * u4 + 2] = fmaf(-a.z, dt, x[4 * u4 + 2]);
+        if (4 * u4 + 3 > t) x[4 * u4 + 3] = fmaf(-a.w, dt, x[4 * u4 + 3]);
       }
     }
     // delta'_t = exp(gamma_{n-1} - gamma_t) delta_t (t < n), as bf16 hi and lo parts
     {
       const float gn2 = sh.gam2[n - 1];
 #pragma unroll
-      for (int c0 = 0; c0 < BM / 2; c0 += 16) {
+      for (int c0 = 0; c0 < C::kDP; c0 += 16) {
         uint32_t hi[16], lo[16];
 #pragma unroll
         for (int e = 0; e < 16; ++e) {
           const int t = 2 * (c0 + e);
-          const float a = t < n ? x[t] * tc::ex2(gn2 - sh.gam2[t]) : 0.f;
-          const float b = t + 1 < n ? x[t + 1] * tc::ex2(gn2 - sh.gam2[t + 1]) : 0.f;
+          float a = 0.f, b = 0.f;
+          if (t < BM) {
+            a = t < n ? x[t] * tc::ex2(gn2 - sh.gam2[t]) : 0.f;
+            b = t + 1 < n ? x[t + 1] * tc::ex2(gn2 - sh.gam2[t + 1]) : 0.f;
+          }
           split_pair(a, b, hi[e], lo[e]);
         }
         tc::tmem_st16(tmW + lane_off + c0, hi);
-        tc::tmem_st16(tmW + lane_off + BM / 2 + c0, lo);
+        tc::tmem_st16(tmW + lane_off + C::kDP + c0, lo);
       }
     }
     tc::tmem_st_wait();
@@ -401,7 +415,7 @@ __global__ void __launch_bounds__(kCtThreads, 2)
       for (int kk = 0; kk < ksteps; ++kk) {
         const uint64_t kb = tc::sdesc_sw128(tc::smem_u32(Ks + kk * 2048), 64 * 128, 1024);
         tc::mma_bf16_ts(tmS, tmW + kk * 8, kb, idU, 1u);
-        tc::mma_bf16_ts(tmS, tmW + BM / 2 + kk * 8, kb, idU, 1u);
+        tc::mma_bf16_ts(tmS, tmW + C::kDP + kk * 8, kb, idU, 1u);
       }
       tc::mma_commit(&sh.bar_mma);
       mma_out = true;
@@ -515,6 +529,7 @@ bool gdr_commit_tc_supported(int B, int dk, int dv) {
 
 cudaError_t launch_gdr_commit_tc(const GdrParams& p, cudaStream_t stream) {
   if (p.R == 0) return cudaSuccess;
+  if (p.B <= 16) return launch_ct<16>(p, stream);
   return p.B <= 32 ? launch_ct<32>(p, stream) : launch_ct<64>(p, stream);
 }
 
