@@ -1016,11 +1016,16 @@ def main():
     ap.add_argument("--cpu-sample-requests", type=int, default=2)
     ap.add_argument("--no-per-config", action="store_true",
                     help="skip timing the other batched workloads after the headline one")
+    ap.add_argument("--requests", type=int, default=0,
+                    help="profiling cut: the workload's shapes with this many requests "
+                         "(its line is no bench value)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "flare":
         ap.error("--warmup must be >= 3")
     training = args.workload in workloads.TWO_STREAM_WORKLOADS
     spec = (workloads.TWO_STREAM_WORKLOADS if training else workloads.WORKLOADS)[args.workload]
+    if args.requests > 0 and not training:
+        spec = spec.replace(num_requests=args.requests)
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))

@@ -63,11 +63,8 @@ struct CtCfg {
   static constexpr int kATs = BM + 4;              // row stride of A^T (floats)
   static constexpr int kAT = BM * kATs * 4;        // A^T[i][t] = A[t][i]
   static constexpr int kV = 2 * BM * 128;          // values: 2 chunks of BM rows x 128 B
-  // the values, once read into registers, make room for A^T; at least 8 KiB,
-  // since the Gram MMA's A operand reads 128 rows from each 64-row key chunk
-  // and the second chunk's surplus rows land here
-  static constexpr int kR0 = kAT > kV ? kAT : kV;
-  static constexpr int kR = kR0 > 8192 ? kR0 : 8192;
+  // the values, once read into registers, make room for A^T
+  static constexpr int kR = kAT > kV ? kAT : kV;
   // tensor-memory columns of each bf16 part of delta'^T (whole 16-column stores)
   static constexpr int kDP = BM / 2 < 16 ? 16 : BM / 2;
   static constexpr int kSmem = kS0 + kK + kR;  // state, keys, values / A^T
@@ -172,7 +169,11 @@ __global__ void __launch_bounds__(kCtThreads, 2)
   const uint32_t tmem = sh.tmem_base;
   const uint32_t tmS = tmem;             // S0^T hi [0,64) and lo [64,128); then D
   const uint32_t tmW = tmem + 128;       // W^T; then delta'^T hi [0,kDP) and lo [kDP,2kDP)
-  const uint32_t tmG = tmem + 128 + BM;  // G (rows t on lanes t)
+  // G: row t on lane kG0 + t, the top BM lanes (warps 2-3), so that warp 0,
+  // which also scans the gates and issues the copies and MMAs, is not the
+  // one building A^T
+  constexpr int kG0 = 128 - BM;
+  const uint32_t tmG = tmem + 128 + BM;
   const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
 
   auto state_of = [&](int item, int s) {
@@ -272,7 +273,7 @@ __global__ void __launch_bounds__(kCtThreads, 2)
     if (!ct_wait(&sh.bar_s0, ph, sh, p.dev_status)) break;
     if (tid == 0) s0_out = false;
     // S0^T (column c = tid of S0) into tensor memory as bf16 hi and lo parts
-#pragma unroll
+#pragma unroll 1
     for (int i0 = 0; i0 < kCtD; i0 += 32) {
       uint32_t hi[16], lo[16];
 #pragma unroll
@@ -290,9 +291,13 @@ __global__ void __launch_bounds__(kCtThreads, 2)
       tc::fence_after_sync();
 #pragma unroll
       for (int kk = 0; kk < kCtD / 16; ++kk) {
-        const uint64_t kd =
-            tc::sdesc_sw128(tc::smem_u32(Ks + (kk >> 2) * (64 * 128) + (kk & 3) * 32), 16, 1024);
-        tc::mma_bf16_ss(tmG, kd, kd, idN, kk > 0);                // G = K K^T
+        const uint8_t* kc = Ks + (kk >> 2) * (64 * 128) + (kk & 3) * 32;
+        const uint64_t kd = tc::sdesc_sw128(tc::smem_u32(kc), 16, 1024);
+        // A operand rows kG0.. are the keys; the rows before read the bytes
+        // ahead of the chunk (the state buffer, then the first chunk), which
+        // only reach lanes nobody reads
+        const uint64_t kg = tc::sdesc_sw128(tc::smem_u32(kc - kG0 * 128), 16, 1024);
+        tc::mma_bf16_ss(tmG, kg, kd, idN, kk > 0);                // G = K K^T
         tc::mma_bf16_ts(tmW, tmS + kk * 8, kd, idN, kk > 0);      // W^T = S0hi^T K^T
         tc::mma_bf16_ts(tmW, tmS + 64 + kk * 8, kd, idN, 1u);     //     + S0lo^T K^T
       }
@@ -314,7 +319,7 @@ __global__ void __launch_bounds__(kCtThreads, 2)
     // the accumulator starts at Gam_{n-1} S0^T (fp32, from the loaded state)
     {
       const float Gn = sh.Gam[n - 1];
-#pragma unroll
+#pragma unroll 2
       for (int i0 = 0; i0 < kCtD; i0 += 16) {
         uint32_t d[16];
 #pragma unroll
@@ -324,14 +329,14 @@ __global__ void __launch_bounds__(kCtThreads, 2)
     }
     // A^T from the Gram rows t < BM (the warps holding those lanes); rows of
     // A at or past n are zero, so the solve below may run all BM steps
-    if (warp < (BM + 31) / 32) {
-      const int t = tid;
+    if (warp >= kG0 / 32) {
+      const int t = tid - kG0;
       uint32_t gr[BM];
 #pragma unroll
       for (int c0 = 0; c0 < BM; c0 += 16)
         tc::tmem_ld16(tmG + lane_off + c0, *reinterpret_cast<uint32_t(*)[16]>(&gr[c0]));
       tc::tmem_ld_wait();
-      if (t < BM) {
+      if (t >= 0) {
         const float bt = sh.beta[t], gt = sh.gam2[t];
         const bool live = t < n;
 #pragma unroll
@@ -435,7 +440,7 @@ __global__ void __launch_bounds__(kCtThreads, 2)
     // the committed state: lane c holds S^(n)[i][c] over i
     {
       float* Sg = state_of(it, slot) + tid;
-#pragma unroll
+#pragma unroll 1
       for (int i0 = 0; i0 < kCtD; i0 += 32) {
         uint32_t d[32];
         tc::tmem_ld16(tmS + lane_off + i0, *reinterpret_cast<uint32_t(*)[16]>(&d[0]));
