@@ -211,10 +211,16 @@ flare_status flare_block_linear_attn(const flare_linear_desc* d, const void* q, 
   p.write_state = 0;
   p.dev_status = dev_status;
   const bool bf16 = d->act_dtype == FLARE_DT_BF16;
-  const cudaError_t e =
-      (bf16 && gdr_denoise_tc_supported(p.B, p.dk, p.dv))
-          ? launch_gdr_denoise_tc(p, static_cast<cudaStream_t>(stream))
-          : launch_gdr_recurrent(p, bf16, static_cast<cudaStream_t>(stream));
+  // bf16: the persistent tensor-core kernel for 128 x 128 states and B <= 32,
+  // the one-CTA-per-item tensor-core kernel for the other shapes; fp32 the
+  // CUDA-core recurrence
+  cudaError_t e;
+  if (bf16 && gdr_denoise_persist_supported(p.B, p.dk, p.dv))
+    e = launch_gdr_denoise_persist(p, static_cast<cudaStream_t>(stream));
+  else if (bf16 && gdr_denoise_tc_supported(p.B, p.dk, p.dv))
+    e = launch_gdr_denoise_tc(p, static_cast<cudaStream_t>(stream));
+  else
+    e = launch_gdr_recurrent(p, bf16, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? FLARE_OK : FLARE_ERR_CUDA;
 }
 

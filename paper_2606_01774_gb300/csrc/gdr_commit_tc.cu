@@ -79,9 +79,10 @@ struct alignas(16) CtShared {
   uint64_t bar_s0, bar_k, bar_mma;
   uint32_t tmem_base;
   int abort_flag;
-  float gam2[64];  // gamma_t log2(e)
-  float Gam[64];   // exp(gamma_t)
-  float beta[64];
+  // 16-byte aligned: read as float4 broadcasts
+  alignas(16) float gam2[64];  // gamma_t log2(e)
+  alignas(16) float Gam[64];   // exp(gamma_t)
+  alignas(16) float beta[64];
 };
 
 __device__ __forceinline__ bool ct_wait(uint64_t* bar, uint32_t parity, CtShared& sh,

@@ -1,0 +1,539 @@
+// Denoise pass of a gated-delta-rule layer for the 128 x 128 state on tcgen05
+// tensor cores, persistent form: bf16 activations, B <= 32.
+//
+// For one (request r, value head j) with q/k head h and frozen state S0, the
+// block-end readout (Eq. noisy-block-fwd) through the chunkwise WY/UT form of
+// the block (appendix "Chunk-corrected values", Eq. chunk-state):
+//
+//   gamma_t = g_0 + ... + g_t,  Gam_t = exp(gamma_t)
+//   A[t][i] = beta_t exp(gamma_t - gamma_i) (k_t . k_i),   i < t
+//   X       = diag(beta) (V - diag(Gam) K S0)
+//   (I + A) delta = X
+//   out[l]  = s (Gam_{B-1} S0^T q_l + sum_i exp(gamma_{B-1} - gamma_i) (q_l . k_i) delta_i)
+//
+// Value column c on tensor-memory lane c; thread c owns column c:
+//
+//   MMA 1  G   = [K;Q] K^T        M=128 ([K;Q] rows on lanes kG0..), N=Bp, K=128
+//          W^T = S0^T [K;Q]^T     M=128 (c), N=2BM, K=128   (A: S0^T, bf16, tensor memory)
+//   solve  (I + A) delta = X      fp32, per column, right-looking
+//   MMA 2  O2^T = delta^T M2^T    M=128 (c), N=Bp, K=Bp     (A: delta^T, bf16, tensor memory)
+//          M2[l][i] = exp(gamma_{B-1} - gamma_i) (q_l . k_i)
+//   out[l][c] = s (Gam_{B-1} W^T[c][BM + l] + O2^T[c][l])
+//
+// Bp = B rounded up to 16; the K, Q and V tiles hold BM = 16 or 32 rows (rows
+// past B read as zero).  Inputs bf16, the state fp32 in memory and rounded to
+// bf16 for the products, all accumulation fp32 (the same precision as the
+// one-CTA-per-item kernel in gdr_tc.cu, which serves the other shapes).
+//
+// Persistent CTAs, two per SM (89-92 KiB of shared memory, 256 tensor-memory
+// columns each), 128 threads, each walking the (request, value head) items
+// blockIdx.x, blockIdx.x + gridDim.x, ...  The state arrives by bulk copy into
+// a 64 KiB buffer that is free again as soon as it has been turned into the
+// bf16 S0^T operand, so the next item's state streams in during this item's
+// products, solve and readout; the next keys and queries follow this item's
+// first MMA, the next values its solve, the next gates and slot one item
+// ahead into registers.  A bad slot is flagged in the device status word and
+// the item skipped (its output untouched).  Every wait is bounded: on a
+// timeout the CTA sets FLARE_DEV_WAIT_TIMEOUT, waits (bounded) for its copies
+// and MMAs in flight, frees its tensor memory and exits.
+#include <cudaTypedefs.h>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "tc.cuh"
+
+namespace flare {
+
+namespace {
+
+constexpr int kDpThreads = 128;
+constexpr int kDpD = 128;  // d_k = d_v
+
+template <int BM>
+struct DpCfg {
+  static constexpr int kS0 = kDpD * kDpD * 4;   // S0 fp32 [i][c]
+  static constexpr int kATs = BM + 4;           // row stride of A^T (floats)
+  static constexpr int kAT = BM * kATs * 4;     // A^T[i][t] = A[t][i]
+  static constexpr int kV = 2 * BM * 128;       // values: 2 chunks of BM rows x 128 B
+  static constexpr int kG0 = 128 - 2 * BM;      // lane of G's first row
+  // the values, then A^T; the Gram MMA's A operand starts kG0 rows ahead of
+  // the [K;Q] tile and reads those bytes here (their rows reach no lane that
+  // is read)
+  static constexpr int kR0 = kAT > kV ? kAT : kV;
+  static constexpr int kR1 = kR0 > kG0 * 128 ? kR0 : kG0 * 128;
+  static constexpr int kR = (kR1 + 1023) / 1024 * 1024;
+  static constexpr int kKQ = 2 * 2 * BM * 128;  // 2 chunks of [K;Q]: 2BM rows x 128 B (SW128)
+  static constexpr int kM2 = BM * 128;          // M2 [l][i], K-major, SW128
+  static constexpr int kSmem = kS0 + kR + kKQ + kM2;
+};
+
+struct alignas(16) DpShared {
+  uint64_t bar_s0, bar_kq, bar_v, bar_mma;
+  uint32_t tmem_base;
+  int abort_flag;
+  // 16-byte aligned: read as float4 broadcasts
+  alignas(16) float gam2[32];  // gamma_t log2(e)
+  alignas(16) float Gam[32];   // exp(gamma_t)
+  alignas(16) float beta[32];
+};
+
+struct DpMaps {
+  CUtensorMap k;  // (128, Hk, B, R) box (64, 1, BM, 1), 128-byte swizzle
+  CUtensorMap q;
+  CUtensorMap v;  // (128, Hv, B, R) box (64, 1, BM, 1), no swizzle
+};
+
+__device__ __forceinline__ bool dp_wait(uint64_t* bar, uint32_t parity, DpShared& sh,
+                                        int32_t* status) {
+  const bool ok = tc::mbar_wait(bar, parity, &sh.abort_flag);
+  const bool all = __syncthreads_and(ok);
+  if (!all && threadIdx.x == 0 && !sh.abort_flag) {
+    sh.abort_flag = 1;
+    flag(status, FLARE_DEV_WAIT_TIMEOUT);
+  }
+  return all;
+}
+
+// The next item at or after `it` (stride gridDim.x) with a valid slot; bad
+// slots are flagged and skipped.  Called by every thread with the same
+// arguments.
+__device__ __forceinline__ int dp_next(const GdrParams& p, int it, int total, int& slot) {
+  for (; it < total; it += gridDim.x) {
+    const int s = p.state_slot[it / p.Hv];
+    if (s < 0 || s >= p.nslots) {
+      if (threadIdx.x == 0) flag(p.dev_status, FLARE_DEV_BAD_SLOT);
+      continue;
+    }
+    slot = s;
+    return it;
+  }
+  return -1;
+}
+
+__device__ __forceinline__ uint32_t dp_pack(float a, float b) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// 16 bf16 values (columns c0..c0+15) into row `row` of a K-major SW128 tile.
+__device__ __forceinline__ void dp_store16_sw128(uint8_t* tile, int row, int c0,
+                                                 const float (&v)[16]) {
+  uint8_t* p = tile + row * 128;
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int g = (c0 >> 3) + h;
+    *reinterpret_cast<uint4*>(p + ((g ^ (row & 7)) << 4)) =
+        make_uint4(dp_pack(v[8 * h], v[8 * h + 1]), dp_pack(v[8 * h + 2], v[8 * h + 3]),
+                   dp_pack(v[8 * h + 4], v[8 * h + 5]), dp_pack(v[8 * h + 6], v[8 * h + 7]));
+  }
+}
+
+}  // namespace
+
+template <int BM>
+__global__ void __launch_bounds__(kDpThreads, 2)
+    gdr_denoise_persist_kernel(const __grid_constant__ DpMaps maps, GdrParams p) {
+  using C = DpCfg<BM>;
+  constexpr int kATs = C::kATs;
+  constexpr int kG0 = C::kG0;
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ DpShared sh;
+  uint8_t* base = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  float* S0s = reinterpret_cast<float*>(base);
+  uint8_t* Rs = base + C::kS0;  // the values, then A^T
+  float* AT = reinterpret_cast<float*>(Rs);
+  uint8_t* KQs = Rs + C::kR;
+  uint8_t* M2s = KQs + C::kKQ;
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int total = p.R * p.Hv;
+  const int B = p.B;
+  const int Bp = (B + 15) & ~15;
+
+  int slot = 0;
+  int it = dp_next(p, blockIdx.x, total, slot);
+  if (it < 0) return;  // the same answer on every thread
+
+  if (tid == 0) {
+    sh.abort_flag = 0;
+    tc::mbar_init(&sh.bar_s0, 1);
+    tc::mbar_init(&sh.bar_kq, 1);
+    tc::mbar_init(&sh.bar_v, 1);
+    tc::mbar_init(&sh.bar_mma, 1);
+    tc::fence_mbar_init();
+  }
+  if (warp == 0) tc::tmem_alloc(&sh.tmem_base, 256);
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = sh.tmem_base;
+  const uint32_t tmS = tmem;                // S0^T bf16 (64 columns); then delta^T
+  const uint32_t tmW = tmem + 64;           // W^T: [K part | Q part], 2BM columns
+  const uint32_t tmG = tmem + 64 + 2 * BM;  // G (rows on lanes kG0..); then O2^T
+  const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
+
+  auto issue_s0 = [&](int item, int s) {
+    const float* src = p.state_pool + ((size_t)s * p.Hv + item % p.Hv) * kDpD * kDpD;
+    tc::mbar_expect_tx(&sh.bar_s0, C::kS0);
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      tc::bulk_load(S0s + q * (kDpD * kDpD / 4), src + q * (kDpD * kDpD / 4), C::kS0 / 4,
+                    &sh.bar_s0);
+  };
+  auto issue_kq = [&](int item) {
+    const int r = item / p.Hv, h = (item % p.Hv) / (p.Hv / p.Hk);
+    tc::mbar_expect_tx(&sh.bar_kq, C::kKQ);
+#pragma unroll
+    for (int c = 0; c < 2; ++c) {
+      tc::tma_load_4d(KQs + c * (2 * BM * 128), &maps.k, &sh.bar_kq, c * 64, h, 0, r);
+      tc::tma_load_4d(KQs + c * (2 * BM * 128) + BM * 128, &maps.q, &sh.bar_kq, c * 64, h, 0, r);
+    }
+  };
+  auto issue_v = [&](int item) {
+    const int r = item / p.Hv, j = item % p.Hv;
+    tc::mbar_expect_tx(&sh.bar_v, C::kV);
+    tc::tma_load_4d(Rs, &maps.v, &sh.bar_v, 0, j, 0, r);
+    tc::tma_load_4d(Rs + BM * 128, &maps.v, &sh.bar_v, 64, j, 0, r);
+  };
+  // warp 0 holds the gates of the item it processes next, loaded one item ahead
+  float gq = 0.f, bq = 0.f;
+  auto load_gates = [&](int item) {
+    const size_t gb = (size_t)(item / p.Hv) * B * p.Hv + item % p.Hv;
+    gq = lane < B ? p.log_decay[gb + (size_t)lane * p.Hv] : 0.f;
+    bq = lane < B ? p.beta[gb + (size_t)lane * p.Hv] : 0.f;
+  };
+  auto cand_slot = [&](int c) { return c < total ? p.state_slot[c / p.Hv] : -1; };
+
+  // thread 0's record of what is in flight (and the parity its barrier
+  // phase completes with), for a clean exit after a timeout
+  bool s0_out = false, kq_out = false, v_out = false, mma_out = false;
+  uint32_t s0_par = 0, kq_par = 0, v_par = 0;
+  if (tid == 0) {
+    tc::prefetch_tmap(&maps.k);
+    tc::prefetch_tmap(&maps.q);
+    tc::prefetch_tmap(&maps.v);
+    issue_s0(it, slot);
+    issue_kq(it);
+    issue_v(it);
+    s0_out = kq_out = v_out = true;
+  }
+  if (warp == 0) load_gates(it);
+  int cand = it + gridDim.x;
+  int cs = cand_slot(cand);
+  uint32_t ph = 0;      // parity of the item's loads
+  uint32_t ph_mma = 0;  // parity of the next MMA completion (two per item)
+  const uint32_t idG = tc::idesc_bf16(128, Bp, false, false);
+  const uint32_t idW = tc::idesc_bf16(128, 2 * BM, false, false);
+  const uint32_t idO = tc::idesc_bf16(128, Bp, false, false);
+
+#pragma unroll 1
+  while (true) {
+    const int r = it / p.Hv, j = it % p.Hv;
+    // the block's gates: gamma = inclusive prefix sum of the log-gates
+    if (warp == 0) {
+      float g = gq;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const float a = __shfl_up_sync(0xffffffffu, g, o);
+        if (lane >= o) g += a;
+      }
+      sh.gam2[lane] = g * 1.4426950408889634f;
+      sh.Gam[lane] = expf(g);
+      sh.beta[lane] = bq;
+    }
+    // the next item: the candidate when its slot is valid, else the first
+    // valid one after it (bad ones flagged on the way)
+    int it_next = -1, slot_next = 0;
+    if (cand < total) {
+      if (cs >= 0 && cs < p.nslots) {
+        it_next = cand;
+        slot_next = cs;
+      } else {
+        it_next = dp_next(p, cand, total, slot_next);
+      }
+    }
+    if (it_next >= 0) {
+      if (warp == 0) load_gates(it_next);
+      cand = it_next + gridDim.x;
+      cs = cand_slot(cand);
+    }
+
+    if (!dp_wait(&sh.bar_s0, ph, sh, p.dev_status)) break;
+    if (tid == 0) s0_out = false;
+    // S0^T (column c = tid of S0) into tensor memory as bf16 pairs
+#pragma unroll 1
+    for (int i0 = 0; i0 < kDpD; i0 += 32) {
+      uint32_t w[16];
+#pragma unroll
+      for (int e = 0; e < 16; ++e)
+        w[e] = dp_pack(S0s[(i0 + 2 * e) * kDpD + tid], S0s[(i0 + 2 * e + 1) * kDpD + tid]);
+      tc::tmem_st16(tmS + lane_off + i0 / 2, w);
+    }
+    tc::tmem_st_wait();
+    tc::fence_before_sync();
+    if (!dp_wait(&sh.bar_kq, ph, sh, p.dev_status)) break;  // also: the state buffer read
+    if (tid == 0) {
+      kq_out = false;
+      // the state buffer is free: the next item's state streams in during
+      // this item's products, solve and readout
+      if (it_next >= 0) {
+        issue_s0(it_next, slot_next);
+        s0_out = true;
+        s0_par = ph ^ 1u;
+      }
+      tc::fence_after_sync();
+#pragma unroll
+      for (int kk = 0; kk < kDpD / 16; ++kk) {
+        const uint8_t* kc = KQs + (kk >> 2) * (2 * BM * 128) + (kk & 3) * 32;
+        const uint64_t kd = tc::sdesc_sw128(tc::smem_u32(kc), 16, 1024);
+        const uint64_t kg = tc::sdesc_sw128(tc::smem_u32(kc - kG0 * 128), 16, 1024);
+        tc::mma_bf16_ss(tmG, kg, kd, idG, kk > 0);            // G = [K;Q] K^T
+        tc::mma_bf16_ts(tmW, tmS + kk * 8, kd, idW, kk > 0);  // W^T = S0^T [K;Q]^T
+      }
+      tc::mma_commit(&sh.bar_mma);
+      mma_out = true;
+    }
+    if (!dp_wait(&sh.bar_v, ph, sh, p.dev_status)) break;
+    if (tid == 0) v_out = false;
+    // this column of the values as bf16 pairs (rows past B arrive as zeros)
+    uint32_t vpk[BM / 2];
+    {
+      const uint8_t* vb = Rs + (tid >> 6) * (BM * 128) + (tid & 63) * 2;
+#pragma unroll
+      for (int t2 = 0; t2 < BM / 2; ++t2)
+        vpk[t2] = (uint32_t)*reinterpret_cast<const unsigned short*>(vb + (2 * t2) * 128) |
+                  ((uint32_t)*reinterpret_cast<const unsigned short*>(vb + (2 * t2 + 1) * 128)
+                   << 16);
+    }
+    if (!dp_wait(&sh.bar_mma, ph_mma, sh, p.dev_status)) break;  // also: the values read
+    ph_mma ^= 1u;
+    tc::fence_after_sync();
+    if (tid == 0) {
+      mma_out = false;
+      if (it_next >= 0) {  // the first MMA, the only reader of [K;Q], is done
+        issue_kq(it_next);
+        kq_out = true;
+        kq_par = ph ^ 1u;
+      }
+    }
+    // A^T (key rows of G) and M2 (query rows), from the lanes that hold G
+    if (warp >= kG0 / 32) {
+      uint32_t gr[BM];
+#pragma unroll
+      for (int c0 = 0; c0 < BM; c0 += 16)
+        tc::tmem_ld16(tmG + lane_off + c0, *reinterpret_cast<uint32_t(*)[16]>(&gr[c0]));
+      tc::tmem_ld_wait();
+      const int row = tid - kG0;
+      if (row >= 0 && row < BM) {
+        const int t = row;
+        const float bt = sh.beta[t], gt = sh.gam2[t];
+        const bool live = t < B;
+#pragma unroll
+        for (int i = 0; i < BM; ++i)
+          AT[i * kATs + t] =
+              (live && i < t) ? bt * tc::ex2(gt - sh.gam2[i]) * __uint_as_float(gr[i]) : 0.f;
+      } else if (row >= BM) {
+        const int l = row - BM;
+        const float gB = sh.gam2[B - 1];
+#pragma unroll
+        for (int c0 = 0; c0 < BM; c0 += 16) {
+          float v[16];
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            const int i = c0 + e;
+            v[e] = (i < B && l < B) ? tc::ex2(gB - sh.gam2[i]) * __uint_as_float(gr[i]) : 0.f;
+          }
+          dp_store16_sw128(M2s, l, c0, v);
+        }
+        tc::fence_async_smem();  // M2 is the second MMA's operand
+      }
+    }
+    // X = diag(beta) (V - diag(Gam) K S0) for this column
+    float x[BM];
+#pragma unroll
+    for (int c0 = 0; c0 < BM; c0 += 16) {
+      uint32_t w[16];
+      tc::tmem_ld16(tmW + lane_off + c0, w);
+      tc::tmem_ld_wait();
+#pragma unroll
+      for (int e4 = 0; e4 < 4; ++e4) {
+        const float4 b4 = *reinterpret_cast<const float4*>(&sh.beta[c0 + 4 * e4]);
+        const float4 g4 = *reinterpret_cast<const float4*>(&sh.Gam[c0 + 4 * e4]);
+        const float bb[4] = {b4.x, b4.y, b4.z, b4.w}, gg[4] = {g4.x, g4.y, g4.z, g4.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int t = c0 + 4 * e4 + e;
+          const uint32_t vp = vpk[t / 2];
+          const float vt = __uint_as_float((t & 1) ? (vp & 0xffff0000u) : (vp << 16));
+          x[t] = bb[e] * (vt - gg[e] * __uint_as_float(w[4 * e4 + e]));
+        }
+      }
+    }
+    tc::fence_before_sync();
+    __syncthreads();  // A^T and M2 published; W^T's key part and G read
+
+    // (I + A) delta = X, right-looking (A^T row t as 16-byte broadcast loads);
+    // rows past B touch only rows past B (A^T is zero there)
+#pragma unroll
+    for (int t = 0; t < BM; ++t) {
+      const float dt = x[t];
+      const float* ar = AT + t * kATs;
+#pragma unroll
+      for (int u4 = (t + 1) / 4; u4 < BM / 4; ++u4) {
+        const float4 a = *reinterpret_cast<const float4*>(ar + 4 * u4);
+        if (4 * u4 + 0 > t) x[4 * u4 + 0] = fmaf(-a.x, dt, x[4 * u4 + 0]);
+        if (4 * u4 + 1 > t) x[4 * u4 + 1] = fmaf(-a.y, dt, x[4 * u4 + 1]);
+        if (4 * u4 + 2 > t) x[4 * u4 + 2] = fmaf(-a.z, dt, x[4 * u4 + 2]);
+        if (4 * u4 + 3 > t) x[4 * u4 + 3] = fmaf(-a.w, dt, x[4 * u4 + 3]);
+      }
+    }
+    // delta^T as bf16 pairs (rows past B zero) over S0^T, which MMA 1 has read
+    {
+      uint32_t w[16];
+#pragma unroll
+      for (int e = 0; e < 16; ++e) {
+        const int t = 2 * e;
+        float a = 0.f, b = 0.f;
+        if (t < BM) {
+          a = t < B ? x[t] : 0.f;
+          b = t + 1 < B ? x[t + 1] : 0.f;
+        }
+        w[e] = dp_pack(a, b);
+      }
+      tc::tmem_st16(tmS + lane_off, w);
+    }
+    tc::tmem_st_wait();
+    tc::fence_before_sync();
+    __syncthreads();  // also: A^T read, its region free for the next values
+    if (tid == 0) {
+      if (it_next >= 0) {
+        tc::fence_async_smem();
+        issue_v(it_next);
+        v_out = true;
+        v_par = ph ^ 1u;
+      }
+      tc::fence_after_sync();
+      for (int kk = 0; kk < Bp / 16; ++kk)
+        tc::mma_bf16_ts(tmG, tmS + kk * 8, tc::sdesc_sw128(tc::smem_u32(M2s + kk * 32), 16, 1024),
+                        idO, kk > 0);  // O2^T = delta^T M2^T, over G
+      tc::mma_commit(&sh.bar_mma);
+      mma_out = true;
+    }
+    if (!dp_wait(&sh.bar_mma, ph_mma, sh, p.dev_status)) break;
+    ph_mma ^= 1u;
+    tc::fence_after_sync();
+    if (tid == 0) mma_out = false;
+    // out[l][c] = s (Gam_{B-1} W^T[c][BM + l] + O2^T[c][l]); adjacent lanes
+    // swap one value so that each stores a bf16 pair of two columns
+    {
+      const float sG = p.scale * sh.Gam[B - 1];
+      uint32_t o2[BM], wq[BM];
+#pragma unroll
+      for (int c0 = 0; c0 < BM; c0 += 16) {
+        tc::tmem_ld16(tmG + lane_off + c0, *reinterpret_cast<uint32_t(*)[16]>(&o2[c0]));
+        tc::tmem_ld16(tmW + lane_off + BM + c0, *reinterpret_cast<uint32_t(*)[16]>(&wq[c0]));
+      }
+      tc::tmem_ld_wait();
+      const bool odd = lane & 1;
+      __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.out_blockend) +
+                           ((size_t)r * B * p.Hv + j) * kDpD + (tid & ~1);
+#pragma unroll
+      for (int l = 0; l < BM; l += 2) {
+        const float a = fmaf(sG, __uint_as_float(wq[l]), p.scale * __uint_as_float(o2[l]));
+        const float b = fmaf(sG, __uint_as_float(wq[l + 1]), p.scale * __uint_as_float(o2[l + 1]));
+        const float recv = __shfl_xor_sync(0xffffffffu, odd ? a : b, 1);
+        const int row = odd ? l + 1 : l;
+        if (row < B)
+          *reinterpret_cast<uint32_t*>(out + (size_t)row * p.Hv * kDpD) =
+              odd ? dp_pack(recv, b) : dp_pack(a, recv);
+      }
+    }
+    if (it_next < 0) break;
+    it = it_next;
+    slot = slot_next;
+    ph ^= 1u;
+  }
+
+  // after a timeout: let the copies and MMAs in flight land before the
+  // shared and tensor memory are given up (bounded waits)
+  if (tid == 0 && sh.abort_flag) {
+    if (s0_out) tc::mbar_wait(&sh.bar_s0, s0_par, nullptr, 100000000ull);
+    if (kq_out) tc::mbar_wait(&sh.bar_kq, kq_par, nullptr, 100000000ull);
+    if (v_out) tc::mbar_wait(&sh.bar_v, v_par, nullptr, 100000000ull);
+    if (mma_out) tc::mbar_wait(&sh.bar_mma, ph_mma, nullptr, 100000000ull);
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == 0) {
+    tc::fence_after_sync();
+    tc::tmem_dealloc(tmem, 256);
+  }
+}
+
+// ------------------------------------------------------------------ host side
+
+namespace {
+
+PFN_cuTensorMapEncodeTiled_v12000 dp_encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+  }
+  return fn;
+}
+
+// [R, B, H, 128] bf16 activations as a 4-D map (128, H, B, R), box (64, 1,
+// rows, 1); rows past B read as zero
+bool dp_act_map(CUtensorMap* m, const void* x, int H, int B, int R, int rows, bool swizzle) {
+  auto fn = dp_encode_fn();
+  if (!fn) return false;
+  cuuint64_t gd[4] = {(cuuint64_t)kDpD, (cuuint64_t)H, (cuuint64_t)B, (cuuint64_t)R};
+  cuuint64_t gs[3] = {(cuuint64_t)kDpD * 2, (cuuint64_t)H * kDpD * 2,
+                      (cuuint64_t)B * H * kDpD * 2};
+  cuuint32_t bx[4] = {64, 1, (cuuint32_t)rows, 1};
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(x), gd, gs, bx, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE,
+            swizzle ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+         CUDA_SUCCESS;
+}
+
+template <int BM>
+cudaError_t launch_dp(const GdrParams& p, cudaStream_t stream) {
+  DpMaps maps;
+  if (!dp_act_map(&maps.k, p.k, p.Hk, p.B, p.R, BM, true) ||
+      !dp_act_map(&maps.q, p.q, p.Hk, p.B, p.R, BM, true) ||
+      !dp_act_map(&maps.v, p.v, p.Hv, p.B, p.R, BM, false))
+    return cudaErrorInvalidValue;
+  const int smem = DpCfg<BM>::kSmem + 1024;
+  cudaError_t e = cudaFuncSetAttribute(gdr_denoise_persist_kernel<BM>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  int dev = 0, sms = kNumSMs;
+  if (cudaGetDevice(&dev) == cudaSuccess)
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const long items = (long)p.R * p.Hv;
+  const int grid = (int)(items < 2L * sms ? items : 2L * sms);
+  gdr_denoise_persist_kernel<BM><<<grid, kDpThreads, smem, stream>>>(maps, p);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+bool gdr_denoise_persist_supported(int B, int dk, int dv) {
+  return B >= 1 && B <= 32 && dk == kDpD && dv == kDpD;
+}
+
+cudaError_t launch_gdr_denoise_persist(const GdrParams& p, cudaStream_t stream) {
+  if (p.R == 0) return cudaSuccess;
+  return p.B <= 16 ? launch_dp<16>(p, stream) : launch_dp<32>(p, stream);
+}
+
+}  // namespace flare

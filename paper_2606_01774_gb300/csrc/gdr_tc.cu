@@ -71,9 +71,10 @@ struct alignas(16) LinShared {
   uint64_t bar_kq, bar_v, bar_mma;
   uint32_t tmem_base;
   int abort_flag;
-  float gam2[kBmax];  // gamma_t * log2(e)
-  float Gam[kBmax];   // exp(gamma_t)
-  float beta[kBmax];
+  // 16-byte aligned: read as float4 broadcasts
+  alignas(16) float gam2[kBmax];  // gamma_t * log2(e)
+  alignas(16) float Gam[kBmax];   // exp(gamma_t)
+  alignas(16) float beta[kBmax];
 };
 
 struct LinMaps {
