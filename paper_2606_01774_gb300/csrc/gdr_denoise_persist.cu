@@ -31,8 +31,9 @@
 // a 64 KiB buffer that is free again as soon as it has been turned into the
 // bf16 S0^T operand, so the next item's state streams in during this item's
 // products, solve and readout; the next keys and queries follow this item's
-// first MMA, the next values its solve, the next gates and slot one item
-// ahead into registers.  A bad slot is flagged in the device status word and
+// first MMA, the next values its second CTA barrier, the next gates and slot
+// one item ahead into registers.  Three CTA barriers per item (S0^T written,
+// A^T and M2 written, delta^T written); every other wait is a thread's own.  A bad slot is flagged in the device status word and
 // the item skipped (its output untouched).  Every wait is bounded: on a
 // timeout the CTA sets FLARE_DEV_WAIT_TIMEOUT, waits (bounded) for its copies
 // and MMAs in flight, frees its tensor memory and exits.
@@ -56,15 +57,14 @@ struct DpCfg {
   static constexpr int kAT = BM * kATs * 4;     // A^T[i][t] = A[t][i]
   static constexpr int kV = 2 * BM * 128;       // values: 2 chunks of BM rows x 128 B
   static constexpr int kG0 = 128 - 2 * BM;      // lane of G's first row
-  // the values, then A^T; the Gram MMA's A operand starts kG0 rows ahead of
-  // the [K;Q] tile and reads those bytes here (their rows reach no lane that
-  // is read)
-  static constexpr int kR0 = kAT > kV ? kAT : kV;
-  static constexpr int kR1 = kR0 > kG0 * 128 ? kR0 : kG0 * 128;
-  static constexpr int kR = (kR1 + 1023) / 1024 * 1024;
+  // the Gram MMA's A operand starts kG0 rows ahead of the [K;Q] tile and
+  // reads those bytes from the value and A^T buffers (their rows reach no
+  // lane that is read): A^T's buffer is padded so that the two cover them
+  static constexpr int kATb0 = (kAT + 1023) / 1024 * 1024;
+  static constexpr int kATb = kV + kATb0 >= kG0 * 128 ? kATb0 : kG0 * 128 - kV;
   static constexpr int kKQ = 2 * 2 * BM * 128;  // 2 chunks of [K;Q]: 2BM rows x 128 B (SW128)
   static constexpr int kM2 = BM * 128;          // M2 [l][i], K-major, SW128
-  static constexpr int kSmem = kS0 + kR + kKQ + kM2;
+  static constexpr int kSmem = kS0 + kV + kATb + kKQ + kM2;
 };
 
 struct alignas(16) DpShared {
@@ -82,17 +82,6 @@ struct DpMaps {
   CUtensorMap q;
   CUtensorMap v;  // (128, Hv, B, R) box (64, 1, BM, 1), no swizzle
 };
-
-__device__ __forceinline__ bool dp_wait(uint64_t* bar, uint32_t parity, DpShared& sh,
-                                        int32_t* status) {
-  const bool ok = tc::mbar_wait(bar, parity, &sh.abort_flag);
-  const bool all = __syncthreads_and(ok);
-  if (!all && threadIdx.x == 0 && !sh.abort_flag) {
-    sh.abort_flag = 1;
-    flag(status, FLARE_DEV_WAIT_TIMEOUT);
-  }
-  return all;
-}
 
 // The next item at or after `it` (stride gridDim.x) with a valid slot; bad
 // slots are flagged and skipped.  Called by every thread with the same
@@ -136,13 +125,16 @@ __global__ void __launch_bounds__(kDpThreads, 2)
   using C = DpCfg<BM>;
   constexpr int kATs = C::kATs;
   constexpr int kG0 = C::kG0;
+  // one thread of warp 1 issues every copy and MMA: warp 0 scans the gates,
+  // warps 2-3 turn G into A^T and M2
+  constexpr int kIssuer = 32;
   extern __shared__ uint8_t smem_raw[];
   __shared__ DpShared sh;
   uint8_t* base = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   float* S0s = reinterpret_cast<float*>(base);
-  uint8_t* Rs = base + C::kS0;  // the values, then A^T
-  float* AT = reinterpret_cast<float*>(Rs);
-  uint8_t* KQs = Rs + C::kR;
+  uint8_t* Vs = base + C::kS0;
+  float* AT = reinterpret_cast<float*>(Vs + C::kV);
+  uint8_t* KQs = Vs + C::kV + C::kATb;
   uint8_t* M2s = KQs + C::kKQ;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -154,7 +146,7 @@ __global__ void __launch_bounds__(kDpThreads, 2)
   int it = dp_next(p, blockIdx.x, total, slot);
   if (it < 0) return;  // the same answer on every thread
 
-  if (tid == 0) {
+  if (tid == kIssuer) {
     sh.abort_flag = 0;
     tc::mbar_init(&sh.bar_s0, 1);
     tc::mbar_init(&sh.bar_kq, 1);
@@ -192,8 +184,8 @@ __global__ void __launch_bounds__(kDpThreads, 2)
   auto issue_v = [&](int item) {
     const int r = item / p.Hv, j = item % p.Hv;
     tc::mbar_expect_tx(&sh.bar_v, C::kV);
-    tc::tma_load_4d(Rs, &maps.v, &sh.bar_v, 0, j, 0, r);
-    tc::tma_load_4d(Rs + BM * 128, &maps.v, &sh.bar_v, 64, j, 0, r);
+    tc::tma_load_4d(Vs, &maps.v, &sh.bar_v, 0, j, 0, r);
+    tc::tma_load_4d(Vs + BM * 128, &maps.v, &sh.bar_v, 64, j, 0, r);
   };
   // warp 0 holds the gates of the item it processes next, loaded one item ahead
   float gq = 0.f, bq = 0.f;
@@ -204,11 +196,11 @@ __global__ void __launch_bounds__(kDpThreads, 2)
   };
   auto cand_slot = [&](int c) { return c < total ? p.state_slot[c / p.Hv] : -1; };
 
-  // thread 0's record of what is in flight (and the parity its barrier
+  // the issuing thread's record of what is in flight (and the parity its barrier
   // phase completes with), for a clean exit after a timeout
   bool s0_out = false, kq_out = false, v_out = false, mma_out = false;
   uint32_t s0_par = 0, kq_par = 0, v_par = 0;
-  if (tid == 0) {
+  if (tid == kIssuer) {
     tc::prefetch_tmap(&maps.k);
     tc::prefetch_tmap(&maps.q);
     tc::prefetch_tmap(&maps.v);
@@ -220,6 +212,7 @@ __global__ void __launch_bounds__(kDpThreads, 2)
   if (warp == 0) load_gates(it);
   int cand = it + gridDim.x;
   int cs = cand_slot(cand);
+  bool bad = false;     // this thread gave up on a wait
   uint32_t ph = 0;      // parity of the item's loads
   uint32_t ph_mma = 0;  // parity of the next MMA completion (two per item)
   const uint32_t idG = tc::idesc_bf16(128, Bp, false, false);
@@ -258,8 +251,10 @@ __global__ void __launch_bounds__(kDpThreads, 2)
       cs = cand_slot(cand);
     }
 
-    if (!dp_wait(&sh.bar_s0, ph, sh, p.dev_status)) break;
-    if (tid == 0) s0_out = false;
+    // Waits on a copy or an MMA are per thread: a thread that gives up
+    // carries `bad` to the next CTA barrier, where the whole CTA stops.
+    bad |= !tc::mbar_wait(&sh.bar_s0, ph, &sh.abort_flag);
+    if (tid == kIssuer) s0_out = false;
     // S0^T (column c = tid of S0) into tensor memory as bf16 pairs
 #pragma unroll 1
     for (int i0 = 0; i0 < kDpD; i0 += 32) {
@@ -271,9 +266,8 @@ __global__ void __launch_bounds__(kDpThreads, 2)
     }
     tc::tmem_st_wait();
     tc::fence_before_sync();
-    if (!dp_wait(&sh.bar_kq, ph, sh, p.dev_status)) break;  // also: the state buffer read
-    if (tid == 0) {
-      kq_out = false;
+    if (__syncthreads_or(bad)) break;  // S0^T complete, the state buffer read
+    if (tid == kIssuer) {
       // the state buffer is free: the next item's state streams in during
       // this item's products, solve and readout
       if (it_next >= 0) {
@@ -281,6 +275,8 @@ __global__ void __launch_bounds__(kDpThreads, 2)
         s0_out = true;
         s0_par = ph ^ 1u;
       }
+      bad |= !tc::mbar_wait(&sh.bar_kq, ph, &sh.abort_flag);
+      kq_out = false;
       tc::fence_after_sync();
 #pragma unroll
       for (int kk = 0; kk < kDpD / 16; ++kk) {
@@ -293,22 +289,22 @@ __global__ void __launch_bounds__(kDpThreads, 2)
       tc::mma_commit(&sh.bar_mma);
       mma_out = true;
     }
-    if (!dp_wait(&sh.bar_v, ph, sh, p.dev_status)) break;
-    if (tid == 0) v_out = false;
+    bad |= !tc::mbar_wait(&sh.bar_v, ph, &sh.abort_flag);
+    if (tid == kIssuer) v_out = false;
     // this column of the values as bf16 pairs (rows past B arrive as zeros)
     uint32_t vpk[BM / 2];
     {
-      const uint8_t* vb = Rs + (tid >> 6) * (BM * 128) + (tid & 63) * 2;
+      const uint8_t* vb = Vs + (tid >> 6) * (BM * 128) + (tid & 63) * 2;
 #pragma unroll
       for (int t2 = 0; t2 < BM / 2; ++t2)
         vpk[t2] = (uint32_t)*reinterpret_cast<const unsigned short*>(vb + (2 * t2) * 128) |
                   ((uint32_t)*reinterpret_cast<const unsigned short*>(vb + (2 * t2 + 1) * 128)
                    << 16);
     }
-    if (!dp_wait(&sh.bar_mma, ph_mma, sh, p.dev_status)) break;  // also: the values read
+    bad |= !tc::mbar_wait(&sh.bar_mma, ph_mma, &sh.abort_flag);
     ph_mma ^= 1u;
     tc::fence_after_sync();
-    if (tid == 0) {
+    if (tid == kIssuer) {
       mma_out = false;
       if (it_next >= 0) {  // the first MMA, the only reader of [K;Q], is done
         issue_kq(it_next);
@@ -369,8 +365,17 @@ __global__ void __launch_bounds__(kDpThreads, 2)
         }
       }
     }
+    // the readout's scale, read here: the gates' buffer is rewritten for the
+    // next item once every thread is past the barrier before the second MMA
+    const float sG = p.scale * sh.Gam[B - 1];
     tc::fence_before_sync();
-    __syncthreads();  // A^T and M2 published; W^T's key part and G read
+    if (__syncthreads_or(bad)) break;  // A^T and M2 published; the values, W^T's key part and G read
+    if (tid == kIssuer && it_next >= 0) {
+      tc::fence_async_smem();
+      issue_v(it_next);
+      v_out = true;
+      v_par = ph ^ 1u;
+    }
 
     // (I + A) delta = X, right-looking (A^T row t as 16-byte broadcast loads);
     // rows past B touch only rows past B (A^T is zero there)
@@ -404,14 +409,8 @@ __global__ void __launch_bounds__(kDpThreads, 2)
     }
     tc::tmem_st_wait();
     tc::fence_before_sync();
-    __syncthreads();  // also: A^T read, its region free for the next values
-    if (tid == 0) {
-      if (it_next >= 0) {
-        tc::fence_async_smem();
-        issue_v(it_next);
-        v_out = true;
-        v_par = ph ^ 1u;
-      }
+    if (__syncthreads_or(bad)) break;  // delta^T complete; A^T read
+    if (tid == kIssuer) {
       tc::fence_after_sync();
       for (int kk = 0; kk < Bp / 16; ++kk)
         tc::mma_bf16_ts(tmG, tmS + kk * 8, tc::sdesc_sw128(tc::smem_u32(M2s + kk * 32), 16, 1024),
@@ -419,14 +418,13 @@ __global__ void __launch_bounds__(kDpThreads, 2)
       tc::mma_commit(&sh.bar_mma);
       mma_out = true;
     }
-    if (!dp_wait(&sh.bar_mma, ph_mma, sh, p.dev_status)) break;
+    bad |= !tc::mbar_wait(&sh.bar_mma, ph_mma, &sh.abort_flag);
     ph_mma ^= 1u;
     tc::fence_after_sync();
-    if (tid == 0) mma_out = false;
+    if (tid == kIssuer) mma_out = false;
     // out[l][c] = s (Gam_{B-1} W^T[c][BM + l] + O2^T[c][l]); adjacent lanes
     // swap one value so that each stores a bf16 pair of two columns
     {
-      const float sG = p.scale * sh.Gam[B - 1];
       uint32_t o2[BM], wq[BM];
 #pragma unroll
       for (int c0 = 0; c0 < BM; c0 += 16) {
@@ -453,10 +451,16 @@ __global__ void __launch_bounds__(kDpThreads, 2)
     slot = slot_next;
     ph ^= 1u;
   }
+  bad = __syncthreads_or(bad);
+  if (bad && tid == 0 && !sh.abort_flag) {
+    sh.abort_flag = 1;
+    flag(p.dev_status, FLARE_DEV_WAIT_TIMEOUT);
+  }
+  __syncthreads();
 
   // after a timeout: let the copies and MMAs in flight land before the
   // shared and tensor memory are given up (bounded waits)
-  if (tid == 0 && sh.abort_flag) {
+  if (tid == kIssuer && bad) {
     if (s0_out) tc::mbar_wait(&sh.bar_s0, s0_par, nullptr, 100000000ull);
     if (kq_out) tc::mbar_wait(&sh.bar_kq, kq_par, nullptr, 100000000ull);
     if (v_out) tc::mbar_wait(&sh.bar_v, v_par, nullptr, 100000000ull);
