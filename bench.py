@@ -146,9 +146,16 @@ def verify_commit_bytes(spec, verify_len, accept):
 # ---------------------------------------------------------------- ncu traffic
 
 
-KERNEL_OF = {"linear": "gdr_denoise_tc_kernel", "softmax": "softmax_tc_kernel",
-             "commit": "gdr_commit_kernel", "shortconv": "short_conv_kernel",
-             "shortconv_commit": "short_conv_kernel"}
+def kernel_of_call(spec):
+    """The kernel each layer call of `spec` runs (the library's dispatch: bf16
+    128 x 128 states take the persistent denoise kernel for B <= 32 and the
+    tensor-core commit; other shapes the one-CTA-per-item kernels)."""
+    tc_state = spec.act_dtype == "bf16" and spec.head_dim_k == 128 and spec.head_dim_v == 128
+    return {"linear": ("gdr_denoise_persist_kernel" if tc_state and spec.block_len <= 32
+                       else "gdr_denoise_tc_kernel"),
+            "softmax": "softmax_tc_kernel",
+            "commit": "gdr_commit_tc_kernel" if tc_state else "gdr_commit_kernel",
+            "shortconv": "short_conv_kernel", "shortconv_commit": "short_conv_kernel"}
 VERIFY_KERNEL_OF = {"linear": "gdr_commit_kernel", "softmax": "softmax_tc_kernel",
                     "commit": "verify_commit_kernel"}
 
@@ -765,7 +772,7 @@ def summarise(fr, per, timed_s, clk):
                 "peak": peaks["hbm_gbs"], "unit": "GB/s"}
         peak_source = f"{peaks['source']} (hbm_gbs)"
     roof["frac"] = roof["achieved"] / roof["peak"]
-    kernel_of = VERIFY_KERNEL_OF if fr.verify else KERNEL_OF
+    kernel_of = VERIFY_KERNEL_OF if fr.verify else kernel_of_call(s)
     roof["traffic"] = profiled_traffic(kernel_of[dom], s.name) if dom in kernel_of else None
     roof["kernel"] = kd["kernel"]
     roof["peak_source"] = peak_source
