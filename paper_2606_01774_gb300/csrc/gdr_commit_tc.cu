@@ -83,6 +83,7 @@ struct alignas(16) CtShared {
   alignas(16) float gam2[64];  // gamma_t log2(e)
   alignas(16) float Gam[64];   // exp(gamma_t)
   alignas(16) float beta[64];
+  alignas(16) float dsc[64];   // exp(gamma_{n-1} - gamma_t) for t < n, else 0 (delta' factor)
 };
 
 __device__ __forceinline__ bool ct_wait(uint64_t* bar, uint32_t parity, CtShared& sh,
@@ -245,12 +246,19 @@ __global__ void __launch_bounds__(kCtThreads, 2)
         }
       }
       g1 += __shfl_sync(0xffffffffu, g0, 31);
-      sh.gam2[lane] = g0 * 1.4426950408889634f;
-      sh.gam2[lane + 32] = g1 * 1.4426950408889634f;
+      const float g20 = g0 * 1.4426950408889634f, g21 = g1 * 1.4426950408889634f;
+      // gamma_{n-1}: lane (n - 1) % 32 of the half holding it
+      const float gn0 = __shfl_sync(0xffffffffu, g20, (n - 1) & 31);
+      const float gn1 = __shfl_sync(0xffffffffu, g21, (n - 1) & 31);
+      const float gn2 = n > 32 ? gn1 : gn0;
+      sh.gam2[lane] = g20;
+      sh.gam2[lane + 32] = g21;
       sh.Gam[lane] = expf(g0);
       sh.Gam[lane + 32] = expf(g1);
       sh.beta[lane] = bq0;
       sh.beta[lane + 32] = bq1;
+      sh.dsc[lane] = lane < n ? tc::ex2(gn2 - g20) : 0.f;
+      sh.dsc[lane + 32] = lane + 32 < n ? tc::ex2(gn2 - g21) : 0.f;
     }
     // the next item: the candidate when it is valid and has n > 0, else the
     // first such item after it (bad ones flagged on the way)
@@ -338,12 +346,22 @@ __global__ void __launch_bounds__(kCtThreads, 2)
         tc::tmem_ld16(tmG + lane_off + c0, *reinterpret_cast<uint32_t(*)[16]>(&gr[c0]));
       tc::tmem_ld_wait();
       if (t >= 0) {
+        // the log-gates go to registers first (16-byte loads) and every
+        // exponential is taken unconditionally, the mask applied as a
+        // select: a branch per element would serialise the chains
+        float g2r[BM];
+#pragma unroll
+        for (int i4 = 0; i4 < BM / 4; ++i4) {
+          const float4 q = *reinterpret_cast<const float4*>(&sh.gam2[4 * i4]);
+          g2r[4 * i4] = q.x, g2r[4 * i4 + 1] = q.y, g2r[4 * i4 + 2] = q.z, g2r[4 * i4 + 3] = q.w;
+        }
         const float bt = sh.beta[t], gt = sh.gam2[t];
         const bool live = t < n;
 #pragma unroll
-        for (int i = 0; i < BM; ++i)
-          AT[i * kATs + t] =
-              (live && i < t) ? bt * tc::ex2(gt - sh.gam2[i]) * __uint_as_float(gr[i]) : 0.f;
+        for (int i = 0; i < BM; ++i) {
+          const float a = bt * tc::ex2(gt - g2r[i]) * __uint_as_float(gr[i]);
+          AT[i * kATs + t] = (live && i < t) ? a : 0.f;
+        }
       }
     }
     // X = diag(beta) (V - diag(Gam) W) for this thread's column
@@ -392,7 +410,12 @@ __global__ void __launch_bounds__(kCtThreads, 2)
     }
     // delta'_t = exp(gamma_{n-1} - gamma_t) delta_t (t < n), as bf16 hi and lo parts
     {
-      const float gn2 = sh.gam2[n - 1];
+      float dr[BM];
+#pragma unroll
+      for (int i4 = 0; i4 < BM / 4; ++i4) {
+        const float4 q = *reinterpret_cast<const float4*>(&sh.dsc[4 * i4]);
+        dr[4 * i4] = q.x, dr[4 * i4 + 1] = q.y, dr[4 * i4 + 2] = q.z, dr[4 * i4 + 3] = q.w;
+      }
 #pragma unroll
       for (int c0 = 0; c0 < C::kDP; c0 += 16) {
         uint32_t hi[16], lo[16];
@@ -401,8 +424,9 @@ __global__ void __launch_bounds__(kCtThreads, 2)
           const int t = 2 * (c0 + e);
           float a = 0.f, b = 0.f;
           if (t < BM) {
-            a = t < n ? x[t] * tc::ex2(gn2 - sh.gam2[t]) : 0.f;
-            b = t + 1 < n ? x[t + 1] * tc::ex2(gn2 - sh.gam2[t + 1]) : 0.f;
+            const float xa = x[t] * dr[t], xb = x[t + 1] * dr[t + 1];
+            a = t < n ? xa : 0.f;
+            b = t + 1 < n ? xb : 0.f;
           }
           split_pair(a, b, hi[e], lo[e]);
         }

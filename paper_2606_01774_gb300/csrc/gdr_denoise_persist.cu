@@ -75,6 +75,7 @@ struct alignas(16) DpShared {
   alignas(16) float gam2[32];  // gamma_t log2(e)
   alignas(16) float Gam[32];   // exp(gamma_t)
   alignas(16) float beta[32];
+  alignas(16) float eB[32];    // exp(gamma_{B-1} - gamma_i) for i < B, else 0 (the M2 row factor)
 };
 
 struct DpMaps {
@@ -230,9 +231,12 @@ __global__ void __launch_bounds__(kDpThreads, 2)
         const float a = __shfl_up_sync(0xffffffffu, g, o);
         if (lane >= o) g += a;
       }
-      sh.gam2[lane] = g * 1.4426950408889634f;
+      const float g2 = g * 1.4426950408889634f;
+      const float gB2 = __shfl_sync(0xffffffffu, g2, B - 1);
+      sh.gam2[lane] = g2;
       sh.Gam[lane] = expf(g);
       sh.beta[lane] = bq;
+      sh.eB[lane] = lane < B ? tc::ex2(gB2 - g2) : 0.f;
     }
     // the next item: the candidate when its slot is valid, else the first
     // valid one after it (bad ones flagged on the way)
@@ -320,24 +324,40 @@ __global__ void __launch_bounds__(kDpThreads, 2)
         tc::tmem_ld16(tmG + lane_off + c0, *reinterpret_cast<uint32_t(*)[16]>(&gr[c0]));
       tc::tmem_ld_wait();
       const int row = tid - kG0;
+      // the gate factors go to registers first (16-byte loads) and every
+      // exponential is taken unconditionally, the masks applied as selects:
+      // a branch per element would serialise the load / exponential chains
       if (row >= 0 && row < BM) {
         const int t = row;
+        float g2r[BM];
+#pragma unroll
+        for (int i4 = 0; i4 < BM / 4; ++i4) {
+          const float4 q = *reinterpret_cast<const float4*>(&sh.gam2[4 * i4]);
+          g2r[4 * i4] = q.x, g2r[4 * i4 + 1] = q.y, g2r[4 * i4 + 2] = q.z, g2r[4 * i4 + 3] = q.w;
+        }
         const float bt = sh.beta[t], gt = sh.gam2[t];
         const bool live = t < B;
 #pragma unroll
-        for (int i = 0; i < BM; ++i)
-          AT[i * kATs + t] =
-              (live && i < t) ? bt * tc::ex2(gt - sh.gam2[i]) * __uint_as_float(gr[i]) : 0.f;
+        for (int i = 0; i < BM; ++i) {
+          const float a = bt * tc::ex2(gt - g2r[i]) * __uint_as_float(gr[i]);
+          AT[i * kATs + t] = (live && i < t) ? a : 0.f;
+        }
       } else if (row >= BM) {
         const int l = row - BM;
-        const float gB = sh.gam2[B - 1];
+        float er[BM];
+#pragma unroll
+        for (int i4 = 0; i4 < BM / 4; ++i4) {
+          const float4 q = *reinterpret_cast<const float4*>(&sh.eB[4 * i4]);
+          er[4 * i4] = q.x, er[4 * i4 + 1] = q.y, er[4 * i4 + 2] = q.z, er[4 * i4 + 3] = q.w;
+        }
 #pragma unroll
         for (int c0 = 0; c0 < BM; c0 += 16) {
           float v[16];
 #pragma unroll
           for (int e = 0; e < 16; ++e) {
             const int i = c0 + e;
-            v[e] = (i < B && l < B) ? tc::ex2(gB - sh.gam2[i]) * __uint_as_float(gr[i]) : 0.f;
+            const float m = er[i] * __uint_as_float(gr[i]);
+            v[e] = (i < B && l < B) ? m : 0.f;
           }
           dp_store16_sw128(M2s, l, c0, v);
         }

@@ -290,8 +290,10 @@ __global__ void __launch_bounds__(kLinThreads, LinCfg<DK, DV, BM>::kMinBlocks)
 #pragma unroll
         for (int e = 0; e < 16; ++e) {
           const int i = c0 + e;
-          // A[t][i] = beta_t exp(gamma_t - gamma_i) (k_t . k_i), i < t < B
-          v[e] = (i < row && row < B) ? bt * tc::ex2(gt - g2[e]) * __uint_as_float(gr[i]) : 0.f;
+          // A[t][i] = beta_t exp(gamma_t - gamma_i) (k_t . k_i), i < t < B (the
+          // exponential taken unconditionally, the mask as a select)
+          const float a = bt * tc::ex2(gt - g2[e]) * __uint_as_float(gr[i]);
+          v[e] = (i < row && row < B) ? a : 0.f;
         }
 #pragma unroll
         for (int e = 0; e < 16; ++e) AT[(c0 + e) * kATs + row] = v[e];
@@ -299,7 +301,8 @@ __global__ void __launch_bounds__(kLinThreads, LinCfg<DK, DV, BM>::kMinBlocks)
 #pragma unroll
         for (int e = 0; e < 16; ++e) {
           const int i = c0 + e;
-          v[e] = (i < B && row < B) ? tc::ex2(gB - g2[e]) * __uint_as_float(gr[i]) : 0.f;
+          const float m = tc::ex2(gB - g2[e]) * __uint_as_float(gr[i]);
+          v[e] = (i < B && row < B) ? m : 0.f;
         }
         store16_sw128(M2s, row, c0, v);
       }
