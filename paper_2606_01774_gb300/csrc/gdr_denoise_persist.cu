@@ -68,7 +68,7 @@ struct DpCfg {
 };
 
 struct alignas(16) DpShared {
-  uint64_t bar_s0, bar_kq, bar_v, bar_mma;
+  uint64_t bar_s0, bar_kq, bar_v, bar_g, bar_mma;
   uint32_t tmem_base;
   int abort_flag;
   // 16-byte aligned: read as float4 broadcasts
@@ -152,6 +152,7 @@ __global__ void __launch_bounds__(kDpThreads, 2)
     tc::mbar_init(&sh.bar_s0, 1);
     tc::mbar_init(&sh.bar_kq, 1);
     tc::mbar_init(&sh.bar_v, 1);
+    tc::mbar_init(&sh.bar_g, 1);
     tc::mbar_init(&sh.bar_mma, 1);
     tc::fence_mbar_init();
   }
@@ -168,10 +169,7 @@ __global__ void __launch_bounds__(kDpThreads, 2)
   auto issue_s0 = [&](int item, int s) {
     const float* src = p.state_pool + ((size_t)s * p.Hv + item % p.Hv) * kDpD * kDpD;
     tc::mbar_expect_tx(&sh.bar_s0, C::kS0);
-#pragma unroll
-    for (int q = 0; q < 4; ++q)
-      tc::bulk_load(S0s + q * (kDpD * kDpD / 4), src + q * (kDpD * kDpD / 4), C::kS0 / 4,
-                    &sh.bar_s0);
+    tc::bulk_load(S0s, src, C::kS0, &sh.bar_s0);
   };
   auto issue_kq = [&](int item) {
     const int r = item / p.Hv, h = (item % p.Hv) / (p.Hv / p.Hk);
@@ -272,26 +270,34 @@ __global__ void __launch_bounds__(kDpThreads, 2)
     tc::fence_before_sync();
     if (__syncthreads_or(bad)) break;  // S0^T complete, the state buffer read
     if (tid == kIssuer) {
+      bad |= !tc::mbar_wait(&sh.bar_kq, ph, &sh.abort_flag);
+      kq_out = false;
+      tc::fence_after_sync();
+      // the Gram first, committed on its own: A^T and M2 are built while the
+      // state products run
+#pragma unroll
+      for (int kk = 0; kk < kDpD / 16; ++kk) {
+        const uint8_t* kc = KQs + (kk >> 2) * (2 * BM * 128) + (kk & 3) * 32;
+        tc::mma_bf16_ss(tmG, tc::sdesc_sw128(tc::smem_u32(kc - kG0 * 128), 16, 1024),
+                        tc::sdesc_sw128(tc::smem_u32(kc), 16, 1024), idG, kk > 0);  // G = [K;Q] K^T
+      }
+      tc::mma_commit(&sh.bar_g);
+#pragma unroll
+      for (int kk = 0; kk < kDpD / 16; ++kk) {
+        const uint8_t* kc = KQs + (kk >> 2) * (2 * BM * 128) + (kk & 3) * 32;
+        tc::mma_bf16_ts(tmW, tmS + kk * 8, tc::sdesc_sw128(tc::smem_u32(kc), 16, 1024), idW,
+                        kk > 0);  // W^T = S0^T [K;Q]^T
+      }
+      tc::mma_commit(&sh.bar_mma);
+      mma_out = true;
       // the state buffer is free: the next item's state streams in during
-      // this item's products, solve and readout
+      // this item's products, solve and readout (issued after the MMAs, off
+      // their path)
       if (it_next >= 0) {
         issue_s0(it_next, slot_next);
         s0_out = true;
         s0_par = ph ^ 1u;
       }
-      bad |= !tc::mbar_wait(&sh.bar_kq, ph, &sh.abort_flag);
-      kq_out = false;
-      tc::fence_after_sync();
-#pragma unroll
-      for (int kk = 0; kk < kDpD / 16; ++kk) {
-        const uint8_t* kc = KQs + (kk >> 2) * (2 * BM * 128) + (kk & 3) * 32;
-        const uint64_t kd = tc::sdesc_sw128(tc::smem_u32(kc), 16, 1024);
-        const uint64_t kg = tc::sdesc_sw128(tc::smem_u32(kc - kG0 * 128), 16, 1024);
-        tc::mma_bf16_ss(tmG, kg, kd, idG, kk > 0);            // G = [K;Q] K^T
-        tc::mma_bf16_ts(tmW, tmS + kk * 8, kd, idW, kk > 0);  // W^T = S0^T [K;Q]^T
-      }
-      tc::mma_commit(&sh.bar_mma);
-      mma_out = true;
     }
     bad |= !tc::mbar_wait(&sh.bar_v, ph, &sh.abort_flag);
     if (tid == kIssuer) v_out = false;
@@ -305,19 +311,11 @@ __global__ void __launch_bounds__(kDpThreads, 2)
                   ((uint32_t)*reinterpret_cast<const unsigned short*>(vb + (2 * t2 + 1) * 128)
                    << 16);
     }
-    bad |= !tc::mbar_wait(&sh.bar_mma, ph_mma, &sh.abort_flag);
-    ph_mma ^= 1u;
-    tc::fence_after_sync();
-    if (tid == kIssuer) {
-      mma_out = false;
-      if (it_next >= 0) {  // the first MMA, the only reader of [K;Q], is done
-        issue_kq(it_next);
-        kq_out = true;
-        kq_par = ph ^ 1u;
-      }
-    }
-    // A^T (key rows of G) and M2 (query rows), from the lanes that hold G
+    // A^T (key rows of G) and M2 (query rows), from the lanes that hold G,
+    // once the Gram is in
     if (warp >= kG0 / 32) {
+      bad |= !tc::mbar_wait(&sh.bar_g, ph, &sh.abort_flag);
+      tc::fence_after_sync();
       uint32_t gr[BM];
 #pragma unroll
       for (int c0 = 0; c0 < BM; c0 += 16)
@@ -362,6 +360,17 @@ __global__ void __launch_bounds__(kDpThreads, 2)
           dp_store16_sw128(M2s, l, c0, v);
         }
         tc::fence_async_smem();  // M2 is the second MMA's operand
+      }
+    }
+    bad |= !tc::mbar_wait(&sh.bar_mma, ph_mma, &sh.abort_flag);
+    ph_mma ^= 1u;
+    tc::fence_after_sync();
+    if (tid == kIssuer) {
+      mma_out = false;
+      if (it_next >= 0) {  // the first MMAs, the only readers of [K;Q], are done
+        issue_kq(it_next);
+        kq_out = true;
+        kq_par = ph ^ 1u;
       }
     }
     // X = diag(beta) (V - diag(Gam) K S0) for this column
