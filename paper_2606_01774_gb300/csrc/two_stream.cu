@@ -348,7 +348,7 @@ int two_stream_chunk_len() { return kTsChunk; }
 cudaError_t launch_two_stream_fwd(const TwoStreamParams& p, bool bf16, cudaStream_t stream) {
   if (p.N == 0) return cudaSuccess;
   // bf16 activations take the tensor-core kernel (two_stream_tc.cu)
-  if (bf16 && two_stream_tc_supported(p.B, p.dk, p.dv)) return launch_two_stream_tc(p, stream);
+  if (bf16 && two_stream_chunk_supported(p.B, p.dk, p.dv)) return launch_two_stream_chunk(p, stream);
   return bf16 ? launch_ts_d<__nv_bfloat16>(p, stream) : launch_ts_d<float>(p, stream);
 }
 
