@@ -25,16 +25,17 @@
 //                                         chunk needs (K K^T, K K~^T, K Q~^T, K~ K~^T, K~ Q~^T)
 //   solve  (I + A) delta = X             fp32, per column, right-looking (warps 0-3)
 //   MMA 2  C^T = delta^T P               M=128 (c), N=128, K=64    (A: delta^T bf16, tensor memory)
-//   noisy  S_(m)^T y = Gam_{mB-1} W^T + C^T, the B x B solves and the readouts (warps 4-7)
+//   noisy  S_(m)^T y = Gam_{mB-1} W^T + C^T, the B x B solves and the readouts (both groups)
 // bf16 operands and fp32 accumulation throughout (the state rounded to bf16
 // for its products, as in the denoise kernels).
 //
 // Persistent CTAs, one per SM (208 KiB of shared memory, 448 tensor-memory
 // columns), 256 threads: warps 0-3 and 4-7 are two groups on the same 128
-// lanes.  The next chunk's state streams into the state buffer as soon as it
+// lanes, which build the tables together and take half of the noisy tokens
+// each.  The next chunk's state streams into the state buffer as soon as it
 // has been turned into S0^T, its keys and queries once the first MMAs are
-// done, its values after the tables of this chunk are built; its gates are
-// loaded into registers one chunk ahead.  Every wait is bounded: on a timeout
+// done, its values once this chunk's are read; its gates are loaded into
+// registers one chunk ahead.  Every wait is bounded: on a timeout
 // the CTA sets FLARE_DEV_WAIT_TIMEOUT, waits (bounded) for its copies and
 // MMAs in flight, frees its tensor memory and exits.
 #include <cudaTypedefs.h>
@@ -89,9 +90,6 @@ __device__ __forceinline__ uint32_t ck_pack(float a, float b) {
   __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
   return *reinterpret_cast<uint32_t*>(&h);
 }
-
-__device__ __forceinline__ float ck_bf_lo(uint32_t u) { return __uint_as_float(u << 16); }
-__device__ __forceinline__ float ck_bf_hi(uint32_t u) { return __uint_as_float(u & 0xffff0000u); }
 
 // 64 table values of one row, 16-byte stores
 __device__ __forceinline__ void ck_store_row(float* row, const float (&v)[kCkC]) {
@@ -296,18 +294,6 @@ __global__ void __launch_bounds__(kCkThreads, 1)
         s0_par = ph ^ 1u;
       }
     }
-    bad |= !tc::mbar_wait(&sh.bar_v, ph, &sh.abort_flag);
-    if (tid == kIssuer) v_out = false;
-    // this column of the clean (group 0) or noisy (group 1) values, bf16 pairs
-    uint32_t vpk[kCkC / 2];
-    {
-      const uint8_t* vb = (grp == 0 ? Vc : Vn) + (col >> 6) * (kCkC * 128) + (col & 63) * 2;
-#pragma unroll
-      for (int t2 = 0; t2 < kCkC / 2; ++t2)
-        vpk[t2] = (uint32_t)*reinterpret_cast<const unsigned short*>(vb + (2 * t2) * 128) |
-                  ((uint32_t)*reinterpret_cast<const unsigned short*>(vb + (2 * t2 + 1) * 128)
-                   << 16);
-    }
     bad |= !tc::mbar_wait(&sh.bar_mma, ph_mma, &sh.abort_flag);
     ph_mma ^= 1u;
     tc::fence_after_sync();
@@ -396,33 +382,23 @@ __global__ void __launch_bounds__(kCkThreads, 1)
         }
       }
     }
-    // ---- group 0: X = diag(beta) (V - diag(Gam) K S0); group 1: the part of
-    // the noisy X and of the query products that does not need delta
+    // ---- group 0: X = diag(beta) (V - diag(Gam) K S0)
+    bad |= !tc::mbar_wait(&sh.bar_v, ph, &sh.abort_flag);
+    if (tid == kIssuer) v_out = false;
     float x[kCkC];
-    {
+    if (grp == 0) {
       uint32_t w[kCkC];
-      ck_ld64(tmW + lane_off + (grp == 0 ? 0 : 64), w);
+      ck_ld64(tmW + lane_off, w);
+      const uint8_t* vb = Vc + (col >> 6) * (kCkC * 128) + (col & 63) * 2;
 #pragma unroll
       for (int t = 0; t < kCkC; ++t) {
-        const uint32_t vp = vpk[t / 2];
-        const float vt = (t & 1) ? ck_bf_hi(vp) : ck_bf_lo(vp);
-        if (grp == 0) {
-          x[t] = sh.bc[t] * (vt - sh.Gc[t] * __uint_as_float(w[t]));
-        } else {
-          const int mb = t & ~(B - 1);
-          const float am = mb > 0 ? sh.Gc[mb - 1] : 1.f;  // Gam_{mB-1}
-          x[t] = sh.bn[t] * (vt - sh.Gn[t] * am * __uint_as_float(w[t]));
-        }
+        const float vt = __uint_as_float(
+            (uint32_t)*reinterpret_cast<const unsigned short*>(vb + t * 128) << 16);
+        x[t] = sh.bc[t] * (vt - sh.Gc[t] * __uint_as_float(w[t]));
       }
     }
     tc::fence_before_sync();
-    if (__syncthreads_or(bad)) break;  // the tables published; the values, W^T's key parts, G read
-    if (tid == kIssuer && it_next >= 0) {
-      tc::fence_async_smem();
-      issue_v(it_next);
-      v_out = true;
-      v_par = ph ^ 1u;
-    }
+    if (__syncthreads_or(bad)) break;  // the tables published; G read
 
     if (grp == 0) {
       // (I + A) delta = X, right-looking (A^T row t as 16-byte broadcast loads)
@@ -466,37 +442,58 @@ __global__ void __launch_bounds__(kCkThreads, 1)
     tc::fence_after_sync();
     if (tid == kIssuer) mma_out = false;
 
-    if (grp == 1) {
-      // ---- noisy blocks: X~ = (the part above) - beta~ Gam~ C^T[k~], the
-      // B x B solves, then o~_l = s (Gam~_end (Gam_{mB-1} W^T[q~] + C^T[q~]) + Aqk delta~)
+    // ---- noisy blocks, tokens 32 grp .. 32 grp + 31 of the chunk (whole
+    // blocks: B divides 32):
+    //   X~_t = beta~_t (v~_t - Gam~_t (Gam_{mB-1} W^T[k~_t] + C^T[k~_t])),
+    //   the B x B solves, then
+    //   o~_l = s (Gam~_end (Gam_{mB-1} W^T[q~_l] + C^T[q~_l]) + Aqk delta~)
+    {
+      constexpr int kH = kCkC / 2;
+      const int t0 = grp * kH;
+      float xn[kH];
       {
-        uint32_t cr[kCkC];
-        ck_ld64(tmG + lane_off, cr);  // C^T, noisy keys
+        uint32_t wk[16], ck[16];
+        const uint8_t* vb = Vn + (col >> 6) * (kCkC * 128) + (col & 63) * 2;
 #pragma unroll
-        for (int t = 0; t < kCkC; ++t) x[t] -= sh.bn[t] * sh.Gn[t] * __uint_as_float(cr[t]);
+        for (int c0 = 0; c0 < kH; c0 += 16) {
+          tc::tmem_ld16(tmW + lane_off + 64 + t0 + c0, wk);  // W^T, noisy keys
+          tc::tmem_ld16(tmG + lane_off + t0 + c0, ck);       // C^T, noisy keys
+          tc::tmem_ld_wait();
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            const int t = t0 + c0 + e;
+            const int mb = t & ~(B - 1);
+            const float am = mb > 0 ? sh.Gc[mb - 1] : 1.f;  // Gam_{mB-1}
+            const float vt = __uint_as_float(
+                (uint32_t)*reinterpret_cast<const unsigned short*>(vb + t * 128) << 16);
+            xn[c0 + e] = sh.bn[t] * (vt - sh.Gn[t] * (am * __uint_as_float(wk[e]) +
+                                                       __uint_as_float(ck[e])));
+          }
+        }
       }
+      // (I + A~) delta~ = X~ per block, forward substitution
 #pragma unroll
-      for (int t = 0; t < kCkC; ++t) {
-        const int m0 = t & ~(B - 1);  // compile-time: t is unrolled
-        const float* ar = An + t * kCkC + m0;
-        float acc = x[t];
-        if constexpr (B >= 4) {  // m0 is then a multiple of 4: 16-byte loads
+      for (int u = 0; u < kH; ++u) {
+        const int m0u = u & ~(B - 1);     // block start, local index (compile-time)
+        const float* ar = An + (t0 + u) * kCkC + t0 + m0u;
+        float acc = xn[u];
+        if constexpr (B >= 4) {  // (t0 + m0u) is then a multiple of 4: 16-byte loads
 #pragma unroll
           for (int i4 = 0; i4 < B / 4; ++i4) {
             const float4 a = reinterpret_cast<const float4*>(ar)[i4];
             const float av[4] = {a.x, a.y, a.z, a.w};
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
-              const int i = m0 + 4 * i4 + e;
-              if (i < t) acc = fmaf(-av[e], x[i], acc);
+              const int i = m0u + 4 * i4 + e;
+              if (i < u) acc = fmaf(-av[e], xn[i], acc);
             }
           }
         } else {
 #pragma unroll
           for (int e = 0; e < B; ++e)
-            if (m0 + e < t) acc = fmaf(-ar[e], x[m0 + e], acc);
+            if (m0u + e < u) acc = fmaf(-ar[e], xn[m0u + e], acc);
         }
-        x[t] = acc;
+        xn[u] = acc;
       }
       // readout; adjacent lanes swap one value so that each stores a bf16
       // pair of two columns
@@ -504,31 +501,43 @@ __global__ void __launch_bounds__(kCkThreads, 1)
       __nv_bfloat16* out =
           static_cast<__nv_bfloat16*>(p.out) + (L.tok0 * p.Hv + L.j) * kCkD + (col & ~1);
 #pragma unroll
-      for (int c0 = 0; c0 < kCkC; c0 += 16) {
+      for (int c0 = 0; c0 < kH; c0 += 16) {
         uint32_t cq[16], wq[16];
-        tc::tmem_ld16(tmG + lane_off + 64 + c0, cq);   // C^T, noisy queries
-        tc::tmem_ld16(tmW + lane_off + 128 + c0, wq);  // W^T, noisy queries
+        tc::tmem_ld16(tmG + lane_off + 64 + t0 + c0, cq);   // C^T, noisy queries
+        tc::tmem_ld16(tmW + lane_off + 128 + t0 + c0, wq);  // W^T, noisy queries
         tc::tmem_ld_wait();
 #pragma unroll
         for (int e2 = 0; e2 < 16; e2 += 2) {
           float o[2];
 #pragma unroll
           for (int f = 0; f < 2; ++f) {
-            const int l = c0 + e2 + f;
-            const int m0 = l & ~(B - 1);
+            const int u = c0 + e2 + f;  // local index
+            const int l = t0 + u;
+            const int m0u = u & ~(B - 1);
+            const int m0 = t0 + m0u;
             const float am = m0 > 0 ? sh.Gc[m0 - 1] : 1.f;
             const float ge = sh.Gn[m0 + B - 1];
             float acc = ge * (am * __uint_as_float(wq[e2 + f]) + __uint_as_float(cq[e2 + f]));
 #pragma unroll
-            for (int e = 0; e < B; ++e) acc = fmaf(AqT[(m0 + e) * kCkC + l], x[m0 + e], acc);
+            for (int e = 0; e < B; ++e) acc = fmaf(AqT[(m0 + e) * kCkC + l], xn[m0u + e], acc);
             o[f] = p.scale * acc;
           }
           const float recv = __shfl_xor_sync(0xffffffffu, odd ? o[0] : o[1], 1);
-          const int l = odd ? c0 + e2 + 1 : c0 + e2;
+          const int l = t0 + (odd ? c0 + e2 + 1 : c0 + e2);
           *reinterpret_cast<uint32_t*>(out + (size_t)l * p.Hv * kCkD) =
               odd ? ck_pack(recv, o[1]) : ck_pack(o[0], recv);
         }
       }
+    }
+    // the next chunk's values: both groups are past their reads of these
+    // (the clean ones before the second barrier, the noisy ones just now)
+    tc::fence_before_sync();
+    if (__syncthreads_or(bad)) break;
+    if (tid == kIssuer && it_next >= 0) {
+      tc::fence_async_smem();
+      issue_v(it_next);
+      v_out = true;
+      v_par = ph ^ 1u;
     }
     ph ^= 1u;
   }
