@@ -23,7 +23,11 @@
 //   MMA 1  W^T = S0^T [K; K~; Q~]^T      M=128 (c), N=192, K=128   (A: S0^T bf16, tensor memory)
 //          G   = [K; K~] [K; K~; Q~]^T   M=128 (rows), N=192, K=128: every dot product the
 //                                         chunk needs (K K^T, K K~^T, K Q~^T, K~ K~^T, K~ Q~^T)
-//   solve  (I + A) delta = X             fp32, per column, right-looking (warps 0-3)
+//   T      = (I + A)^{-1}                 fp32, 16 x 16 blocks: the diagonal ones by forward
+//                                         substitution, then T_ab = -T_aa sum_c A_ac T_cb by block
+//                                         columns, right-looking, within lanes (all warps)
+//   MMA d  delta^T = X^T T^T             M=128 (c), N=64, K=64     (X and T as bf16 high + low
+//                                         parts, three products: fp32-grade delta)
 //   MMA 2  C^T = delta^T P               M=128 (c), N=128, K=64    (A: delta^T bf16, tensor memory)
 //   noisy  S_(m)^T y = Gam_{mB-1} W^T + C^T, the B x B solves and the readouts (both groups)
 // bf16 operands and fp32 accumulation throughout (the state rounded to bf16
@@ -66,7 +70,10 @@ struct CkCfg {
   static constexpr int oAn = oAT + kT;   // A~[t][i] (noisy, zero outside the block)
   static constexpr int oAq = oAn + kT;   // Aqk^T[i][l] (noisy readout, zero outside the block)
   static constexpr int oP = oAq + kT;
-  static constexpr int kSmem = oP + kP;
+  static constexpr int oT = oP + kP;     // T[t][j] fp32, the lower blocks
+  static constexpr int kSmem = oT + kT;
+  // once the clean values are read, their buffer holds T as bf16 high and low
+  // parts (K-major SW128, rows of 64 elements, 8 KiB each): MMA d's operand
 };
 
 struct alignas(16) CkShared {
@@ -91,19 +98,149 @@ __device__ __forceinline__ uint32_t ck_pack(float a, float b) {
   return *reinterpret_cast<uint32_t*>(&h);
 }
 
-// 64 table values of one row, 16-byte stores
-__device__ __forceinline__ void ck_store_row(float* row, const float (&v)[kCkC]) {
-#pragma unroll
-  for (int q = 0; q < kCkC / 4; ++q)
-    reinterpret_cast<float4*>(row)[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+// Word offset of element (r, c) of a 64 x 64 fp32 table whose 16-byte units
+// are XOR-swizzled by the row (unit c / 4 of row r at unit (c / 4) ^ (r % 16)),
+// so that a warp writing one row per lane spreads over every bank.
+__device__ __forceinline__ int ck_sw(int r, int c) {
+  return r * kCkC + (((c >> 2) ^ (r & 15)) << 2) + (c & 3);
 }
 
-// this lane's 64 columns of tensor memory starting at `taddr`
-__device__ __forceinline__ void ck_ld64(uint32_t taddr, uint32_t (&r)[kCkC]) {
+// 32 table values of row r, columns c0 .. c0 + 31 (c0 a multiple of 4)
+__device__ __forceinline__ void ck_store32(float* tbl, int r, int c0, const float (&v)[32]) {
 #pragma unroll
-  for (int c0 = 0; c0 < kCkC; c0 += 16)
-    tc::tmem_ld16(taddr + c0, *reinterpret_cast<uint32_t(*)[16]>(&r[c0]));
+  for (int q = 0; q < 8; ++q)
+    *reinterpret_cast<float4*>(tbl + ck_sw(r, c0 + 4 * q)) =
+        make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+}
+
+// this lane's 32 columns of tensor memory starting at `taddr`
+__device__ __forceinline__ void ck_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+  tc::tmem_ld16(taddr, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
+  tc::tmem_ld16(taddr + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
   tc::tmem_ld_wait();
+}
+
+// x = hi + lo to about 2^-16 relative, each a bf16 pair (a low, b high)
+__device__ __forceinline__ void ck_split(float a, float b, uint32_t& hi, uint32_t& lo) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  const __nv_bfloat162 l =
+      __floats2bfloat162_rn(a - __low2float(h), b - __high2float(h));
+  hi = *reinterpret_cast<const uint32_t*>(&h);
+  lo = *reinterpret_cast<const uint32_t*>(&l);
+}
+
+// Column j of the diagonal block T_aa = (I + A_aa)^{-1}, forward substitution
+// (x_t -= A[t][i] x_i for t > i, the A^T rows as 16-byte loads),
+// stored whole (zeros above the diagonal) into the swizzled T table.
+__device__ __forceinline__ void ck_diag_inverse(const float* AT, float* Tf, int a, int j) {
+  float x[16];
+#pragma unroll
+  for (int t = 0; t < 16; ++t) x[t] = t == j ? 1.f : 0.f;
+#pragma unroll
+  for (int i = 0; i < 15; ++i) {
+    const float xi = x[i];
+#pragma unroll
+    for (int u = (i + 1) / 4; u < 4; ++u) {
+      const float4 q = *reinterpret_cast<const float4*>(AT + ck_sw(16 * a + i, 16 * a + 4 * u));
+      const float qv[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e)
+        if (4 * u + e > i) x[4 * u + e] = fmaf(-qv[e], xi, x[4 * u + e]);
+    }
+  }
+#pragma unroll
+  for (int t = 0; t < 16; ++t) Tf[ck_sw(16 * a + t, 16 * a + j)] = x[t];
+}
+
+// Block column BC of T below its diagonal block.  Column s of the block
+// column lives on R = NT / 16 adjacent lanes, lane g holding rows g, g + R, ..
+// of every block, so that all of its dependencies travel by shuffles (and the
+// R lanes' rows fall in distinct banks of the swizzled tables).
+// Right-looking (T_c,BC = -T_cc sum_{BC <= d < c} A_cd T_d,BC): once block d
+// of the column is known, acc_a += A_ad T_d,BC for every a > d, and the next
+// block is T_d+1,BC = -T_d+1,d+1 acc_d+1.  The accumulators are a shift
+// register (acc[k] for block row d + 1 + k) so that the loop over d stays a
+// loop.  Then the strips BC .. BC + nstrip - 1 (columns 16 BC ..) of T as bf16
+// high and low parts into Tb (K-major SW128 rows of 64 elements, zero above
+// the diagonal).
+template <int NT, int BC>
+__device__ __forceinline__ void ck_tcol(const float* AT, float* Tf, uint8_t* Tb, int nstrip, int q,
+                                        uint32_t bar_id) {
+  constexpr int R = NT / 16, RPT = 16 / R;
+  const int s = q / R, g = q % R, lane = q & 31;
+  const int src0 = lane & ~(R - 1);  // the first lane of this column
+  const int cs = 16 * BC + s;        // the column of T
+  float acc[3][RPT];                 // acc[k][e]: row 16 (d + 1 + k) + g + R e
+#pragma unroll
+  for (int k = 0; k < 3; ++k)
+#pragma unroll
+    for (int e = 0; e < RPT; ++e) acc[k][e] = 0.f;
+  float v[16];  // T_d,BC[i][s] of the block d just known
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = Tf[ck_sw(16 * BC + i, cs)];
+#pragma unroll 1
+  for (int d = BC; d < 3; ++d) {
+#pragma unroll
+    for (int k = 0; k < 3; ++k) {
+      const int a = d + 1 + k;
+      if (a < 4) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+#pragma unroll
+          for (int e = 0; e < RPT; ++e)  // A[16a + g + R e][16d + i]
+            acc[k][e] = fmaf(AT[ck_sw(16 * d + i, 16 * a + g + R * e)], v[i], acc[k][e]);
+        }
+      }
+    }
+    // block d + 1: T = -T_cc acc[0], acc[0] gathered from the column's lanes
+    const int c = d + 1;
+    float w[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) w[i] = __shfl_sync(0xffffffffu, acc[0][i / R], src0 + i % R);
+    float o[RPT];
+#pragma unroll
+    for (int e = 0; e < RPT; ++e) {
+      const int r = 16 * c + g + R * e;  // T_cc row
+      float x = 0.f;
+#pragma unroll
+      for (int i4 = 0; i4 < 4; ++i4) {
+        const float4 t4 = *reinterpret_cast<const float4*>(Tf + ck_sw(r, 16 * c + 4 * i4));
+        x = fmaf(t4.x, w[4 * i4], x);
+        x = fmaf(t4.y, w[4 * i4 + 1], x);
+        x = fmaf(t4.z, w[4 * i4 + 2], x);
+        x = fmaf(t4.w, w[4 * i4 + 3], x);
+      }
+      o[e] = -x;
+      Tf[ck_sw(r, cs)] = o[e];
+    }
+#pragma unroll
+    for (int e = 0; e < RPT; ++e) {
+      acc[0][e] = acc[1][e];
+      acc[1][e] = acc[2][e];
+      acc[2][e] = 0.f;
+    }
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __shfl_sync(0xffffffffu, o[i / R], src0 + i % R);
+  }
+  tc::named_bar_sync(bar_id, NT);  // the block column complete
+  // the strips: 64 rows x 2 units of 8 columns each; zero above the diagonal
+#pragma unroll 1
+  for (int k = q; k < 128 * nstrip; k += NT) {
+    const int u = 2 * BC + (k >> 6);  // 16-byte unit: columns 8u .. 8u + 7
+    const int t = k & 63;
+    const float4 f0 = *reinterpret_cast<const float4*>(Tf + ck_sw(t, 8 * u));
+    const float4 f1 = *reinterpret_cast<const float4*>(Tf + ck_sw(t, 8 * u + 4));
+    const float fv[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
+    uint32_t hi[4], lo[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e)
+      ck_split(8 * u + 2 * e <= t ? fv[2 * e] : 0.f, 8 * u + 2 * e + 1 <= t ? fv[2 * e + 1] : 0.f,
+               hi[e], lo[e]);
+    const int off = t * 128 + ((u ^ (t & 7)) << 4);
+    *reinterpret_cast<uint4*>(Tb + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+    *reinterpret_cast<uint4*>(Tb + 8192 + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+  }
+  tc::fence_async_smem();  // T is MMA d's operand
 }
 
 }  // namespace
@@ -124,6 +261,7 @@ __global__ void __launch_bounds__(kCkThreads, 1)
   float* An = reinterpret_cast<float*>(base + C::oAn);
   float* AqT = reinterpret_cast<float*>(base + C::oAq);
   uint8_t* Ps = base + C::oP;
+  float* Tf = reinterpret_cast<float*>(base + C::oT);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int col = tid & 127, grp = tid >> 7;  // value column (= lane of tensor memory), group
@@ -143,9 +281,10 @@ __global__ void __launch_bounds__(kCkThreads, 1)
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = sh.tmem_base;
-  const uint32_t tmS = tmem;        // S0^T bf16 (64 columns); then delta^T (32)
+  const uint32_t tmS = tmem;        // S0^T bf16 (64 columns); X^T high | low; delta^T (32)
   const uint32_t tmW = tmem + 64;   // W^T: [K | K~ | Q~] parts, 3 x 64 columns
   const uint32_t tmG = tmem + 256;  // G (rows on lanes), 192 columns; then C^T (128)
+  const uint32_t tmD = tmem + 448;  // delta^T fp32, 64 columns
   const uint32_t lane_off = (uint32_t)((warp & 3) * 32) << 16;
 
   struct Loc {
@@ -223,6 +362,7 @@ __global__ void __launch_bounds__(kCkThreads, 1)
   uint32_t ph = 0, ph_mma = 0;
   const uint32_t id192 = tc::idesc_bf16(128, 192, false, false);
   const uint32_t id128 = tc::idesc_bf16(128, 128, false, true);
+  const uint32_t id64 = tc::idesc_bf16(128, 64, false, false);
 
 #pragma unroll 1
   for (; it < total; it += (int)gridDim.x) {
@@ -306,61 +446,86 @@ __global__ void __launch_bounds__(kCkThreads, 1)
       }
     }
 
-    // ---- tables from G.  Lanes 0..63 hold the rows of K, 64..127 those of
-    // K~; every exponential is taken unconditionally and the masks applied as
-    // selects (a branch per element would serialise the chains).
+    // ---- tables from G, 32 columns at a time.  Lanes 0..63 hold the rows of
+    // K, 64..127 those of K~; every exponential is taken unconditionally and
+    // the masks applied as selects (a branch per element would serialise the
+    // chains).
     {
       const int row = col & 63;
       const bool krow = col < 64;
-      uint32_t gr[kCkC];
+      const int m0 = row & ~(B - 1);  // the block start of this row's token
       if (grp == 0) {
-        // warps 0-1: A^T row i of the clean system; warps 2-3: A~ row t
-        ck_ld64(tmG + lane_off + (krow ? 0 : 64), gr);
-        float v[kCkC];
         if (krow) {
+          // warps 0-1: A^T row i of the clean system
           const float gi = sh.gc2[row];
 #pragma unroll
-          for (int t = 0; t < kCkC; ++t) {
-            const float a = sh.bc[t] * tc::ex2(sh.gc2[t] - gi) * __uint_as_float(gr[t]);
-            v[t] = t > row ? a : 0.f;
+          for (int h = 0; h < 2; ++h) {
+            uint32_t gr[32];
+            float v[32];
+            ck_ld32(tmG + lane_off + 32 * h, gr);
+#pragma unroll
+            for (int k = 0; k < 32; ++k) {
+              const int t = 32 * h + k;
+              const float a = sh.bc[t] * tc::ex2(sh.gc2[t] - gi) * __uint_as_float(gr[k]);
+              v[k] = t > row ? a : 0.f;
+            }
+            ck_store32(AT, row, 32 * h, v);
           }
-          ck_store_row(AT + row * kCkC, v);
+          // this warp's A^T rows are A's columns 32 warp .. + 31: the diagonal
+          // blocks 2 warp and 2 warp + 1 of T, a column of one per lane
+          __syncwarp();
+          ck_diag_inverse(AT, Tf, 2 * warp + (lane >> 4), lane & 15);
         } else {
-          const int m0 = row & ~(B - 1);  // this token's block start
+          // warps 2-3: A~ row t
           const float bt = sh.bn[row], gt = sh.gn2[row];
 #pragma unroll
-          for (int i = 0; i < kCkC; ++i) {
-            const float a = bt * tc::ex2(gt - sh.gn2[i]) * __uint_as_float(gr[i]);
-            v[i] = (i >= m0 && i < row) ? a : 0.f;
+          for (int h = 0; h < 2; ++h) {
+            uint32_t gr[32];
+            float v[32];
+            ck_ld32(tmG + lane_off + 64 + 32 * h, gr);
+#pragma unroll
+            for (int k = 0; k < 32; ++k) {
+              const int i = 32 * h + k;
+              const float a = bt * tc::ex2(gt - sh.gn2[i]) * __uint_as_float(gr[k]);
+              v[k] = (i >= m0 && i < row) ? a : 0.f;
+            }
+            ck_store32(An, row, 32 * h, v);
           }
-          ck_store_row(An + row * kCkC, v);
         }
       } else {
         if (krow) {
           // warps 4-5: P row i, 128 columns (the noisy keys, then queries),
           // P[i][y] = [i < mB] exp(gamma_{mB-1} - gamma_i) (k_i . y)
+          // the factor depends on the row and the block only: one per block
           const float gi = sh.gc2[row];
 #pragma unroll 1
-          for (int half = 0; half < 2; ++half) {
-            ck_ld64(tmG + lane_off + 64 + half * 64, gr);
+          for (int h = 0; h < 4; ++h) {  // columns 32 h .. of the 128: tokens 32 (h % 2) ..
+            const int tq = 32 * (h & 1);
+            float fm[32 / B];
 #pragma unroll
-            for (int u = 0; u < 8; ++u) {  // 16-byte units of 8 columns
+            for (int m = 0; m < 32 / B; ++m) {
+              const int mb = tq + m * B;
+              const float a = tc::ex2(sh.gc2[mb > 0 ? mb - 1 : 0] - gi);
+              fm[m] = row < mb ? a : 0.f;
+            }
+            uint32_t gr[32];
+            ck_ld32(tmG + lane_off + 64 + 32 * h, gr);
+#pragma unroll
+            for (int u4 = 0; u4 < 4; ++u4) {  // 16-byte units of 8 columns
+              const int u = 4 * (h & 1) + u4;   // unit within the 64-column chunk
               uint32_t w[4];
 #pragma unroll
               for (int e = 0; e < 4; ++e) {
                 float pv[2];
 #pragma unroll
                 for (int f = 0; f < 2; ++f) {
-                  const int t = 8 * u + 2 * e + f;  // token of this column
-                  const int mb = t & ~(B - 1);      // its block start mB
-                  const float gm = mb > 0 ? sh.gc2[mb - 1] : 0.f;
-                  const float a = tc::ex2(gm - gi) * __uint_as_float(gr[t]);
-                  pv[f] = row < mb ? a : 0.f;
+                  const int k = 8 * u4 + 2 * e + f;  // column within the 32: token tq + k
+                  pv[f] = fm[k / B] * __uint_as_float(gr[k]);
                 }
                 w[e] = ck_pack(pv[0], pv[1]);
               }
-              // MN-major SW128: chunk `half`, row i, 16-byte unit u ^ (i % 8)
-              *reinterpret_cast<uint4*>(Ps + half * (kCkC * 128) + row * 128 +
+              // MN-major SW128: chunk h / 2, row i, 16-byte unit u ^ (i % 8)
+              *reinterpret_cast<uint4*>(Ps + (h >> 1) * (kCkC * 128) + row * 128 +
                                         ((u ^ (row & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
             }
           }
@@ -368,61 +533,92 @@ __global__ void __launch_bounds__(kCkThreads, 1)
         } else {
           // warps 6-7: Aqk^T row i (noisy key i): exp(gamma~_end - gamma~_i) (q~_l . k~_i)
           // for the queries l of its block
-          ck_ld64(tmG + lane_off + 128, gr);
-          const int m0 = row & ~(B - 1);
-          const float gi = sh.gn2[row], ge = sh.gn2[m0 + B - 1];
-          const float f = tc::ex2(ge - gi);
-          float v[kCkC];
+          const float f = tc::ex2(sh.gn2[m0 + B - 1] - sh.gn2[row]);
 #pragma unroll
-          for (int l = 0; l < kCkC; ++l) {
-            const float a = f * __uint_as_float(gr[l]);
-            v[l] = (l >= m0 && l < m0 + B) ? a : 0.f;
+          for (int h = 0; h < 2; ++h) {
+            uint32_t gr[32];
+            float v[32];
+            ck_ld32(tmG + lane_off + 128 + 32 * h, gr);
+#pragma unroll
+            for (int k = 0; k < 32; ++k) {
+              const int l = 32 * h + k;
+              v[k] = (l >= m0 && l < m0 + B) ? f * __uint_as_float(gr[k]) : 0.f;
+            }
+            ck_store32(AqT, row, 32 * h, v);
           }
-          ck_store_row(AqT + row * kCkC, v);
         }
       }
     }
-    // ---- group 0: X = diag(beta) (V - diag(Gam) K S0)
+    // ---- X = diag(beta) (V - diag(Gam) K S0), tokens 32 grp .. 32 grp + 31,
+    // into tensor memory as bf16 high and low parts over S0^T (which the first
+    // MMAs have read)
     bad |= !tc::mbar_wait(&sh.bar_v, ph, &sh.abort_flag);
     if (tid == kIssuer) v_out = false;
-    float x[kCkC];
-    if (grp == 0) {
-      uint32_t w[kCkC];
-      ck_ld64(tmW + lane_off, w);
+    {
+      const int t0 = 32 * grp;
+      uint32_t w0[16], w1[16], hi[16], lo[16];
+      tc::tmem_ld16(tmW + lane_off + t0, w0);
+      tc::tmem_ld16(tmW + lane_off + t0 + 16, w1);
+      tc::tmem_ld_wait();
       const uint8_t* vb = Vc + (col >> 6) * (kCkC * 128) + (col & 63) * 2;
 #pragma unroll
-      for (int t = 0; t < kCkC; ++t) {
-        const float vt = __uint_as_float(
-            (uint32_t)*reinterpret_cast<const unsigned short*>(vb + t * 128) << 16);
-        x[t] = sh.bc[t] * (vt - sh.Gc[t] * __uint_as_float(w[t]));
+      for (int e = 0; e < 16; ++e) {
+        float xv[2];
+#pragma unroll
+        for (int f = 0; f < 2; ++f) {
+          const int u = 2 * e + f, t = t0 + u;
+          const float vt = __uint_as_float(
+              (uint32_t)*reinterpret_cast<const unsigned short*>(vb + t * 128) << 16);
+          const float wt = __uint_as_float(u < 16 ? w0[u & 15] : w1[u & 15]);
+          xv[f] = sh.bc[t] * (vt - sh.Gc[t] * wt);
+        }
+        ck_split(xv[0], xv[1], hi[e], lo[e]);
       }
+      tc::tmem_st16(tmS + lane_off + 16 * grp, hi);
+      tc::tmem_st16(tmS + lane_off + 32 + 16 * grp, lo);
+      tc::tmem_st_wait();
     }
     tc::fence_before_sync();
-    if (__syncthreads_or(bad)) break;  // the tables published; G read
+    if (__syncthreads_or(bad)) break;  // tables, T's diagonal blocks, X^T; G and V read
 
-    if (grp == 0) {
-      // (I + A) delta = X, right-looking (A^T row t as 16-byte broadcast loads)
+    // ---- T = (I + A)^{-1} below its diagonal blocks: block column 0 on
+    // warps 0-3, 1 on warps 4-5, 2 (and the strip of 3) on warps 6-7
+    if (warp < 4)
+      ck_tcol<128, 0>(AT, Tf, Vc, 1, tid, 1);
+    else if (warp < 6)
+      ck_tcol<64, 1>(AT, Tf, Vc, 1, tid - 128, 2);
+    else
+      ck_tcol<64, 2>(AT, Tf, Vc, 2, tid - 192, 3);
+    if (__syncthreads_or(bad)) break;  // T as bf16 high / low parts
+    if (tid == kIssuer) {
+      const uint32_t tb = tc::smem_u32(Vc);
 #pragma unroll
-      for (int t = 0; t < kCkC; ++t) {
-        const float dt = x[t];
-        const float* ar = AT + t * kCkC;
-#pragma unroll
-        for (int u4 = (t + 1) / 4; u4 < kCkC / 4; ++u4) {
-          const float4 a = *reinterpret_cast<const float4*>(ar + 4 * u4);
-          if (4 * u4 + 0 > t) x[4 * u4 + 0] = fmaf(-a.x, dt, x[4 * u4 + 0]);
-          if (4 * u4 + 1 > t) x[4 * u4 + 1] = fmaf(-a.y, dt, x[4 * u4 + 1]);
-          if (4 * u4 + 2 > t) x[4 * u4 + 2] = fmaf(-a.z, dt, x[4 * u4 + 2]);
-          if (4 * u4 + 3 > t) x[4 * u4 + 3] = fmaf(-a.w, dt, x[4 * u4 + 3]);
-        }
+      for (int kk = 0; kk < kCkC / 16; ++kk) {
+        const uint64_t bh = tc::sdesc_sw128(tb + kk * 32, 16, 1024);
+        const uint64_t bl = tc::sdesc_sw128(tb + 8192 + kk * 32, 16, 1024);
+        tc::mma_bf16_ts(tmD, tmS + kk * 8, bh, id64, kk > 0);  // delta^T = X^T T^T
+        tc::mma_bf16_ts(tmD, tmS + kk * 8, bl, id64, 1);
+        tc::mma_bf16_ts(tmD, tmS + 32 + kk * 8, bh, id64, 1);
       }
-      // delta^T as bf16 pairs over S0^T, which the first MMAs have read
+      tc::mma_commit(&sh.bar_mma);
+      mma_out = true;
+    }
+    bad |= !tc::mbar_wait(&sh.bar_mma, ph_mma, &sh.abort_flag);
+    ph_mma ^= 1u;
+    tc::fence_after_sync();
+    if (tid == kIssuer) mma_out = false;
+    // delta^T as bf16 pairs over X^T's high part, tokens 32 grp .. 32 grp + 31
+    {
+      uint32_t d0[16], d1[16], w[16];
+      tc::tmem_ld16(tmD + lane_off + 32 * grp, d0);
+      tc::tmem_ld16(tmD + lane_off + 32 * grp + 16, d1);
+      tc::tmem_ld_wait();
 #pragma unroll
-      for (int c0 = 0; c0 < kCkC / 2; c0 += 16) {
-        uint32_t w[16];
-#pragma unroll
-        for (int e = 0; e < 16; ++e) w[e] = ck_pack(x[2 * (c0 + e)], x[2 * (c0 + e) + 1]);
-        tc::tmem_st16(tmS + lane_off + c0, w);
+      for (int e = 0; e < 8; ++e) {
+        w[e] = ck_pack(__uint_as_float(d0[2 * e]), __uint_as_float(d0[2 * e + 1]));
+        w[8 + e] = ck_pack(__uint_as_float(d1[2 * e]), __uint_as_float(d1[2 * e + 1]));
       }
+      tc::tmem_st16(tmS + lane_off + 16 * grp, w);
       tc::tmem_st_wait();
     }
     tc::fence_before_sync();
@@ -442,95 +638,92 @@ __global__ void __launch_bounds__(kCkThreads, 1)
     tc::fence_after_sync();
     if (tid == kIssuer) mma_out = false;
 
-    // ---- noisy blocks, tokens 32 grp .. 32 grp + 31 of the chunk (whole
-    // blocks: B divides 32):
+    // ---- noisy blocks, tokens 32 grp .. 32 grp + 31 of the chunk, 16 at a
+    // time (whole blocks: B divides 16):
     //   X~_t = beta~_t (v~_t - Gam~_t (Gam_{mB-1} W^T[k~_t] + C^T[k~_t])),
     //   the B x B solves, then
     //   o~_l = s (Gam~_end (Gam_{mB-1} W^T[q~_l] + C^T[q~_l]) + Aqk delta~)
     {
-      constexpr int kH = kCkC / 2;
-      const int t0 = grp * kH;
-      float xn[kH];
-      {
-        uint32_t wk[16], ck[16];
-        const uint8_t* vb = Vn + (col >> 6) * (kCkC * 128) + (col & 63) * 2;
-#pragma unroll
-        for (int c0 = 0; c0 < kH; c0 += 16) {
-          tc::tmem_ld16(tmW + lane_off + 64 + t0 + c0, wk);  // W^T, noisy keys
-          tc::tmem_ld16(tmG + lane_off + t0 + c0, ck);       // C^T, noisy keys
-          tc::tmem_ld_wait();
-#pragma unroll
-          for (int e = 0; e < 16; ++e) {
-            const int t = t0 + c0 + e;
-            const int mb = t & ~(B - 1);
-            const float am = mb > 0 ? sh.Gc[mb - 1] : 1.f;  // Gam_{mB-1}
-            const float vt = __uint_as_float(
-                (uint32_t)*reinterpret_cast<const unsigned short*>(vb + t * 128) << 16);
-            xn[c0 + e] = sh.bn[t] * (vt - sh.Gn[t] * (am * __uint_as_float(wk[e]) +
-                                                       __uint_as_float(ck[e])));
-          }
-        }
-      }
-      // (I + A~) delta~ = X~ per block, forward substitution
-#pragma unroll
-      for (int u = 0; u < kH; ++u) {
-        const int m0u = u & ~(B - 1);     // block start, local index (compile-time)
-        const float* ar = An + (t0 + u) * kCkC + t0 + m0u;
-        float acc = xn[u];
-        if constexpr (B >= 4) {  // (t0 + m0u) is then a multiple of 4: 16-byte loads
-#pragma unroll
-          for (int i4 = 0; i4 < B / 4; ++i4) {
-            const float4 a = reinterpret_cast<const float4*>(ar)[i4];
-            const float av[4] = {a.x, a.y, a.z, a.w};
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const int i = m0u + 4 * i4 + e;
-              if (i < u) acc = fmaf(-av[e], xn[i], acc);
-            }
-          }
-        } else {
-#pragma unroll
-          for (int e = 0; e < B; ++e)
-            if (m0u + e < u) acc = fmaf(-ar[e], xn[m0u + e], acc);
-        }
-        xn[u] = acc;
-      }
-      // readout; adjacent lanes swap one value so that each stores a bf16
-      // pair of two columns
+      const uint8_t* vb = Vn + (col >> 6) * (kCkC * 128) + (col & 63) * 2;
       const bool odd = lane & 1;
       __nv_bfloat16* out =
           static_cast<__nv_bfloat16*>(p.out) + (L.tok0 * p.Hv + L.j) * kCkD + (col & ~1);
+#pragma unroll 1
+      for (int g16 = 0; g16 < 2; ++g16) {
+        const int t0 = 32 * grp + 16 * g16;  // the first token of these 16
+        float xn[16];
+        {
+          uint32_t wk[16], ck[16];
+          tc::tmem_ld16(tmW + lane_off + 64 + t0, wk);  // W^T, noisy keys
+          tc::tmem_ld16(tmG + lane_off + t0, ck);       // C^T, noisy keys
+          tc::tmem_ld_wait();
 #pragma unroll
-      for (int c0 = 0; c0 < kH; c0 += 16) {
+          for (int e = 0; e < 16; ++e) {
+            const int t = t0 + e;
+            const int mb = t0 + (e & ~(B - 1));
+            const float am = mb > 0 ? sh.Gc[mb - 1] : 1.f;  // Gam_{mB-1}
+            const float vt = __uint_as_float(
+                (uint32_t)*reinterpret_cast<const unsigned short*>(vb + t * 128) << 16);
+            xn[e] = sh.bn[t] * (vt - sh.Gn[t] * (am * __uint_as_float(wk[e]) +
+                                                  __uint_as_float(ck[e])));
+          }
+        }
+        // (I + A~) delta~ = X~ per block, forward substitution
+#pragma unroll
+        for (int u = 0; u < 16; ++u) {
+          const int m0u = u & ~(B - 1);  // block start within the 16 (compile-time)
+          float acc = xn[u];
+          if constexpr (B >= 4) {  // (t0 + m0u) is then a multiple of 4: 16-byte loads
+#pragma unroll
+            for (int i4 = 0; 4 * i4 < u - m0u; ++i4) {  // the units holding columns < u
+              const float4 a =
+                  *reinterpret_cast<const float4*>(An + ck_sw(t0 + u, t0 + m0u + 4 * i4));
+              const float av[4] = {a.x, a.y, a.z, a.w};
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const int i = m0u + 4 * i4 + e;
+                if (i < u) acc = fmaf(-av[e], xn[i], acc);
+              }
+            }
+          } else {
+#pragma unroll
+            for (int e = 0; e < B; ++e)
+              if (m0u + e < u) acc = fmaf(-An[ck_sw(t0 + u, t0 + m0u + e)], xn[m0u + e], acc);
+          }
+          xn[u] = acc;
+        }
+        // readout; adjacent lanes swap one value so that each stores a bf16
+        // pair of two columns
         uint32_t cq[16], wq[16];
-        tc::tmem_ld16(tmG + lane_off + 64 + t0 + c0, cq);   // C^T, noisy queries
-        tc::tmem_ld16(tmW + lane_off + 128 + t0 + c0, wq);  // W^T, noisy queries
+        tc::tmem_ld16(tmG + lane_off + 64 + t0, cq);   // C^T, noisy queries
+        tc::tmem_ld16(tmW + lane_off + 128 + t0, wq);  // W^T, noisy queries
         tc::tmem_ld_wait();
 #pragma unroll
         for (int e2 = 0; e2 < 16; e2 += 2) {
           float o[2];
 #pragma unroll
           for (int f = 0; f < 2; ++f) {
-            const int u = c0 + e2 + f;  // local index
+            const int u = e2 + f;
             const int l = t0 + u;
             const int m0u = u & ~(B - 1);
             const int m0 = t0 + m0u;
             const float am = m0 > 0 ? sh.Gc[m0 - 1] : 1.f;
             const float ge = sh.Gn[m0 + B - 1];
-            float acc = ge * (am * __uint_as_float(wq[e2 + f]) + __uint_as_float(cq[e2 + f]));
+            float acc = ge * (am * __uint_as_float(wq[u]) + __uint_as_float(cq[u]));
 #pragma unroll
-            for (int e = 0; e < B; ++e) acc = fmaf(AqT[(m0 + e) * kCkC + l], xn[m0u + e], acc);
+            for (int e = 0; e < B; ++e) acc = fmaf(AqT[ck_sw(m0 + e, l)], xn[m0u + e], acc);
             o[f] = p.scale * acc;
           }
           const float recv = __shfl_xor_sync(0xffffffffu, odd ? o[0] : o[1], 1);
-          const int l = t0 + (odd ? c0 + e2 + 1 : c0 + e2);
+          const int l = t0 + (odd ? e2 + 1 : e2);
           *reinterpret_cast<uint32_t*>(out + (size_t)l * p.Hv * kCkD) =
               odd ? ck_pack(recv, o[1]) : ck_pack(o[0], recv);
         }
       }
     }
     // the next chunk's values: both groups are past their reads of these
-    // (the clean ones before the second barrier, the noisy ones just now)
+    // (the clean ones before the second barrier, the T parts over them by
+    // MMA d, the noisy ones just now)
     tc::fence_before_sync();
     if (__syncthreads_or(bad)) break;
     if (tid == kIssuer && it_next >= 0) {
