@@ -105,6 +105,13 @@ __device__ __forceinline__ int ck_sw(int r, int c) {
   return r * kCkC + (((c >> 2) ^ (r & 15)) << 2) + (c & 3);
 }
 
+// The same for the T table, swizzled by r / 2 (unit c / 4 at (c / 4) ^ (r / 2 % 8)):
+// the row groups 2 g .. and 4 g .. that the lanes of a column hold fall in
+// distinct banks, and a warp reading one row per lane still spreads over all.
+__device__ __forceinline__ int ck_swt(int r, int c) {
+  return r * kCkC + (((c >> 2) ^ ((r >> 1) & 7)) << 2) + (c & 3);
+}
+
 // 32 table values of row r, columns c0 .. c0 + 31 (c0 a multiple of 4)
 __device__ __forceinline__ void ck_store32(float* tbl, int r, int c0, const float (&v)[32]) {
 #pragma unroll
@@ -149,13 +156,13 @@ __device__ __forceinline__ void ck_diag_inverse(const float* AT, float* Tf, int 
     }
   }
 #pragma unroll
-  for (int t = 0; t < 16; ++t) Tf[ck_sw(16 * a + t, 16 * a + j)] = x[t];
+  for (int t = 0; t < 16; ++t) Tf[ck_swt(16 * a + t, 16 * a + j)] = x[t];
 }
 
 // Block column BC of T below its diagonal block.  Column s of the block
-// column lives on R = NT / 16 adjacent lanes, lane g holding rows g, g + R, ..
-// of every block, so that all of its dependencies travel by shuffles (and the
-// R lanes' rows fall in distinct banks of the swizzled tables).
+// column lives on R = NT / 16 adjacent lanes, lane g holding rows g RPT ..
+// g RPT + RPT - 1 of every block (RPT = 16 / R), so that all of its
+// dependencies travel by shuffles.
 // Right-looking (T_c,BC = -T_cc sum_{BC <= d < c} A_cd T_d,BC): once block d
 // of the column is known, acc_a += A_ad T_d,BC for every a > d, and the next
 // block is T_d+1,BC = -T_d+1,d+1 acc_d+1.  The accumulators are a shift
@@ -170,14 +177,14 @@ __device__ __forceinline__ void ck_tcol(const float* AT, float* Tf, uint8_t* Tb,
   const int s = q / R, g = q % R, lane = q & 31;
   const int src0 = lane & ~(R - 1);  // the first lane of this column
   const int cs = 16 * BC + s;        // the column of T
-  float acc[3][RPT];                 // acc[k][e]: row 16 (d + 1 + k) + g + R e
+  float acc[3][RPT];                 // acc[k][e]: row 16 (d + 1 + k) + g RPT + e
 #pragma unroll
   for (int k = 0; k < 3; ++k)
 #pragma unroll
     for (int e = 0; e < RPT; ++e) acc[k][e] = 0.f;
   float v[16];  // T_d,BC[i][s] of the block d just known
 #pragma unroll
-  for (int i = 0; i < 16; ++i) v[i] = Tf[ck_sw(16 * BC + i, cs)];
+  for (int i = 0; i < 16; ++i) v[i] = Tf[ck_swt(16 * BC + i, cs)];
 #pragma unroll 1
   for (int d = BC; d < 3; ++d) {
 #pragma unroll
@@ -186,9 +193,17 @@ __device__ __forceinline__ void ck_tcol(const float* AT, float* Tf, uint8_t* Tb,
       if (a < 4) {
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
+          float av[RPT];
+          const float* ap = AT + ck_sw(16 * d + i, 16 * a + g * RPT);  // A[16a + g RPT ..][16d + i]
+          if constexpr (RPT == 4) {
+            const float4 v4 = *reinterpret_cast<const float4*>(ap);
+            av[0] = v4.x; av[1] = v4.y; av[2] = v4.z; av[3] = v4.w;
+          } else {
+            const float2 v2 = *reinterpret_cast<const float2*>(ap);
+            av[0] = v2.x; av[1] = v2.y;
+          }
 #pragma unroll
-          for (int e = 0; e < RPT; ++e)  // A[16a + g + R e][16d + i]
-            acc[k][e] = fmaf(AT[ck_sw(16 * d + i, 16 * a + g + R * e)], v[i], acc[k][e]);
+          for (int e = 0; e < RPT; ++e) acc[k][e] = fmaf(av[e], v[i], acc[k][e]);
         }
       }
     }
@@ -196,22 +211,22 @@ __device__ __forceinline__ void ck_tcol(const float* AT, float* Tf, uint8_t* Tb,
     const int c = d + 1;
     float w[16];
 #pragma unroll
-    for (int i = 0; i < 16; ++i) w[i] = __shfl_sync(0xffffffffu, acc[0][i / R], src0 + i % R);
+    for (int i = 0; i < 16; ++i) w[i] = __shfl_sync(0xffffffffu, acc[0][i % RPT], src0 + i / RPT);
     float o[RPT];
 #pragma unroll
     for (int e = 0; e < RPT; ++e) {
-      const int r = 16 * c + g + R * e;  // T_cc row
+      const int r = 16 * c + g * RPT + e;  // T_cc row
       float x = 0.f;
 #pragma unroll
       for (int i4 = 0; i4 < 4; ++i4) {
-        const float4 t4 = *reinterpret_cast<const float4*>(Tf + ck_sw(r, 16 * c + 4 * i4));
+        const float4 t4 = *reinterpret_cast<const float4*>(Tf + ck_swt(r, 16 * c + 4 * i4));
         x = fmaf(t4.x, w[4 * i4], x);
         x = fmaf(t4.y, w[4 * i4 + 1], x);
         x = fmaf(t4.z, w[4 * i4 + 2], x);
         x = fmaf(t4.w, w[4 * i4 + 3], x);
       }
       o[e] = -x;
-      Tf[ck_sw(r, cs)] = o[e];
+      Tf[ck_swt(r, cs)] = o[e];
     }
 #pragma unroll
     for (int e = 0; e < RPT; ++e) {
@@ -220,7 +235,7 @@ __device__ __forceinline__ void ck_tcol(const float* AT, float* Tf, uint8_t* Tb,
       acc[2][e] = 0.f;
     }
 #pragma unroll
-    for (int i = 0; i < 16; ++i) v[i] = __shfl_sync(0xffffffffu, o[i / R], src0 + i % R);
+    for (int i = 0; i < 16; ++i) v[i] = __shfl_sync(0xffffffffu, o[i % RPT], src0 + i / RPT);
   }
   tc::named_bar_sync(bar_id, NT);  // the block column complete
   // the strips: 64 rows x 2 units of 8 columns each; zero above the diagonal
@@ -228,8 +243,8 @@ __device__ __forceinline__ void ck_tcol(const float* AT, float* Tf, uint8_t* Tb,
   for (int k = q; k < 128 * nstrip; k += NT) {
     const int u = 2 * BC + (k >> 6);  // 16-byte unit: columns 8u .. 8u + 7
     const int t = k & 63;
-    const float4 f0 = *reinterpret_cast<const float4*>(Tf + ck_sw(t, 8 * u));
-    const float4 f1 = *reinterpret_cast<const float4*>(Tf + ck_sw(t, 8 * u + 4));
+    const float4 f0 = *reinterpret_cast<const float4*>(Tf + ck_swt(t, 8 * u));
+    const float4 f1 = *reinterpret_cast<const float4*>(Tf + ck_swt(t, 8 * u + 4));
     const float fv[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
     uint32_t hi[4], lo[4];
 #pragma unroll
