@@ -486,10 +486,7 @@ __global__ void __launch_bounds__(kCkThreads, 1)
             }
             ck_store32(AT, row, 32 * h, v);
           }
-          // this warp's A^T rows are A's columns 32 warp .. + 31: the diagonal
-          // blocks 2 warp and 2 warp + 1 of T, a column of one per lane
-          __syncwarp();
-          ck_diag_inverse(AT, Tf, 2 * warp + (lane >> 4), lane & 15);
+          tc::named_bar_arrive(4, 128);  // A^T to warps 4-5
         } else {
           // warps 2-3: A~ row t
           const float bt = sh.bn[row], gt = sh.gn2[row];
@@ -545,6 +542,10 @@ __global__ void __launch_bounds__(kCkThreads, 1)
             }
           }
           tc::fence_async_smem();  // P is the second MMA's operand
+          // the diagonal blocks of T once warps 0-1 have written A^T: blocks
+          // 2 (warp - 4) and 2 (warp - 4) + 1, a column of one per lane
+          tc::named_bar_sync(4, 128);
+          ck_diag_inverse(AT, Tf, 2 * (warp - 4) + (lane >> 4), lane & 15);
         } else {
           // warps 6-7: Aqk^T row i (noisy key i): exp(gamma~_end - gamma~_i) (q~_l . k~_i)
           // for the queries l of its block
@@ -707,32 +708,65 @@ __global__ void __launch_bounds__(kCkThreads, 1)
           }
           xn[u] = acc;
         }
-        // readout; adjacent lanes swap one value so that each stores a bf16
-        // pair of two columns
+        // readout, block by block (the block's queries from one AqT row
+        // segment per key); adjacent lanes swap one value so that each stores
+        // a bf16 pair of two columns
         uint32_t cq[16], wq[16];
         tc::tmem_ld16(tmG + lane_off + 64 + t0, cq);   // C^T, noisy queries
         tc::tmem_ld16(tmW + lane_off + 128 + t0, wq);  // W^T, noisy queries
         tc::tmem_ld_wait();
+        // the stores of one pair of queries (u, u + 1)
+        auto store_pair = [&](int u, float o0, float o1) {
+          o0 *= p.scale;
+          o1 *= p.scale;
+          const float recv = __shfl_xor_sync(0xffffffffu, odd ? o0 : o1, 1);
+          const int l = t0 + (odd ? u + 1 : u);
+          *reinterpret_cast<uint32_t*>(out + (size_t)l * p.Hv * kCkD) =
+              odd ? ck_pack(recv, o1) : ck_pack(o0, recv);
+        };
+        if constexpr (B == 1) {
 #pragma unroll
-        for (int e2 = 0; e2 < 16; e2 += 2) {
-          float o[2];
+          for (int u = 0; u < 16; u += 2) {
+            float o[2];
 #pragma unroll
-          for (int f = 0; f < 2; ++f) {
-            const int u = e2 + f;
-            const int l = t0 + u;
-            const int m0u = u & ~(B - 1);
-            const int m0 = t0 + m0u;
+            for (int f = 0; f < 2; ++f) {
+              const int l = t0 + u + f;
+              const float am = l > 0 ? sh.Gc[l - 1] : 1.f;
+              o[f] = sh.Gn[l] * (am * __uint_as_float(wq[u + f]) + __uint_as_float(cq[u + f])) +
+                     AqT[ck_sw(l, l)] * xn[u + f];
+            }
+            store_pair(u, o[0], o[1]);
+          }
+        } else {
+#pragma unroll
+          for (int mb = 0; mb < 16; mb += B) {
+            const int m0 = t0 + mb;  // the block's first token
             const float am = m0 > 0 ? sh.Gc[m0 - 1] : 1.f;
             const float ge = sh.Gn[m0 + B - 1];
-            float acc = ge * (am * __uint_as_float(wq[u]) + __uint_as_float(cq[u]));
+            float o[B];
 #pragma unroll
-            for (int e = 0; e < B; ++e) acc = fmaf(AqT[ck_sw(m0 + e, l)], xn[m0u + e], acc);
-            o[f] = p.scale * acc;
+            for (int l = 0; l < B; ++l)
+              o[l] = ge * (am * __uint_as_float(wq[mb + l]) + __uint_as_float(cq[mb + l]));
+#pragma unroll
+            for (int e = 0; e < B; ++e) {  // key m0 + e: AqT[m0 + e][m0 .. m0 + B - 1]
+              float aq[B];
+              if constexpr (B >= 4) {
+#pragma unroll
+                for (int i4 = 0; i4 < B / 4; ++i4) {
+                  const float4 a =
+                      *reinterpret_cast<const float4*>(AqT + ck_sw(m0 + e, m0 + 4 * i4));
+                  aq[4 * i4] = a.x; aq[4 * i4 + 1] = a.y; aq[4 * i4 + 2] = a.z; aq[4 * i4 + 3] = a.w;
+                }
+              } else {
+                const float2 a = *reinterpret_cast<const float2*>(AqT + ck_sw(m0 + e, m0));
+                aq[0] = a.x; aq[1] = a.y;
+              }
+#pragma unroll
+              for (int l = 0; l < B; ++l) o[l] = fmaf(aq[l], xn[mb + e], o[l]);
+            }
+#pragma unroll
+            for (int l = 0; l < B; l += 2) store_pair(mb + l, o[l], o[l + 1]);
           }
-          const float recv = __shfl_xor_sync(0xffffffffu, odd ? o[0] : o[1], 1);
-          const int l = t0 + (odd ? e2 + 1 : e2);
-          *reinterpret_cast<uint32_t*>(out + (size_t)l * p.Hv * kCkD) =
-              odd ? ck_pack(recv, o[1]) : ck_pack(o[0], recv);
         }
       }
     }
