@@ -23,6 +23,9 @@ CASES = {
                          prefix_hi=128, seed=74),
     "w4_fp32_small": W["tiny_fp32"].replace(num_requests=3, block_len=9, conv_width=4, seed=75),
     "w4_small_model": W["small_model_batch256"].replace(num_requests=5, conv_width=4, seed=76),
+    # 120 channels: rows that do not tile by 512 bytes (one copy per row)
+    "w4_c120": SC.replace(num_requests=3, block_len=11, num_qk_heads=1, num_v_heads=1,
+                          head_dim_k=40, head_dim_v=40, prefix_lo=64, prefix_hi=128, seed=77),
 }
 
 
