@@ -123,8 +123,6 @@ struct TwoStreamParams {
 };
 int two_stream_chunk_len();
 cudaError_t launch_two_stream_fwd(const TwoStreamParams& p, bool bf16, cudaStream_t stream);
-bool two_stream_tc_supported(int B, int dk, int dv);
-cudaError_t launch_two_stream_tc(const TwoStreamParams& p, cudaStream_t stream);
 bool two_stream_chunk_supported(int B, int dk, int dv);
 cudaError_t launch_two_stream_chunk(const TwoStreamParams& p, cudaStream_t stream);
 cudaError_t launch_gdr_denoise_tc(const GdrParams& p, cudaStream_t stream);

@@ -2,7 +2,7 @@
 // (appendix "Two-stream recurrence and block-level chain rule",
 // Eq. noisy-block-fwd; the Route II fused forward), CUDA-core form in exact
 // fp32.  It serves fp32 activations; bf16 activations (d_k = d_v = 128) take
-// the tensor-core kernel in two_stream_tc.cu.
+// the chunkwise tensor-core kernel in two_stream_chunk.cu.
 //
 // One CTA per (sequence, value head, chunk of 64 tokens).  The clean state
 // S_[c] at the chunk start (from the clean chunkwise pass) is loaded into
@@ -347,7 +347,7 @@ int two_stream_chunk_len() { return kTsChunk; }
 
 cudaError_t launch_two_stream_fwd(const TwoStreamParams& p, bool bf16, cudaStream_t stream) {
   if (p.N == 0) return cudaSuccess;
-  // bf16 activations take the tensor-core kernel (two_stream_tc.cu)
+  // bf16 activations take the chunkwise tensor-core kernel (two_stream_chunk.cu)
   if (bf16 && two_stream_chunk_supported(p.B, p.dk, p.dv)) return launch_two_stream_chunk(p, stream);
   return bf16 ? launch_ts_d<__nv_bfloat16>(p, stream) : launch_ts_d<float>(p, stream);
 }
