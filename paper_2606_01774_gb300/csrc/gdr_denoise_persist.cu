@@ -15,9 +15,11 @@
 //
 //   MMA 1  G   = [K;Q] K^T        M=128 ([K;Q] rows on lanes kG0..), N=Bp, K=128
 //          W^T = S0^T [K;Q]^T     M=128 (c), N=2BM, K=128   (A: S0^T, bf16, tensor memory)
-//   solve  (I + A) delta = X      fp32, per column, right-looking
-//   MMA 2  O2^T = delta^T M2^T    M=128 (c), N=Bp, K=Bp     (A: delta^T, bf16, tensor memory)
 //          M2[l][i] = exp(gamma_{B-1} - gamma_i) (q_l . k_i)
+//   N      = M2 T, T = (I + A)^{-1}   fp32: T's 16 x 16 diagonal blocks by forward
+//          substitution, then (B > 16) N1 = M2_1 T11, N0 = (M2_0 - N1 A10) T00
+//   MMA 2  O2^T = X^T N^T         M=128 (c), N=Bp, K=Bp     (X and N as bf16 high + low
+//          parts, three products: O2 = delta^T M2^T with delta = T X, never formed)
 //   out[l][c] = s (Gam_{B-1} W^T[c][BM + l] + O2^T[c][l])
 //
 // Bp = B rounded up to 16; the K, Q and V tiles hold BM = 16 or 32 rows (rows
@@ -33,7 +35,8 @@
 // products, solve and readout; the next keys and queries follow this item's
 // first MMA, the next values its second CTA barrier, the next gates and slot
 // one item ahead into registers.  Three CTA barriers per item (S0^T written,
-// A^T and M2 written, delta^T written); every other wait is a thread's own.  A bad slot is flagged in the device status word and
+// A^T, M2, T's diagonal blocks and X^T written, N written); every other wait
+// is a thread's own.  A bad slot is flagged in the device status word and
 // the item skipped (its output untouched).  Every wait is bounded: on a
 // timeout the CTA sets FLARE_DEV_WAIT_TIMEOUT, waits (bounded) for its copies
 // and MMAs in flight, frees its tensor memory and exits.
@@ -63,8 +66,9 @@ struct DpCfg {
   static constexpr int kATb0 = (kAT + 1023) / 1024 * 1024;
   static constexpr int kATb = kV + kATb0 >= kG0 * 128 ? kATb0 : kG0 * 128 - kV;
   static constexpr int kKQ = 2 * 2 * BM * 128;  // 2 chunks of [K;Q]: 2BM rows x 128 B (SW128)
-  static constexpr int kM2 = BM * 128;          // M2 [l][i], K-major, SW128
-  static constexpr int kSmem = kS0 + kV + kATb + kKQ + kM2;
+  static constexpr int kNb = 2 * BM * 128;      // N [l][j] bf16 high, then low: K-major, SW128
+  static constexpr int kMf = BM * kATs * 4;     // an fp32 table: M2 [l][i], T [i][j]
+  static constexpr int kSmem = kS0 + kV + kATb + kKQ + kNb + 2 * kMf;
 };
 
 struct alignas(16) DpShared {
@@ -105,17 +109,36 @@ __device__ __forceinline__ uint32_t dp_pack(float a, float b) {
   return *reinterpret_cast<uint32_t*>(&h);
 }
 
-// 16 bf16 values (columns c0..c0+15) into row `row` of a K-major SW128 tile.
-__device__ __forceinline__ void dp_store16_sw128(uint8_t* tile, int row, int c0,
-                                                 const float (&v)[16]) {
-  uint8_t* p = tile + row * 128;
+// x = hi + lo to about 2^-16 relative, each a bf16 pair (a low, b high)
+__device__ __forceinline__ void dp_split(float a, float b, uint32_t& hi, uint32_t& lo) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  const __nv_bfloat162 l = __floats2bfloat162_rn(a - __low2float(h), b - __high2float(h));
+  hi = *reinterpret_cast<const uint32_t*>(&h);
+  lo = *reinterpret_cast<const uint32_t*>(&l);
+}
+
+// Column j of the diagonal block T_aa = (I + A_aa)^{-1} (16 x 16): forward
+// substitution, x_t -= A[t][i] x_i for t > i with row i of A^T (A's column i)
+// as 16-byte loads; stored whole (zeros above the diagonal) into T[t][j].
+template <int kATs>
+__device__ __forceinline__ void dp_diag_inverse(const float* AT, float* Tf, int a, int j) {
+  float x[16];
 #pragma unroll
-  for (int h = 0; h < 2; ++h) {
-    const int g = (c0 >> 3) + h;
-    *reinterpret_cast<uint4*>(p + ((g ^ (row & 7)) << 4)) =
-        make_uint4(dp_pack(v[8 * h], v[8 * h + 1]), dp_pack(v[8 * h + 2], v[8 * h + 3]),
-                   dp_pack(v[8 * h + 4], v[8 * h + 5]), dp_pack(v[8 * h + 6], v[8 * h + 7]));
+  for (int t = 0; t < 16; ++t) x[t] = t == j ? 1.f : 0.f;
+#pragma unroll
+  for (int i = 0; i < 15; ++i) {
+    const float xi = x[i];
+#pragma unroll
+    for (int u = (i + 1) / 4; u < 4; ++u) {
+      const float4 q = *reinterpret_cast<const float4*>(AT + (16 * a + i) * kATs + 16 * a + 4 * u);
+      const float qv[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e)
+        if (4 * u + e > i) x[4 * u + e] = fmaf(-qv[e], xi, x[4 * u + e]);
+    }
   }
+#pragma unroll
+  for (int t = 0; t < 16; ++t) Tf[(16 * a + t) * kATs + 16 * a + j] = x[t];
 }
 
 }  // namespace
@@ -136,7 +159,9 @@ __global__ void __launch_bounds__(kDpThreads, 2)
   uint8_t* Vs = base + C::kS0;
   float* AT = reinterpret_cast<float*>(Vs + C::kV);
   uint8_t* KQs = Vs + C::kV + C::kATb;
-  uint8_t* M2s = KQs + C::kKQ;
+  uint8_t* Nbs = KQs + C::kKQ;
+  float* M2f = reinterpret_cast<float*>(Nbs + C::kNb);
+  float* Tf = M2f + BM * kATs;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int total = p.R * p.Hv;
@@ -161,7 +186,7 @@ __global__ void __launch_bounds__(kDpThreads, 2)
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = sh.tmem_base;
-  const uint32_t tmS = tmem;                // S0^T bf16 (64 columns); then delta^T
+  const uint32_t tmS = tmem;                // S0^T bf16 (64 columns); then X^T high | low
   const uint32_t tmW = tmem + 64;           // W^T: [K part | Q part], 2BM columns
   const uint32_t tmG = tmem + 64 + 2 * BM;  // G (rows on lanes kG0..); then O2^T
   const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
@@ -349,18 +374,21 @@ __global__ void __launch_bounds__(kDpThreads, 2)
           er[4 * i4] = q.x, er[4 * i4 + 1] = q.y, er[4 * i4 + 2] = q.z, er[4 * i4 + 3] = q.w;
         }
 #pragma unroll
-        for (int c0 = 0; c0 < BM; c0 += 16) {
-          float v[16];
+        for (int i4 = 0; i4 < BM / 4; ++i4) {
+          float v[4];
 #pragma unroll
-          for (int e = 0; e < 16; ++e) {
-            const int i = c0 + e;
+          for (int e = 0; e < 4; ++e) {
+            const int i = 4 * i4 + e;
             const float m = er[i] * __uint_as_float(gr[i]);
             v[e] = (i < B && l < B) ? m : 0.f;
           }
-          dp_store16_sw128(M2s, l, c0, v);
+          *reinterpret_cast<float4*>(M2f + l * kATs + 4 * i4) = make_float4(v[0], v[1], v[2], v[3]);
         }
-        tc::fence_async_smem();  // M2 is the second MMA's operand
       }
+      // T's diagonal blocks from this warp's A^T rows (A's columns), a column
+      // of one block per lane
+      __syncwarp();
+      if (row >= 0 && row < BM) dp_diag_inverse<kATs>(AT, Tf, row >> 4, row & 15);
     }
     bad |= !tc::mbar_wait(&sh.bar_mma, ph_mma, &sh.abort_flag);
     ph_mma ^= 1u;
@@ -394,11 +422,31 @@ __global__ void __launch_bounds__(kDpThreads, 2)
         }
       }
     }
+    // X^T into tensor memory as bf16 high and low parts, over S0^T (read by
+    // the first MMAs): high parts in columns 0 .. BM/2 - 1, low parts after
+    {
+      uint32_t hi[BM / 2], lo[BM / 2];
+#pragma unroll
+      for (int e = 0; e < BM / 2; ++e) dp_split(x[2 * e], x[2 * e + 1], hi[e], lo[e]);
+      if constexpr (BM == 32) {
+        tc::tmem_st16(tmS + lane_off, hi);
+        tc::tmem_st16(tmS + lane_off + 16, lo);
+      } else {
+        uint32_t w[16];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          w[e] = hi[e];
+          w[8 + e] = lo[e];
+        }
+        tc::tmem_st16(tmS + lane_off, w);
+      }
+      tc::tmem_st_wait();
+    }
     // the readout's scale, read here: the gates' buffer is rewritten for the
     // next item once every thread is past the barrier before the second MMA
     const float sG = p.scale * sh.Gam[B - 1];
     tc::fence_before_sync();
-    if (__syncthreads_or(bad)) break;  // A^T and M2 published; the values, W^T's key part and G read
+    if (__syncthreads_or(bad)) break;  // A^T, M2, T's diagonal and X^T published; the values, W^T's key part and G read
     if (tid == kIssuer && it_next >= 0) {
       tc::fence_async_smem();
       issue_v(it_next);
@@ -406,44 +454,93 @@ __global__ void __launch_bounds__(kDpThreads, 2)
       v_par = ph ^ 1u;
     }
 
-    // (I + A) delta = X, right-looking (A^T row t as 16-byte broadcast loads);
-    // rows past B touch only rows past B (A^T is zero there)
-#pragma unroll
-    for (int t = 0; t < BM; ++t) {
-      const float dt = x[t];
-      const float* ar = AT + t * kATs;
-#pragma unroll
-      for (int u4 = (t + 1) / 4; u4 < BM / 4; ++u4) {
-        const float4 a = *reinterpret_cast<const float4*>(ar + 4 * u4);
-        if (4 * u4 + 0 > t) x[4 * u4 + 0] = fmaf(-a.x, dt, x[4 * u4 + 0]);
-        if (4 * u4 + 1 > t) x[4 * u4 + 1] = fmaf(-a.y, dt, x[4 * u4 + 1]);
-        if (4 * u4 + 2 > t) x[4 * u4 + 2] = fmaf(-a.z, dt, x[4 * u4 + 2]);
-        if (4 * u4 + 3 > t) x[4 * u4 + 3] = fmaf(-a.w, dt, x[4 * u4 + 3]);
-      }
-    }
-    // delta^T as bf16 pairs (rows past B zero) over S0^T, which MMA 1 has read
+    // N = M2 T with T = (I + A)^{-1} from its diagonal blocks (rows and
+    // columns past B: M2 and A are zero there, T the identity).  Four lanes per
+    // row l of N, columns 4q .. 4q + 3 of each 16-column half; a row's values
+    // travel between its lanes by shuffles.
     {
-      uint32_t w[16];
+      const int l = tid >> 2, q = tid & 3, src0 = lane & ~3;
+      if (l < BM) {  // every lane of a warp alike
+        const float* m2r = M2f + l * kATs;
+        float w[16];  // the left factor of N0: Y = M2_0 - N1 A10 (BM = 32) or M2 (BM = 16)
+        float n1[4] = {0.f, 0.f, 0.f, 0.f};
+        if constexpr (BM == 32) {
+          float m1[16];
 #pragma unroll
-      for (int e = 0; e < 16; ++e) {
-        const int t = 2 * e;
-        float a = 0.f, b = 0.f;
-        if (t < BM) {
-          a = t < B ? x[t] : 0.f;
-          b = t + 1 < B ? x[t + 1] : 0.f;
+          for (int i4 = 0; i4 < 4; ++i4) {
+            const float4 v4 = *reinterpret_cast<const float4*>(m2r + 16 + 4 * i4);
+            m1[4 * i4] = v4.x, m1[4 * i4 + 1] = v4.y, m1[4 * i4 + 2] = v4.z, m1[4 * i4 + 3] = v4.w;
+          }
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {  // N1 = M2_1 T11
+            const float4 t4 = *reinterpret_cast<const float4*>(Tf + (16 + i) * kATs + 16 + 4 * q);
+            n1[0] = fmaf(m1[i], t4.x, n1[0]);
+            n1[1] = fmaf(m1[i], t4.y, n1[1]);
+            n1[2] = fmaf(m1[i], t4.z, n1[2]);
+            n1[3] = fmaf(m1[i], t4.w, n1[3]);
+          }
+          float v[16];  // N1's row l
+#pragma unroll
+          for (int i = 0; i < 16; ++i) v[i] = __shfl_sync(0xffffffffu, n1[i & 3], src0 + (i >> 2));
+          const float4 m0 = *reinterpret_cast<const float4*>(m2r + 4 * q);
+          float y[4] = {m0.x, m0.y, m0.z, m0.w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {  // Y = M2_0 - N1 A10, A[16 + i][4q + e] = A^T row 4q + e
+            const float* ar = AT + (4 * q + e) * kATs + 16;
+#pragma unroll
+            for (int i4 = 0; i4 < 4; ++i4) {
+              const float4 a4 = *reinterpret_cast<const float4*>(ar + 4 * i4);
+              y[e] = fmaf(-a4.x, v[4 * i4], y[e]);
+              y[e] = fmaf(-a4.y, v[4 * i4 + 1], y[e]);
+              y[e] = fmaf(-a4.z, v[4 * i4 + 2], y[e]);
+              y[e] = fmaf(-a4.w, v[4 * i4 + 3], y[e]);
+            }
+          }
+#pragma unroll
+          for (int i = 0; i < 16; ++i) w[i] = __shfl_sync(0xffffffffu, y[i & 3], src0 + (i >> 2));
+        } else {
+#pragma unroll
+          for (int i4 = 0; i4 < 4; ++i4) {
+            const float4 v4 = *reinterpret_cast<const float4*>(m2r + 4 * i4);
+            w[4 * i4] = v4.x, w[4 * i4 + 1] = v4.y, w[4 * i4 + 2] = v4.z, w[4 * i4 + 3] = v4.w;
+          }
         }
-        w[e] = dp_pack(a, b);
+        float n0[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {  // N0 = (.) T00
+          const float4 t4 = *reinterpret_cast<const float4*>(Tf + i * kATs + 4 * q);
+          n0[0] = fmaf(w[i], t4.x, n0[0]);
+          n0[1] = fmaf(w[i], t4.y, n0[1]);
+          n0[2] = fmaf(w[i], t4.z, n0[2]);
+          n0[3] = fmaf(w[i], t4.w, n0[3]);
+        }
+        // row l of N as bf16 high and low parts, K-major SW128 (columns c ..
+        // c + 3 in the 16-byte unit c / 8)
+        auto put4 = [&](int c, const float (&v)[4]) {
+          uint32_t h0, l0, h1, l1;
+          dp_split(v[0], v[1], h0, l0);
+          dp_split(v[2], v[3], h1, l1);
+          const int off = l * 128 + ((((c >> 3) ^ (l & 7))) << 4) + (c & 7) * 2;
+          *reinterpret_cast<uint2*>(Nbs + off) = make_uint2(h0, h1);
+          *reinterpret_cast<uint2*>(Nbs + BM * 128 + off) = make_uint2(l0, l1);
+        };
+        put4(4 * q, n0);
+        if constexpr (BM == 32) put4(16 + 4 * q, n1);
+        tc::fence_async_smem();  // N is the second MMA's operand
       }
-      tc::tmem_st16(tmS + lane_off, w);
     }
-    tc::tmem_st_wait();
     tc::fence_before_sync();
-    if (__syncthreads_or(bad)) break;  // delta^T complete; A^T read
+    if (__syncthreads_or(bad)) break;  // N complete; A^T, M2 and T read
     if (tid == kIssuer) {
       tc::fence_after_sync();
-      for (int kk = 0; kk < Bp / 16; ++kk)
-        tc::mma_bf16_ts(tmG, tmS + kk * 8, tc::sdesc_sw128(tc::smem_u32(M2s + kk * 32), 16, 1024),
-                        idO, kk > 0);  // O2^T = delta^T M2^T, over G
+#pragma unroll
+      for (int kk = 0; kk < BM / 16; ++kk) {  // O2^T = X^T N^T, over G
+        const uint64_t nh = tc::sdesc_sw128(tc::smem_u32(Nbs + kk * 32), 16, 1024);
+        const uint64_t nl = tc::sdesc_sw128(tc::smem_u32(Nbs + BM * 128 + kk * 32), 16, 1024);
+        tc::mma_bf16_ts(tmG, tmS + kk * 8, nh, idO, kk > 0);
+        tc::mma_bf16_ts(tmG, tmS + kk * 8, nl, idO, 1);
+        tc::mma_bf16_ts(tmG, tmS + BM / 2 + kk * 8, nh, idO, 1);
+      }
       tc::mma_commit(&sh.bar_mma);
       mma_out = true;
     }
