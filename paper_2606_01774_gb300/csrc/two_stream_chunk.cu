@@ -77,7 +77,7 @@ struct CkCfg {
 };
 
 struct alignas(16) CkShared {
-  uint64_t bar_s0, bar_kx, bar_v, bar_mma;
+  uint64_t bar_s0, bar_kx, bar_v, bar_g, bar_mma;
   uint32_t tmem_base;
   int abort_flag;
   alignas(16) float gc2[kCkC];  // clean gamma_t log2(e), from the chunk start
@@ -170,9 +170,9 @@ __device__ __forceinline__ void ck_diag_inverse(const float* AT, float* Tf, int 
 // loop.  Then the strips BC .. BC + nstrip - 1 (columns 16 BC ..) of T as bf16
 // high and low parts into Tb (K-major SW128 rows of 64 elements, zero above
 // the diagonal).
-template <int NT, int BC>
-__device__ __forceinline__ void ck_tcol(const float* AT, float* Tf, uint8_t* Tb, int nstrip, int q,
-                                        uint32_t bar_id) {
+template <int NT>
+__device__ __forceinline__ void ck_tcol(const float* AT, float* Tf, uint8_t* Tb, int BC, int nstrip,
+                                        int q, uint32_t bar_id) {
   constexpr int R = NT / 16, RPT = 16 / R;
   const int s = q / R, g = q % R, lane = q & 31;
   const int src0 = lane & ~(R - 1);  // the first lane of this column
@@ -288,6 +288,7 @@ __global__ void __launch_bounds__(kCkThreads, 1)
     tc::mbar_init(&sh.bar_s0, 1);
     tc::mbar_init(&sh.bar_kx, 1);
     tc::mbar_init(&sh.bar_v, 1);
+    tc::mbar_init(&sh.bar_g, 1);
     tc::mbar_init(&sh.bar_mma, 1);
     tc::fence_mbar_init();
   }
@@ -434,11 +435,19 @@ __global__ void __launch_bounds__(kCkThreads, 1)
       bad |= !tc::mbar_wait(&sh.bar_kx, ph, &sh.abort_flag);
       kx_out = false;
       tc::fence_after_sync();
+      // the Gram first, committed on its own: the tables are built from it
+      // while the state products run
 #pragma unroll
       for (int kk = 0; kk < kCkD / 16; ++kk) {
         const uint64_t kd = tc::sdesc_sw128(
             tc::smem_u32(KX + (kk >> 2) * (192 * 128) + (kk & 3) * 32), 16, 1024);
-        tc::mma_bf16_ss(tmG, kd, kd, id192, kk > 0);          // G = [K; K~] [K; K~; Q~]^T
+        tc::mma_bf16_ss(tmG, kd, kd, id192, kk > 0);  // G = [K; K~] [K; K~; Q~]^T
+      }
+      tc::mma_commit(&sh.bar_g);
+#pragma unroll
+      for (int kk = 0; kk < kCkD / 16; ++kk) {
+        const uint64_t kd = tc::sdesc_sw128(
+            tc::smem_u32(KX + (kk >> 2) * (192 * 128) + (kk & 3) * 32), 16, 1024);
         tc::mma_bf16_ts(tmW, tmS + kk * 8, kd, id192, kk > 0);  // W^T = S0^T [K; K~; Q~]^T
       }
       tc::mma_commit(&sh.bar_mma);
@@ -449,17 +458,8 @@ __global__ void __launch_bounds__(kCkThreads, 1)
         s0_par = ph ^ 1u;
       }
     }
-    bad |= !tc::mbar_wait(&sh.bar_mma, ph_mma, &sh.abort_flag);
-    ph_mma ^= 1u;
+    bad |= !tc::mbar_wait(&sh.bar_g, ph, &sh.abort_flag);
     tc::fence_after_sync();
-    if (tid == kIssuer) {
-      mma_out = false;
-      if (it_next >= 0) {  // the first MMAs, the readers of [K; K~; Q~], are done
-        issue_kx(it_next);
-        kx_out = true;
-        kx_par = ph ^ 1u;
-      }
-    }
 
     // ---- tables from G, 32 columns at a time.  Lanes 0..63 hold the rows of
     // K, 64..127 those of K~; every exponential is taken unconditionally and
@@ -486,7 +486,7 @@ __global__ void __launch_bounds__(kCkThreads, 1)
             }
             ck_store32(AT, row, 32 * h, v);
           }
-          tc::named_bar_arrive(4, 128);  // A^T to warps 4-5
+          tc::named_bar_arrive(5, 128);  // A^T to warps 4-5
         } else {
           // warps 2-3: A~ row t
           const float bt = sh.bn[row], gt = sh.gn2[row];
@@ -544,7 +544,7 @@ __global__ void __launch_bounds__(kCkThreads, 1)
           tc::fence_async_smem();  // P is the second MMA's operand
           // the diagonal blocks of T once warps 0-1 have written A^T: blocks
           // 2 (warp - 4) and 2 (warp - 4) + 1, a column of one per lane
-          tc::named_bar_sync(4, 128);
+          tc::named_bar_sync(5, 128);
           ck_diag_inverse(AT, Tf, 2 * (warp - 4) + (lane >> 4), lane & 15);
         } else {
           // warps 6-7: Aqk^T row i (noisy key i): exp(gamma~_end - gamma~_i) (q~_l . k~_i)
@@ -568,6 +568,17 @@ __global__ void __launch_bounds__(kCkThreads, 1)
     // ---- X = diag(beta) (V - diag(Gam) K S0), tokens 32 grp .. 32 grp + 31,
     // into tensor memory as bf16 high and low parts over S0^T (which the first
     // MMAs have read)
+    bad |= !tc::mbar_wait(&sh.bar_mma, ph_mma, &sh.abort_flag);
+    ph_mma ^= 1u;
+    tc::fence_after_sync();
+    if (tid == kIssuer) {
+      mma_out = false;
+      if (it_next >= 0) {  // the first MMAs, the readers of [K; K~; Q~], are done
+        issue_kx(it_next);
+        kx_out = true;
+        kx_par = ph ^ 1u;
+      }
+    }
     bad |= !tc::mbar_wait(&sh.bar_v, ph, &sh.abort_flag);
     if (tid == kIssuer) v_out = false;
     {
@@ -599,12 +610,12 @@ __global__ void __launch_bounds__(kCkThreads, 1)
 
     // ---- T = (I + A)^{-1} below its diagonal blocks: block column 0 on
     // warps 0-3, 1 on warps 4-5, 2 (and the strip of 3) on warps 6-7
+    // (columns 1 and 2 share one code path, the block column a run-time
+    // value: the groups run at once, so each copy crowds the instruction cache)
     if (warp < 4)
-      ck_tcol<128, 0>(AT, Tf, Vc, 1, tid, 1);
-    else if (warp < 6)
-      ck_tcol<64, 1>(AT, Tf, Vc, 1, tid - 128, 2);
+      ck_tcol<128>(AT, Tf, Vc, 0, 1, tid, 1);
     else
-      ck_tcol<64, 2>(AT, Tf, Vc, 2, tid - 192, 3);
+      ck_tcol<64>(AT, Tf, Vc, 1 + ((warp - 4) >> 1), warp < 6 ? 1 : 2, tid & 63, warp < 6 ? 2 : 3);
     if (__syncthreads_or(bad)) break;  // T as bf16 high / low parts
     if (tid == kIssuer) {
       const uint32_t tb = tc::smem_u32(Vc);
