@@ -211,12 +211,14 @@ flare_status flare_block_linear_attn(const flare_linear_desc* d, const void* q, 
   p.write_state = 0;
   p.dev_status = dev_status;
   const bool bf16 = d->act_dtype == FLARE_DT_BF16;
-  // bf16: the persistent tensor-core kernel for 128 x 128 states and B <= 32,
-  // the one-CTA-per-item tensor-core kernel for the other shapes; fp32 the
-  // CUDA-core recurrence
+  // bf16: the persistent tensor-core kernels for 128 x 128 states (B <= 32,
+  // and 33..64 as one chunk), the one-CTA-per-item tensor-core kernel for the
+  // other shapes; fp32 the CUDA-core recurrence
   cudaError_t e;
   if (bf16 && gdr_denoise_persist_supported(p.B, p.dk, p.dv))
     e = launch_gdr_denoise_persist(p, static_cast<cudaStream_t>(stream));
+  else if (bf16 && gdr_denoise_chunk64_supported(p.B, p.dk, p.dv))
+    e = launch_gdr_denoise_chunk64(p, static_cast<cudaStream_t>(stream));
   else if (bf16 && gdr_denoise_tc_supported(p.B, p.dk, p.dv))
     e = launch_gdr_denoise_tc(p, static_cast<cudaStream_t>(stream));
   else

@@ -74,6 +74,8 @@ size_t gdr_recurrent_smem_bytes(int dk, int dv, int threads);
 bool gdr_denoise_tc_supported(int B, int dk, int dv);
 bool gdr_denoise_persist_supported(int B, int dk, int dv);
 cudaError_t launch_gdr_denoise_persist(const GdrParams& p, cudaStream_t stream);
+bool gdr_denoise_chunk64_supported(int B, int dk, int dv);
+cudaError_t launch_gdr_denoise_chunk64(const GdrParams& p, cudaStream_t stream);
 cudaError_t launch_gdr_commit(const GdrParams& p, bool bf16, cudaStream_t stream);
 bool gdr_commit_tc_supported(int B, int dk, int dv);
 cudaError_t launch_gdr_commit_tc(const GdrParams& p, cudaStream_t stream);

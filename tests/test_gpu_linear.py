@@ -22,6 +22,9 @@ CASES = {
                                                      prefix_hi=70, seed=21),
     "d64_bf16": W["tiny_fp32"].replace(act_dtype="bf16", num_requests=3, num_v_heads=4,
                                        block_len=40, seed=22),
+    # 33..64 rows: the block as one chunk, rows past B zero
+    "ragged_block_b45": W["serving_batch64"].replace(num_requests=3, block_len=45, prefix_lo=0,
+                                                     prefix_hi=70, seed=23),
 }
 
 
