@@ -148,11 +148,17 @@ def verify_commit_bytes(spec, verify_len, accept):
 
 def kernel_of_call(spec):
     """The kernel each layer call of `spec` runs (the library's dispatch: bf16
-    128 x 128 states take the persistent denoise kernel for B <= 32 and the
-    tensor-core commit; other shapes the one-CTA-per-item kernels)."""
+    128 x 128 states take the persistent denoise kernels -- B <= 32, and 33..64
+    as one chunk -- and the tensor-core commit; other shapes the
+    one-CTA-per-item kernels)."""
     tc_state = spec.act_dtype == "bf16" and spec.head_dim_k == 128 and spec.head_dim_v == 128
-    return {"linear": ("gdr_denoise_persist_kernel" if tc_state and spec.block_len <= 32
-                       else "gdr_denoise_tc_kernel"),
+    if tc_state and spec.block_len <= 32:
+        linear = "gdr_denoise_persist_kernel"
+    elif tc_state and spec.block_len <= 64:
+        linear = "gdr_denoise_chunk64_kernel"
+    else:
+        linear = "gdr_denoise_tc_kernel"
+    return {"linear": linear,
             "softmax": "softmax_tc_kernel",
             "commit": "gdr_commit_tc_kernel" if tc_state else "gdr_commit_kernel",
             "shortconv": "short_conv_kernel", "shortconv_commit": "short_conv_kernel"}
