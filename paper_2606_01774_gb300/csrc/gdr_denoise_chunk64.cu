@@ -284,55 +284,50 @@ __global__ void __launch_bounds__(kD6Threads, 1)
     bad |= !tc::mbar_wait(&sh.bar_g, ph, &sh.abort_flag);
     tc::fence_after_sync();
 
-    // ---- tables from G, 32 columns at a time; every exponential is taken
-    // unconditionally and the masks applied as selects
-    if (grp == 0) {
+    // ---- tables from G, each group 32 of the 64 columns; every exponential
+    // is taken unconditionally and the masks applied as selects
+    {
       const int row = col & 63;
+      const int h = grp;  // columns 32 h .. 32 h + 31
+      uint32_t gr[32];
+      ck_ld32(tmG + lane_off + 32 * h, gr);
       if (col < 64) {
-        // warps 0-1: A^T row i (G's key row i)
+        // warps 0-1 and 4-5: A^T row i (G's key row i)
         const float gi = sh.gc2[row];
-#pragma unroll 1
-        for (int h = 0; h < 2; ++h) {
-          uint32_t gr[32];
-          float v[32];
-          ck_ld32(tmG + lane_off + 32 * h, gr);
+        float v[32];
 #pragma unroll
-          for (int k = 0; k < 32; ++k) {
-            const int t = 32 * h + k;
-            const float a = sh.bc[t] * tc::ex2(sh.gc2[t] - gi) * __uint_as_float(gr[k]);
-            v[k] = t > row ? a : 0.f;
-          }
-          ck_store32(AT, row, 32 * h, v);
+        for (int k = 0; k < 32; ++k) {
+          const int t = 32 * h + k;
+          const float a = sh.bc[t] * tc::ex2(sh.gc2[t] - gi) * __uint_as_float(gr[k]);
+          v[k] = t > row ? a : 0.f;
         }
-        tc::named_bar_arrive(5, 128);  // A^T to warps 4-5
+        ck_store32(AT, row, 32 * h, v);
+        if (grp == 0) {
+          tc::named_bar_arrive(5, 128);  // A^T to warps 4-5
+        } else {
+          // warps 4-5: T's diagonal blocks once both halves of A^T are in
+          tc::named_bar_sync(5, 128);
+          ck_diag_inverse(AT, Tf, 2 * (warp - 4) + (lane >> 4), lane & 15);
+        }
       } else {
-        // warps 2-3: M2 row l (G's query row l), bf16 K-major SW128
+        // warps 2-3 and 6-7: M2 row l (G's query row l), bf16 K-major SW128
         const bool live = row < B;
-#pragma unroll 1
-        for (int h = 0; h < 2; ++h) {
-          uint32_t gr[32];
-          ck_ld32(tmG + lane_off + 32 * h, gr);
 #pragma unroll
-          for (int u4 = 0; u4 < 4; ++u4) {  // 16-byte units of 8 columns
-            const int u = 4 * h + u4;
-            uint32_t w[4];
+        for (int u4 = 0; u4 < 4; ++u4) {  // 16-byte units of 8 columns
+          const int u = 4 * h + u4;
+          uint32_t w[4];
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const int i = 8 * u + 2 * e;
-              const float m0 = sh.eB[i] * __uint_as_float(gr[8 * u4 + 2 * e]);
-              const float m1 = sh.eB[i + 1] * __uint_as_float(gr[8 * u4 + 2 * e + 1]);
-              w[e] = ck_pack(live ? m0 : 0.f, live ? m1 : 0.f);
-            }
-            *reinterpret_cast<uint4*>(M2s + row * 128 + ((u ^ (row & 7)) << 4)) =
-                make_uint4(w[0], w[1], w[2], w[3]);
+          for (int e = 0; e < 4; ++e) {
+            const int i = 8 * u + 2 * e;
+            const float m0 = sh.eB[i] * __uint_as_float(gr[8 * u4 + 2 * e]);
+            const float m1 = sh.eB[i + 1] * __uint_as_float(gr[8 * u4 + 2 * e + 1]);
+            w[e] = ck_pack(live ? m0 : 0.f, live ? m1 : 0.f);
           }
+          *reinterpret_cast<uint4*>(M2s + row * 128 + ((u ^ (row & 7)) << 4)) =
+              make_uint4(w[0], w[1], w[2], w[3]);
         }
         tc::fence_async_smem();  // M2 is the second MMA's operand
       }
-    } else if (warp < 6) {
-      // warps 4-5: T's diagonal blocks once warps 0-1 have written A^T
-      tc::named_bar_sync(5, 128);
-      ck_diag_inverse(AT, Tf, 2 * (warp - 4) + (lane >> 4), lane & 15);
     }
 
     // ---- X = diag(beta) (V - diag(Gam) K S0), tokens 32 grp .. 32 grp + 31,
