@@ -45,8 +45,13 @@ def test_bounded_wait_gives_up_and_reports():
     assert torch.isfinite(out.float()).all()
 
 
-def test_bad_state_slot_sets_bit_and_skips_request():
-    spec = reduced(W["small_model_batch256"], 3)
+@pytest.mark.parametrize("name,args", [("small_model_batch256", ()),
+                                       ("serving_batch64", (64, 200)),
+                                       ("multistep_batch128", (100, 900))])
+def test_bad_state_slot_sets_bit_and_skips_request(name, args):
+    """Each denoise kernel (B = 16 and 32 persistent, B = 64 as one chunk)
+    skips a request whose slot is out of range and flags it."""
+    spec = reduced(W[name], 3, *args)
     w = gen(spec)
     install_states(w)
     nslots = w.state_pool.shape[0]

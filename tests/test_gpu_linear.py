@@ -25,6 +25,8 @@ CASES = {
     # 33..64 rows: the block as one chunk, rows past B zero
     "ragged_block_b45": W["serving_batch64"].replace(num_requests=3, block_len=45, prefix_lo=0,
                                                      prefix_hi=70, seed=23),
+    "ragged_block_b33": W["serving_batch64"].replace(num_requests=2, block_len=33, prefix_lo=0,
+                                                     prefix_hi=70, seed=24),
 }
 
 
