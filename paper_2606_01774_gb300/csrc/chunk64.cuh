@@ -82,9 +82,9 @@ __device__ __forceinline__ void ck_diag_inverse(const float* AT, float* Tf, int 
 }
 
 // Block column BC of T below its diagonal block.  Column s of the block
-// column lives on R = NT / 16 adjacent lanes, lane g holding rows g RPT ..
-// g RPT + RPT - 1 of every block (RPT = 16 / R), so that all of its
-// dependencies travel by shuffles.
+// column lives on R = NT / 16 adjacent lanes (NT = 32, 64 or 128), lane g
+// holding rows g RPT .. g RPT + RPT - 1 of every block (RPT = 16 / R), so
+// that all of its dependencies travel by shuffles.
 // Right-looking (T_c,BC = -T_cc sum_{BC <= d < c} A_cd T_d,BC): once block d
 // of the column is known, acc_a += A_ad T_d,BC for every a > d, and the next
 // block is T_d+1,BC = -T_d+1,d+1 acc_d+1.  The accumulators are a shift
@@ -115,13 +115,17 @@ __device__ __forceinline__ void ck_tcol(const float* AT, float* Tf, uint8_t* Tb,
       if (a < 4) {
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
-          float av[RPT];
-          const float* ap = AT + ck_sw(16 * d + i, 16 * a + g * RPT);  // A[16a + g RPT ..][16d + i]
-          if constexpr (RPT == 4) {
-            const float4 v4 = *reinterpret_cast<const float4*>(ap);
-            av[0] = v4.x; av[1] = v4.y; av[2] = v4.z; av[3] = v4.w;
+          float av[RPT];  // A[16a + g RPT ..][16d + i], 16-byte units addressed one by one
+          if constexpr (RPT >= 4) {
+#pragma unroll
+            for (int e4 = 0; e4 < RPT / 4; ++e4) {
+              const float4 v4 = *reinterpret_cast<const float4*>(
+                  AT + ck_sw(16 * d + i, 16 * a + g * RPT + 4 * e4));
+              av[4 * e4] = v4.x; av[4 * e4 + 1] = v4.y; av[4 * e4 + 2] = v4.z; av[4 * e4 + 3] = v4.w;
+            }
           } else {
-            const float2 v2 = *reinterpret_cast<const float2*>(ap);
+            const float2 v2 =
+                *reinterpret_cast<const float2*>(AT + ck_sw(16 * d + i, 16 * a + g * RPT));
             av[0] = v2.x; av[1] = v2.y;
           }
 #pragma unroll

@@ -11,11 +11,11 @@
 //   X       = diag(beta) (V - diag(Gam) K S0),   delta = (I + A)^{-1} X
 //   out[l]  = s (Gam_{B-1} S0^T q_l + sum_i exp(gamma_{B-1} - gamma_i) (q_l . k_i) delta_i)
 //
-// Value column c on tensor-memory lane c.  Per item:
+// Value column c on tensor-memory lane c; thread c owns column c.  Per item:
 //   MMA 1  G   = [K; Q] K^T       M=128 (K rows on lanes 0..63, Q rows on 64..127), N=64, K=128
 //          W^T = S0^T [K; Q]^T    M=128 (c), N=128, K=128   (A: S0^T bf16, tensor memory)
 //   T      = (I + A)^{-1}          fp32, 16 x 16 blocks: the diagonal ones by forward
-//                                  substitution, then block columns (all warps)
+//                                  substitution, then block columns
 //   MMA d  delta^T = X^T T^T      M=128, N=64, K=64  (X and T as bf16 high + low parts,
 //                                  three products: fp32-grade delta)
 //   MMA 2  O2^T = delta^T M2^T    M=128, N=64, K=64  (delta^T bf16, tensor memory;
@@ -24,14 +24,17 @@
 // Rows past B read as zero (the block's tensor maps end at B), so A, M2 and X
 // vanish there and T is the identity.
 //
-// Persistent CTAs, one per SM (152 KiB of shared memory, 512 tensor-memory
-// columns), 256 threads: warps 0-3 and 4-7 are two groups on the same 128
-// lanes.  The next item's state streams into the state buffer as soon as it
-// has been turned into S0^T, its keys and queries once the first MMAs are
-// done, its values once this item's T (held in the values' buffer) has been
-// read; its gates are loaded into registers one item ahead.  Every wait is
-// bounded: on a timeout the CTA sets FLARE_DEV_WAIT_TIMEOUT, waits (bounded)
-// for its copies and MMAs in flight, frees its tensor memory and exits.
+// Persistent CTAs, two per SM (81 KiB of shared memory, 256 tensor-memory
+// columns and 128 threads each), so that each SM holds two items' latency
+// chains.  The buffers serve twice: the state arrives in two 32 KiB halves
+// into one buffer that then holds A^T and T; the key/query buffer holds M2
+// and T's bf16 parts once the first MMAs have read it; delta^T's fp32 product
+// lands over W^T's key columns, which X has read.  The next item's first
+// state half is requested once T is formed, its keys and queries once the
+// second MMA has read M2, its values once X has read this item's; its gates
+// are loaded into registers one item ahead.  Every wait is bounded: on a
+// timeout the CTA sets FLARE_DEV_WAIT_TIMEOUT, waits (bounded) for its copies
+// and MMAs in flight, frees its tensor memory and exits.
 #include <cudaTypedefs.h>
 
 #include "chunk64.cuh"
@@ -43,25 +46,25 @@ namespace flare {
 
 namespace {
 
-constexpr int kD6Threads = 256;
+constexpr int kD6Threads = 128;
 constexpr int kD6D = 128;  // d_k = d_v
 using namespace chunk64;   // kCkC = 64 and the chunk-system helpers
 
 struct D6Cfg {
-  static constexpr int kS0 = kD6D * kD6D * 4;   // S0 fp32 [i][c]
-  static constexpr int kKQ = 2 * 128 * 128;     // [K; Q]: 2 chunks of 128 rows x 128 B (SW128)
-  static constexpr int kV = 2 * kCkC * 128;     // values: 2 chunks of 64 rows x 128 B
-  static constexpr int kT = kCkC * kCkC * 4;    // a 64 x 64 fp32 table
-  static constexpr int kM2 = kCkC * 128;        // M2 [l][i] bf16, K-major SW128
-  static constexpr int oS0 = 0;
-  static constexpr int oKQ = oS0 + kS0;
+  static constexpr int kS0h = 64 * kD6D * 4;   // half of S0 fp32: rows 64 h .. 64 h + 63
+  static constexpr int kKQ = 2 * 128 * 128;    // [K; Q]: 2 chunks of 128 rows x 128 B (SW128)
+  static constexpr int kV = 2 * kCkC * 128;    // values: 2 chunks of 64 rows x 128 B
+  static constexpr int kT = kCkC * kCkC * 4;   // a 64 x 64 fp32 table
+  static constexpr int kM2 = kCkC * 128;       // M2 [l][i] bf16, K-major SW128
+  static constexpr int oS0 = 0;                // the state half; then A^T and T
+  static constexpr int oAT = oS0;
+  static constexpr int oT = oS0 + kT;
+  static constexpr int oKQ = oS0 + kS0h;       // [K; Q]; then M2 and T's bf16 parts
+  static constexpr int oM2 = oKQ;
+  static constexpr int oTb = oKQ + kM2;        // T high, then low (8 KiB each)
   static constexpr int oV = oKQ + kKQ;
-  static constexpr int oAT = oV + kV;   // A^T[i][t]
-  static constexpr int oM2 = oAT + kT;
-  static constexpr int oT = oM2 + kM2;  // T[t][j] fp32, the lower blocks
-  static constexpr int kSmem = oT + kT;
-  // once the values are read, their buffer holds T as bf16 high and low parts
-  // (K-major SW128, rows of 64 elements, 8 KiB each): MMA d's operand
+  static constexpr int kSmem = oV + kV;
+  static_assert(2 * kT <= kS0h && kM2 + 2 * 8192 <= kKQ, "buffer reuse");
 };
 
 struct alignas(16) D6Shared {
@@ -97,7 +100,7 @@ __device__ __forceinline__ int d6_next(const GdrParams& p, int it, int total, in
 
 }  // namespace
 
-__global__ void __launch_bounds__(kD6Threads, 1)
+__global__ void __launch_bounds__(kD6Threads, 2)
     gdr_denoise_chunk64_kernel(const __grid_constant__ D6Maps maps, GdrParams p) {
   using C = D6Cfg;
   constexpr int kIssuer = 32;  // one thread of warp 1 issues every copy and MMA
@@ -105,14 +108,14 @@ __global__ void __launch_bounds__(kD6Threads, 1)
   __shared__ D6Shared sh;
   uint8_t* base = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   float* S0s = reinterpret_cast<float*>(base + C::oS0);
-  uint8_t* KQ = base + C::oKQ;
-  uint8_t* Vs = base + C::oV;
   float* AT = reinterpret_cast<float*>(base + C::oAT);
-  uint8_t* M2s = base + C::oM2;
   float* Tf = reinterpret_cast<float*>(base + C::oT);
+  uint8_t* KQ = base + C::oKQ;
+  uint8_t* M2s = base + C::oM2;
+  uint8_t* Tb = base + C::oTb;
+  uint8_t* Vs = base + C::oV;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int col = tid & 127, grp = tid >> 7;  // value column (= lane of tensor memory), group
   const int total = p.R * p.Hv;
   const int B = p.B;
 
@@ -129,21 +132,21 @@ __global__ void __launch_bounds__(kD6Threads, 1)
     tc::mbar_init(&sh.bar_mma, 1);
     tc::fence_mbar_init();
   }
-  if (warp == 0) tc::tmem_alloc(&sh.tmem_base, 512);
+  if (warp == 0) tc::tmem_alloc(&sh.tmem_base, 256);
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = sh.tmem_base;
   const uint32_t tmS = tmem;        // S0^T bf16 (64 columns); X^T high | low; delta^T (32)
-  const uint32_t tmW = tmem + 64;   // W^T: [K | Q] parts, 2 x 64 columns
+  const uint32_t tmW = tmem + 64;   // W^T: [K | Q] parts, 2 x 64 columns; delta^T fp32 over K
   const uint32_t tmG = tmem + 192;  // G (rows on lanes), 64 columns; then O2^T
-  const uint32_t tmD = tmem + 256;  // delta^T fp32, 64 columns
-  const uint32_t lane_off = (uint32_t)((warp & 3) * 32) << 16;
+  const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
 
-  auto issue_s0 = [&](int item, int s) {
-    const float* src = p.state_pool + ((size_t)s * p.Hv + item % p.Hv) * kD6D * kD6D;
-    tc::mbar_expect_tx(&sh.bar_s0, C::kS0);
-    tc::bulk_load(S0s, src, C::kS0, &sh.bar_s0);
+  auto issue_s0 = [&](int item, int s, int h) {  // rows 64 h .. 64 h + 63 of the state
+    const float* src = p.state_pool + ((size_t)s * p.Hv + item % p.Hv) * kD6D * kD6D +
+                       (size_t)h * 64 * kD6D;
+    tc::mbar_expect_tx(&sh.bar_s0, C::kS0h);
+    tc::bulk_load(S0s, src, C::kS0h, &sh.bar_s0);
   };
   auto issue_kq = [&](int item) {
     const int r = item / p.Hv, h = (item % p.Hv) / (p.Hv / p.Hk);
@@ -177,14 +180,16 @@ __global__ void __launch_bounds__(kD6Threads, 1)
   // barrier phase completes with), for a clean exit after a timeout
   bool s0_out = false, kq_out = false, v_out = false, mma_out = false;
   uint32_t s0_par = 0, kq_par = 0, v_par = 0;
+  uint32_t s0_ph = 0;  // parity of the state buffer's next completion (two per item)
   if (tid == kIssuer) {
     tc::prefetch_tmap(&maps.k);
     tc::prefetch_tmap(&maps.q);
     tc::prefetch_tmap(&maps.v);
-    issue_s0(it, slot);
+    issue_s0(it, slot, 0);
     issue_kq(it);
     issue_v(it);
     s0_out = kq_out = v_out = true;
+    s0_par = 0;
   }
   if (warp == 0) load_gates(it);
   int cand = it + gridDim.x;
@@ -213,7 +218,7 @@ __global__ void __launch_bounds__(kD6Threads, 1)
       }
       x1 += __shfl_sync(0xffffffffu, x0, 31);
       const float g0 = x0 * 1.4426950408889634f, g1 = x1 * 1.4426950408889634f;
-      const float gB = B > 32 ? __shfl_sync(0xffffffffu, g1, B - 33) : __shfl_sync(0xffffffffu, g0, B - 1);
+      const float gB = __shfl_sync(0xffffffffu, g1, B - 33);  // B > 32
       sh.gc2[lane] = g0;
       sh.gc2[lane + 32] = g1;
       sh.Gc[lane] = expf(x0);
@@ -240,20 +245,33 @@ __global__ void __launch_bounds__(kD6Threads, 1)
       cs = cand_slot(cand);
     }
 
-    bad |= !tc::mbar_wait(&sh.bar_s0, ph, &sh.abort_flag);
-    if (tid == kIssuer) s0_out = false;
-    // S0^T into tensor memory as bf16 pairs, each group half of the rows
+    // S0^T into tensor memory as bf16 pairs, the state in two halves through
+    // one buffer
 #pragma unroll 1
-    for (int i0 = grp * 64; i0 < grp * 64 + 64; i0 += 32) {
-      uint32_t w[16];
+    for (int h = 0; h < 2; ++h) {
+      bad |= !tc::mbar_wait(&sh.bar_s0, s0_ph, &sh.abort_flag);
+      s0_ph ^= 1u;
+      if (tid == kIssuer) s0_out = false;
+#pragma unroll 1
+      for (int i0 = 0; i0 < 64; i0 += 32) {
+        uint32_t w[16];
 #pragma unroll
-      for (int e = 0; e < 16; ++e)
-        w[e] = ck_pack(S0s[(i0 + 2 * e) * kD6D + col], S0s[(i0 + 2 * e + 1) * kD6D + col]);
-      tc::tmem_st16(tmS + lane_off + i0 / 2, w);
+        for (int e = 0; e < 16; ++e)
+          w[e] = ck_pack(S0s[(i0 + 2 * e) * kD6D + tid], S0s[(i0 + 2 * e + 1) * kD6D + tid]);
+        tc::tmem_st16(tmS + lane_off + (64 * h + i0) / 2, w);
+      }
+      bad = __syncthreads_or(bad);  // this half read
+      if (bad) break;
+      if (h == 0 && tid == kIssuer) {
+        issue_s0(it, slot, 1);
+        s0_out = true;
+        s0_par = s0_ph;
+      }
     }
+    if (bad) break;
     tc::tmem_st_wait();
     tc::fence_before_sync();
-    if (__syncthreads_or(bad)) break;  // S0^T complete, the state buffer read
+    if (__syncthreads_or(bad)) break;  // S0^T complete
     if (tid == kIssuer) {
       bad |= !tc::mbar_wait(&sh.bar_kq, ph, &sh.abort_flag);
       kq_out = false;
@@ -275,120 +293,119 @@ __global__ void __launch_bounds__(kD6Threads, 1)
       }
       tc::mma_commit(&sh.bar_mma);
       mma_out = true;
-      if (it_next >= 0) {  // the state buffer is free
-        issue_s0(it_next, slot_next);
-        s0_out = true;
-        s0_par = ph ^ 1u;
-      }
     }
     bad |= !tc::mbar_wait(&sh.bar_g, ph, &sh.abort_flag);
     tc::fence_after_sync();
 
-    // ---- tables from G, each group 32 of the 64 columns; every exponential
-    // is taken unconditionally and the masks applied as selects
+    // ---- tables from G (every exponential taken unconditionally, the masks
+    // applied as selects): warps 0-1 A^T (key rows), warps 2-3 M2 (query rows,
+    // stored over [K; Q] once the state products have read it) and then T's
+    // diagonal blocks
     {
-      const int row = col & 63;
-      const int h = grp;  // columns 32 h .. 32 h + 31
-      uint32_t gr[32];
-      ck_ld32(tmG + lane_off + 32 * h, gr);
-      if (col < 64) {
-        // warps 0-1 and 4-5: A^T row i (G's key row i)
+      const int row = tid & 63;
+      if (tid < 64) {
         const float gi = sh.gc2[row];
-        float v[32];
+#pragma unroll 1
+        for (int h = 0; h < 2; ++h) {
+          uint32_t gr[32];
+          float v[32];
+          ck_ld32(tmG + lane_off + 32 * h, gr);
 #pragma unroll
-        for (int k = 0; k < 32; ++k) {
-          const int t = 32 * h + k;
-          const float a = sh.bc[t] * tc::ex2(sh.gc2[t] - gi) * __uint_as_float(gr[k]);
-          v[k] = t > row ? a : 0.f;
-        }
-        ck_store32(AT, row, 32 * h, v);
-        if (grp == 0) {
-          tc::named_bar_arrive(5, 128);  // A^T to warps 4-5
-        } else {
-          // warps 4-5: T's diagonal blocks once both halves of A^T are in
-          tc::named_bar_sync(5, 128);
-          ck_diag_inverse(AT, Tf, 2 * (warp - 4) + (lane >> 4), lane & 15);
-        }
-      } else {
-        // warps 2-3 and 6-7: M2 row l (G's query row l), bf16 K-major SW128
-        const bool live = row < B;
-#pragma unroll
-        for (int u4 = 0; u4 < 4; ++u4) {  // 16-byte units of 8 columns
-          const int u = 4 * h + u4;
-          uint32_t w[4];
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const int i = 8 * u + 2 * e;
-            const float m0 = sh.eB[i] * __uint_as_float(gr[8 * u4 + 2 * e]);
-            const float m1 = sh.eB[i + 1] * __uint_as_float(gr[8 * u4 + 2 * e + 1]);
-            w[e] = ck_pack(live ? m0 : 0.f, live ? m1 : 0.f);
+          for (int k = 0; k < 32; ++k) {
+            const int t = 32 * h + k;
+            const float a = sh.bc[t] * tc::ex2(sh.gc2[t] - gi) * __uint_as_float(gr[k]);
+            v[k] = t > row ? a : 0.f;
           }
-          *reinterpret_cast<uint4*>(M2s + row * 128 + ((u ^ (row & 7)) << 4)) =
-              make_uint4(w[0], w[1], w[2], w[3]);
+          ck_store32(AT, row, 32 * h, v);
         }
+        tc::named_bar_arrive(5, 128);  // A^T to warps 2-3
+      } else {
+        const bool live = row < B;
+        uint32_t wv[32];  // the row's 64 values as bf16 pairs
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          uint32_t gr[32];
+          ck_ld32(tmG + lane_off + 32 * h, gr);
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            const int i = 32 * h + 2 * e;
+            const float m0 = sh.eB[i] * __uint_as_float(gr[2 * e]);
+            const float m1 = sh.eB[i + 1] * __uint_as_float(gr[2 * e + 1]);
+            wv[16 * h + e] = ck_pack(live ? m0 : 0.f, live ? m1 : 0.f);
+          }
+        }
+        bad |= !tc::mbar_wait(&sh.bar_mma, ph_mma, &sh.abort_flag);  // [K; Q] read
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          *reinterpret_cast<uint4*>(M2s + row * 128 + ((u ^ (row & 7)) << 4)) =
+              make_uint4(wv[4 * u], wv[4 * u + 1], wv[4 * u + 2], wv[4 * u + 3]);
         tc::fence_async_smem();  // M2 is the second MMA's operand
+        tc::named_bar_sync(5, 128);
+        ck_diag_inverse(AT, Tf, 2 * (warp - 2) + (lane >> 4), lane & 15);
       }
     }
 
-    // ---- X = diag(beta) (V - diag(Gam) K S0), tokens 32 grp .. 32 grp + 31,
-    // into tensor memory as bf16 high and low parts over S0^T (which the first
-    // MMAs have read)
+    // ---- X = diag(beta) (V - diag(Gam) K S0), all 64 tokens, into tensor
+    // memory as bf16 high and low parts over S0^T (which the first MMAs have read)
     bad |= !tc::mbar_wait(&sh.bar_mma, ph_mma, &sh.abort_flag);
     ph_mma ^= 1u;
     tc::fence_after_sync();
-    if (tid == kIssuer) {
-      mma_out = false;
-      if (it_next >= 0) {  // the first MMAs, the readers of [K; Q], are done
-        issue_kq(it_next);
-        kq_out = true;
-        kq_par = ph ^ 1u;
-      }
-    }
+    if (tid == kIssuer) mma_out = false;
     bad |= !tc::mbar_wait(&sh.bar_v, ph, &sh.abort_flag);
     if (tid == kIssuer) v_out = false;
     {
-      const int t0 = 32 * grp;
-      uint32_t w0[16], w1[16], hi[16], lo[16];
-      tc::tmem_ld16(tmW + lane_off + t0, w0);
-      tc::tmem_ld16(tmW + lane_off + t0 + 16, w1);
-      tc::tmem_ld_wait();
-      const uint8_t* vb = Vs + (col >> 6) * (kCkC * 128) + (col & 63) * 2;
+      const uint8_t* vb = Vs + (tid >> 6) * (kCkC * 128) + (tid & 63) * 2;
+#pragma unroll 1
+      for (int h = 0; h < 2; ++h) {
+        const int t0 = 32 * h;
+        uint32_t w[32], hi[16], lo[16];
+        ck_ld32(tmW + lane_off + t0, w);
 #pragma unroll
-      for (int e = 0; e < 16; ++e) {
-        float xv[2];
+        for (int e = 0; e < 16; ++e) {
+          float xv[2];
 #pragma unroll
-        for (int f = 0; f < 2; ++f) {
-          const int u = 2 * e + f, t = t0 + u;
-          const float vt = __uint_as_float(
-              (uint32_t)*reinterpret_cast<const unsigned short*>(vb + t * 128) << 16);
-          const float wt = __uint_as_float(u < 16 ? w0[u & 15] : w1[u & 15]);
-          xv[f] = sh.bc[t] * (vt - sh.Gc[t] * wt);
+          for (int f = 0; f < 2; ++f) {
+            const int u = 2 * e + f, t = t0 + u;
+            const float vt = __uint_as_float(
+                (uint32_t)*reinterpret_cast<const unsigned short*>(vb + t * 128) << 16);
+            xv[f] = sh.bc[t] * (vt - sh.Gc[t] * __uint_as_float(w[u]));
+          }
+          ck_split(xv[0], xv[1], hi[e], lo[e]);
         }
-        ck_split(xv[0], xv[1], hi[e], lo[e]);
+        tc::tmem_st16(tmS + lane_off + 16 * h, hi);
+        tc::tmem_st16(tmS + lane_off + 32 + 16 * h, lo);
       }
-      tc::tmem_st16(tmS + lane_off + 16 * grp, hi);
-      tc::tmem_st16(tmS + lane_off + 32 + 16 * grp, lo);
       tc::tmem_st_wait();
     }
     tc::fence_before_sync();
     if (__syncthreads_or(bad)) break;  // tables, T's diagonal blocks, X^T; G and V read
+    if (tid == kIssuer && it_next >= 0) {
+      issue_v(it_next);
+      v_out = true;
+      v_par = ph ^ 1u;
+    }
 
     // ---- T = (I + A)^{-1} below its diagonal blocks: block column 0 on
-    // warps 0-3, 1 on warps 4-5, 2 (and the strip of 3) on warps 6-7
-    if (warp < 4)
-      ck_tcol<128>(AT, Tf, Vs, 0, 1, tid, 1);
+    // warps 0-1, 1 on warp 2, 2 (and the strip of 3) on warp 3
+    if (warp < 2)
+      ck_tcol<64>(AT, Tf, Tb, 0, 1, tid, 1);
     else
-      ck_tcol<64>(AT, Tf, Vs, 1 + ((warp - 4) >> 1), warp < 6 ? 1 : 2, tid & 63, warp < 6 ? 2 : 3);
-    if (__syncthreads_or(bad)) break;  // T as bf16 high / low parts
+      ck_tcol<32>(AT, Tf, Tb, warp - 1, warp == 2 ? 1 : 2, lane, warp);
+    if (__syncthreads_or(bad)) break;  // T as bf16 high / low parts; A^T and T read
     if (tid == kIssuer) {
-      const uint32_t tb = tc::smem_u32(Vs);
+      if (it_next >= 0) {  // the state buffer is free: the next item's first half
+        issue_s0(it_next, slot_next, 0);
+        s0_out = true;
+        s0_par = s0_ph;
+      }
+      const uint32_t tb = tc::smem_u32(Tb);
 #pragma unroll
       for (int kk = 0; kk < kCkC / 16; ++kk) {
         const uint64_t bh = tc::sdesc_sw128(tb + kk * 32, 16, 1024);
         const uint64_t bl = tc::sdesc_sw128(tb + 8192 + kk * 32, 16, 1024);
-        tc::mma_bf16_ts(tmD, tmS + kk * 8, bh, id64, kk > 0);  // delta^T = X^T T^T
-        tc::mma_bf16_ts(tmD, tmS + kk * 8, bl, id64, 1);
-        tc::mma_bf16_ts(tmD, tmS + 32 + kk * 8, bh, id64, 1);
+        tc::mma_bf16_ts(tmW, tmS + kk * 8, bh, id64, kk > 0);  // delta^T = X^T T^T
+        tc::mma_bf16_ts(tmW, tmS + kk * 8, bl, id64, 1);
+        tc::mma_bf16_ts(tmW, tmS + 32 + kk * 8, bh, id64, 1);
       }
       tc::mma_commit(&sh.bar_mma);
       mma_out = true;
@@ -397,20 +414,16 @@ __global__ void __launch_bounds__(kD6Threads, 1)
     ph_mma ^= 1u;
     tc::fence_after_sync();
     if (tid == kIssuer) mma_out = false;
-    // delta^T as bf16 pairs over X^T's high part, tokens 32 grp .. 32 grp + 31
-    {
-      uint32_t d0[16], d1[16], w[16];
-      tc::tmem_ld16(tmD + lane_off + 32 * grp, d0);
-      tc::tmem_ld16(tmD + lane_off + 32 * grp + 16, d1);
-      tc::tmem_ld_wait();
+    // delta^T as bf16 pairs over X^T's high part
+#pragma unroll 1
+    for (int h = 0; h < 2; ++h) {
+      uint32_t d[32], w[16];
+      ck_ld32(tmW + lane_off + 32 * h, d);
 #pragma unroll
-      for (int e = 0; e < 8; ++e) {
-        w[e] = ck_pack(__uint_as_float(d0[2 * e]), __uint_as_float(d0[2 * e + 1]));
-        w[8 + e] = ck_pack(__uint_as_float(d1[2 * e]), __uint_as_float(d1[2 * e + 1]));
-      }
-      tc::tmem_st16(tmS + lane_off + 16 * grp, w);
-      tc::tmem_st_wait();
+      for (int e = 0; e < 16; ++e) w[e] = ck_pack(__uint_as_float(d[2 * e]), __uint_as_float(d[2 * e + 1]));
+      tc::tmem_st16(tmS + lane_off + 16 * h, w);
     }
+    tc::tmem_st_wait();
     tc::fence_before_sync();
     if (__syncthreads_or(bad)) break;  // delta^T complete
     if (tid == kIssuer) {
@@ -425,44 +438,47 @@ __global__ void __launch_bounds__(kD6Threads, 1)
     bad |= !tc::mbar_wait(&sh.bar_mma, ph_mma, &sh.abort_flag);
     ph_mma ^= 1u;
     tc::fence_after_sync();
-    if (tid == kIssuer) mma_out = false;
-
-    // ---- out[l][c] = s (Gam_{B-1} W^T[c][64 + l] + O2^T[c][l]), rows 32 grp
-    // .. 32 grp + 31; adjacent lanes swap one value so that each stores a bf16
-    // pair of two columns
-    {
-      const int t0 = 32 * grp;
-      const float sG = p.scale * sh.Gc[B - 1];
-      uint32_t o2[32], wq[32];
-      tc::tmem_ld16(tmG + lane_off + t0, *reinterpret_cast<uint32_t(*)[16]>(&o2[0]));
-      tc::tmem_ld16(tmG + lane_off + t0 + 16, *reinterpret_cast<uint32_t(*)[16]>(&o2[16]));
-      tc::tmem_ld16(tmW + lane_off + 64 + t0, *reinterpret_cast<uint32_t(*)[16]>(&wq[0]));
-      tc::tmem_ld16(tmW + lane_off + 64 + t0 + 16, *reinterpret_cast<uint32_t(*)[16]>(&wq[16]));
-      tc::tmem_ld_wait();
-      const bool odd = lane & 1;
-      __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.out_blockend) +
-                           ((size_t)r * B * p.Hv + j) * kD6D + (col & ~1);
-#pragma unroll
-      for (int l = 0; l < 32; l += 2) {
-        const float a = fmaf(sG, __uint_as_float(wq[l]), p.scale * __uint_as_float(o2[l]));
-        const float b =
-            fmaf(sG, __uint_as_float(wq[l + 1]), p.scale * __uint_as_float(o2[l + 1]));
-        const float recv = __shfl_xor_sync(0xffffffffu, odd ? a : b, 1);
-        const int row = t0 + (odd ? l + 1 : l);
-        if (row < B)
-          *reinterpret_cast<uint32_t*>(out + (size_t)row * p.Hv * kD6D) =
-              odd ? ck_pack(recv, b) : ck_pack(a, recv);
+    if (tid == kIssuer) {
+      mma_out = false;
+      if (it_next >= 0) {  // M2 and T's parts read: the buffer takes the next [K; Q]
+        tc::fence_async_smem();
+        issue_kq(it_next);
+        kq_out = true;
+        kq_par = ph ^ 1u;
       }
     }
-    // the next item's values: T (over the values' buffer) has been read by MMA d
-    tc::fence_before_sync();
-    if (__syncthreads_or(bad)) break;
-    if (tid == kIssuer && it_next >= 0) {
-      tc::fence_async_smem();
-      issue_v(it_next);
-      v_out = true;
-      v_par = ph ^ 1u;
+
+    // ---- out[l][c] = s (Gam_{B-1} W^T[c][64 + l] + O2^T[c][l]); adjacent
+    // lanes swap one value so that each stores a bf16 pair of two columns
+    {
+      const float sG = p.scale * sh.Gc[B - 1];
+      const bool odd = lane & 1;
+      __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.out_blockend) +
+                           ((size_t)r * B * p.Hv + j) * kD6D + (tid & ~1);
+#pragma unroll 1
+      for (int h = 0; h < 2; ++h) {
+        const int t0 = 32 * h;
+        uint32_t o2[32], wq[32];
+        tc::tmem_ld16(tmG + lane_off + t0, *reinterpret_cast<uint32_t(*)[16]>(&o2[0]));
+        tc::tmem_ld16(tmG + lane_off + t0 + 16, *reinterpret_cast<uint32_t(*)[16]>(&o2[16]));
+        tc::tmem_ld16(tmW + lane_off + 64 + t0, *reinterpret_cast<uint32_t(*)[16]>(&wq[0]));
+        tc::tmem_ld16(tmW + lane_off + 64 + t0 + 16, *reinterpret_cast<uint32_t(*)[16]>(&wq[16]));
+        tc::tmem_ld_wait();
+#pragma unroll
+        for (int l = 0; l < 32; l += 2) {
+          const float a = fmaf(sG, __uint_as_float(wq[l]), p.scale * __uint_as_float(o2[l]));
+          const float b =
+              fmaf(sG, __uint_as_float(wq[l + 1]), p.scale * __uint_as_float(o2[l + 1]));
+          const float recv = __shfl_xor_sync(0xffffffffu, odd ? a : b, 1);
+          const int row = t0 + (odd ? l + 1 : l);
+          if (row < B)
+            *reinterpret_cast<uint32_t*>(out + (size_t)row * p.Hv * kD6D) =
+                odd ? ck_pack(recv, b) : ck_pack(a, recv);
+        }
+      }
     }
+    tc::fence_before_sync();
+    if (__syncthreads_or(bad)) break;  // the gates and tensor memory free for the next item
     if (it_next < 0) break;
     it = it_next;
     slot = slot_next;
@@ -483,7 +499,7 @@ __global__ void __launch_bounds__(kD6Threads, 1)
   __syncthreads();
   if (warp == 0) {
     tc::fence_after_sync();
-    tc::tmem_dealloc(tmem, 512);
+    tc::tmem_dealloc(tmem, 256);
   }
 }
 
@@ -542,7 +558,7 @@ cudaError_t launch_gdr_denoise_chunk64(const GdrParams& p, cudaStream_t stream) 
   if (cudaGetDevice(&dev) == cudaSuccess)
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const long items = (long)p.R * p.Hv;
-  const int grid = (int)(items < sms ? items : sms);
+  const int grid = (int)(items < 2L * sms ? items : 2L * sms);
   gdr_denoise_chunk64_kernel<<<grid, kD6Threads, smem, stream>>>(maps, p);
   note_launches(1);
   return cudaGetLastError();
