@@ -27,6 +27,12 @@ CASES = {
                                                      prefix_hi=70, seed=23),
     "ragged_block_b33": W["serving_batch64"].replace(num_requests=2, block_len=33, prefix_lo=0,
                                                      prefix_hi=70, seed=24),
+    # more (request, value head) items than the persistent kernel's CTAs, so
+    # that CTAs walk a second item with a ragged block
+    "ragged_block_b50_r12": W["serving_batch64"].replace(num_requests=12, block_len=50,
+                                                         prefix_lo=0, prefix_hi=70, seed=25),
+    "ragged_block_b27_r12": W["serving_batch64"].replace(num_requests=12, block_len=27,
+                                                         prefix_lo=0, prefix_hi=70, seed=26),
 }
 
 
