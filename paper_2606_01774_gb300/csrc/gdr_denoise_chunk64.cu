@@ -24,17 +24,19 @@
 // Rows past B read as zero (the block's tensor maps end at B), so A, M2 and X
 // vanish there and T is the identity.
 //
-// Persistent CTAs, two per SM (81 KiB of shared memory, 256 tensor-memory
+// Persistent CTAs, two per SM (113 KiB of shared memory, 256 tensor-memory
 // columns and 128 threads each), so that each SM holds two items' latency
-// chains.  The buffers serve twice: the state arrives in two 32 KiB halves
-// into one buffer that then holds A^T and T; the key/query buffer holds M2
-// and T's bf16 parts once the first MMAs have read it; delta^T's fp32 product
-// lands over W^T's key columns, which X has read.  The next item's first
-// state half is requested once T is formed, its keys and queries once the
-// second MMA has read M2, its values once X has read this item's; its gates
-// are loaded into registers one item ahead.  Every wait is bounded: on a
-// timeout the CTA sets FLARE_DEV_WAIT_TIMEOUT, waits (bounded) for its copies
-// and MMAs in flight, frees its tensor memory and exits.
+// chains.  The state arrives in two 32 KiB halves into two buffers: the first
+// half's buffer takes the next item's first half as soon as it has been read,
+// a whole item ahead; the second half's buffer then holds A^T and T, and takes
+// the next item's second half once T is formed.  The key/query buffer holds
+// M2 and T's bf16 parts once the first MMAs have read it; delta^T's fp32
+// product lands over W^T's key columns, which X has read.  The next item's
+// keys and queries are requested once the second MMA has read M2, its values
+// once X has read this item's; its gates are loaded into registers one item
+// ahead.  Every wait is bounded: on a timeout the CTA sets
+// FLARE_DEV_WAIT_TIMEOUT, waits (bounded) for its copies and MMAs in flight,
+// frees its tensor memory and exits.
 #include <cudaTypedefs.h>
 
 #include "chunk64.cuh"
@@ -50,31 +52,34 @@ constexpr int kD6Threads = 128;
 constexpr int kD6D = 128;  // d_k = d_v
 using namespace chunk64;   // kCkC = 64 and the chunk-system helpers
 
+struct alignas(16) D6Shared {
+  uint64_t bar_s0a, bar_s0b, bar_kq, bar_v, bar_g, bar_mma;
+  uint32_t tmem_base;
+  int abort_flag;
+  alignas(16) float gc2[kCkC];  // gamma_t log2(e)
+  alignas(16) float Gc[kCkC];   // exp(gamma_t)
+  alignas(16) float bc[kCkC];   // beta (zero past B)
+};
+
 struct D6Cfg {
   static constexpr int kS0h = 64 * kD6D * 4;   // half of S0 fp32: rows 64 h .. 64 h + 63
   static constexpr int kKQ = 2 * 128 * 128;    // [K; Q]: 2 chunks of 128 rows x 128 B (SW128)
   static constexpr int kV = 2 * kCkC * 128;    // values: 2 chunks of 64 rows x 128 B
   static constexpr int kT = kCkC * kCkC * 4;   // a 64 x 64 fp32 table
   static constexpr int kM2 = kCkC * 128;       // M2 [l][i] bf16, K-major SW128
-  static constexpr int oS0 = 0;                // the state half; then A^T and T
-  static constexpr int oAT = oS0;
-  static constexpr int oT = oS0 + kT;
-  static constexpr int oKQ = oS0 + kS0h;       // [K; Q]; then M2 and T's bf16 parts
+  static constexpr int oS0a = 0;               // the state's first half
+  static constexpr int oS0b = kS0h;            // its second half; then A^T and T
+  static constexpr int oAT = oS0b;
+  static constexpr int oT = oS0b + kT;
+  static constexpr int oKQ = 2 * kS0h;         // [K; Q]; then M2 and T's bf16 parts
   static constexpr int oM2 = oKQ;
   static constexpr int oTb = oKQ + kM2;        // T high, then low (8 KiB each)
   static constexpr int oV = oKQ + kKQ;
-  static constexpr int kSmem = oV + kV;
+  static constexpr int oSh = oV + kV;          // the barriers and gate factors
+  // two CTAs per SM: 2 (kSmem + the 1 KiB the system keeps per CTA) <= 228 KiB
+  static constexpr int kSmem = oSh + (int)sizeof(D6Shared);
   static_assert(2 * kT <= kS0h && kM2 + 2 * 8192 <= kKQ, "buffer reuse");
-};
-
-struct alignas(16) D6Shared {
-  uint64_t bar_s0, bar_kq, bar_v, bar_g, bar_mma;
-  uint32_t tmem_base;
-  int abort_flag;
-  alignas(16) float gc2[kCkC];  // gamma_t log2(e)
-  alignas(16) float Gc[kCkC];   // exp(gamma_t)
-  alignas(16) float bc[kCkC];   // beta (zero past B)
-  alignas(16) float eB[kCkC];   // exp(gamma_{B-1} - gamma_i) for i < B, else 0 (the M2 row factor)
+  static_assert(2 * (kSmem + 1024) <= 228 * 1024, "two CTAs per SM");
 };
 
 struct D6Maps {
@@ -104,10 +109,13 @@ __global__ void __launch_bounds__(kD6Threads, 2)
     gdr_denoise_chunk64_kernel(const __grid_constant__ D6Maps maps, GdrParams p) {
   using C = D6Cfg;
   constexpr int kIssuer = 32;  // one thread of warp 1 issues every copy and MMA
-  extern __shared__ uint8_t smem_raw[];
-  __shared__ D6Shared sh;
-  uint8_t* base = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  float* S0s = reinterpret_cast<float*>(base + C::oS0);
+  // no static shared memory, so that the dynamic window starts 1024-byte
+  // aligned (the 128-byte swizzled operands need it): checked below
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* base = smem_raw;
+  D6Shared& sh = *reinterpret_cast<D6Shared*>(base + C::oSh);
+  float* S0a = reinterpret_cast<float*>(base + C::oS0a);
+  float* S0b = reinterpret_cast<float*>(base + C::oS0b);
   float* AT = reinterpret_cast<float*>(base + C::oAT);
   float* Tf = reinterpret_cast<float*>(base + C::oT);
   uint8_t* KQ = base + C::oKQ;
@@ -122,10 +130,15 @@ __global__ void __launch_bounds__(kD6Threads, 2)
   int slot = 0;
   int it = d6_next(p, blockIdx.x, total, slot);
   if (it < 0) return;  // the same answer on every thread
+  if (tc::smem_u32(smem_raw) & 1023u) {  // a window the swizzled layout cannot use
+    if (tid == 0) flag(p.dev_status, FLARE_DEV_WAIT_TIMEOUT);
+    return;
+  }
 
   if (tid == kIssuer) {
     sh.abort_flag = 0;
-    tc::mbar_init(&sh.bar_s0, 1);
+    tc::mbar_init(&sh.bar_s0a, 1);
+    tc::mbar_init(&sh.bar_s0b, 1);
     tc::mbar_init(&sh.bar_kq, 1);
     tc::mbar_init(&sh.bar_v, 1);
     tc::mbar_init(&sh.bar_g, 1);
@@ -145,8 +158,9 @@ __global__ void __launch_bounds__(kD6Threads, 2)
   auto issue_s0 = [&](int item, int s, int h) {  // rows 64 h .. 64 h + 63 of the state
     const float* src = p.state_pool + ((size_t)s * p.Hv + item % p.Hv) * kD6D * kD6D +
                        (size_t)h * 64 * kD6D;
-    tc::mbar_expect_tx(&sh.bar_s0, C::kS0h);
-    tc::bulk_load(S0s, src, C::kS0h, &sh.bar_s0);
+    uint64_t* bar = h ? &sh.bar_s0b : &sh.bar_s0a;
+    tc::mbar_expect_tx(bar, C::kS0h);
+    tc::bulk_load(h ? S0b : S0a, src, C::kS0h, bar);
   };
   auto issue_kq = [&](int item) {
     const int r = item / p.Hv, h = (item % p.Hv) / (p.Hv / p.Hk);
@@ -178,18 +192,17 @@ __global__ void __launch_bounds__(kD6Threads, 2)
 
   // the issuing thread's record of what is in flight (and the parity its
   // barrier phase completes with), for a clean exit after a timeout
-  bool s0_out = false, kq_out = false, v_out = false, mma_out = false;
-  uint32_t s0_par = 0, kq_par = 0, v_par = 0;
-  uint32_t s0_ph = 0;  // parity of the state buffer's next completion (two per item)
+  bool s0a_out = false, s0b_out = false, kq_out = false, v_out = false, mma_out = false;
+  uint32_t s0a_par = 0, s0b_par = 0, kq_par = 0, v_par = 0;
   if (tid == kIssuer) {
     tc::prefetch_tmap(&maps.k);
     tc::prefetch_tmap(&maps.q);
     tc::prefetch_tmap(&maps.v);
     issue_s0(it, slot, 0);
+    issue_s0(it, slot, 1);
     issue_kq(it);
     issue_v(it);
-    s0_out = kq_out = v_out = true;
-    s0_par = 0;
+    s0a_out = s0b_out = kq_out = v_out = true;
   }
   if (warp == 0) load_gates(it);
   int cand = it + gridDim.x;
@@ -218,15 +231,12 @@ __global__ void __launch_bounds__(kD6Threads, 2)
       }
       x1 += __shfl_sync(0xffffffffu, x0, 31);
       const float g0 = x0 * 1.4426950408889634f, g1 = x1 * 1.4426950408889634f;
-      const float gB = __shfl_sync(0xffffffffu, g1, B - 33);  // B > 32
       sh.gc2[lane] = g0;
       sh.gc2[lane + 32] = g1;
       sh.Gc[lane] = expf(x0);
       sh.Gc[lane + 32] = expf(x1);
       sh.bc[lane] = ba;
       sh.bc[lane + 32] = bb;
-      sh.eB[lane] = lane < B ? tc::ex2(gB - g0) : 0.f;
-      sh.eB[lane + 32] = lane + 32 < B ? tc::ex2(gB - g1) : 0.f;
     }
     // the next item: the candidate when its slot is valid, else the first
     // valid one after it (bad ones flagged on the way)
@@ -245,33 +255,30 @@ __global__ void __launch_bounds__(kD6Threads, 2)
       cs = cand_slot(cand);
     }
 
-    // S0^T into tensor memory as bf16 pairs, the state in two halves through
-    // one buffer
+    // S0^T into tensor memory as bf16 pairs, the state's two halves from
+    // their two buffers
 #pragma unroll 1
     for (int h = 0; h < 2; ++h) {
-      bad |= !tc::mbar_wait(&sh.bar_s0, s0_ph, &sh.abort_flag);
-      s0_ph ^= 1u;
-      if (tid == kIssuer) s0_out = false;
+      bad |= !tc::mbar_wait(h ? &sh.bar_s0b : &sh.bar_s0a, ph, &sh.abort_flag);
+      const float* S0h = h ? S0b : S0a;
 #pragma unroll 1
       for (int i0 = 0; i0 < 64; i0 += 32) {
         uint32_t w[16];
 #pragma unroll
         for (int e = 0; e < 16; ++e)
-          w[e] = ck_pack(S0s[(i0 + 2 * e) * kD6D + tid], S0s[(i0 + 2 * e + 1) * kD6D + tid]);
+          w[e] = ck_pack(S0h[(i0 + 2 * e) * kD6D + tid], S0h[(i0 + 2 * e + 1) * kD6D + tid]);
         tc::tmem_st16(tmS + lane_off + (64 * h + i0) / 2, w);
       }
-      bad = __syncthreads_or(bad);  // this half read
-      if (bad) break;
-      if (h == 0 && tid == kIssuer) {
-        issue_s0(it, slot, 1);
-        s0_out = true;
-        s0_par = s0_ph;
-      }
     }
-    if (bad) break;
+    if (tid == kIssuer) s0a_out = s0b_out = false;
     tc::tmem_st_wait();
     tc::fence_before_sync();
-    if (__syncthreads_or(bad)) break;  // S0^T complete
+    if (__syncthreads_or(bad)) break;  // S0^T complete, both halves read
+    if (tid == kIssuer && it_next >= 0) {  // the first half's buffer is free
+      issue_s0(it_next, slot_next, 0);
+      s0a_out = true;
+      s0a_par = ph ^ 1u;
+    }
     if (tid == kIssuer) {
       bad |= !tc::mbar_wait(&sh.bar_kq, ph, &sh.abort_flag);
       kq_out = false;
@@ -321,6 +328,7 @@ __global__ void __launch_bounds__(kD6Threads, 2)
         tc::named_bar_arrive(5, 128);  // A^T to warps 2-3
       } else {
         const bool live = row < B;
+        const float gB = sh.gc2[B - 1];
         uint32_t wv[32];  // the row's 64 values as bf16 pairs
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
@@ -328,10 +336,12 @@ __global__ void __launch_bounds__(kD6Threads, 2)
           ck_ld32(tmG + lane_off + 32 * h, gr);
 #pragma unroll
           for (int e = 0; e < 16; ++e) {
+            // the row factor exp(gamma_{B-1} - gamma_i), zero for i >= B
             const int i = 32 * h + 2 * e;
-            const float m0 = sh.eB[i] * __uint_as_float(gr[2 * e]);
-            const float m1 = sh.eB[i + 1] * __uint_as_float(gr[2 * e + 1]);
-            wv[16 * h + e] = ck_pack(live ? m0 : 0.f, live ? m1 : 0.f);
+            const float m0 = tc::ex2(gB - sh.gc2[i]) * __uint_as_float(gr[2 * e]);
+            const float m1 = tc::ex2(gB - sh.gc2[i + 1]) * __uint_as_float(gr[2 * e + 1]);
+            wv[16 * h + e] =
+                ck_pack(live && i < B ? m0 : 0.f, live && i + 1 < B ? m1 : 0.f);
           }
         }
         bad |= !tc::mbar_wait(&sh.bar_mma, ph_mma, &sh.abort_flag);  // [K; Q] read
@@ -393,10 +403,10 @@ __global__ void __launch_bounds__(kD6Threads, 2)
       ck_tcol<32>(AT, Tf, Tb, warp - 1, warp == 2 ? 1 : 2, lane, warp);
     if (__syncthreads_or(bad)) break;  // T as bf16 high / low parts; A^T and T read
     if (tid == kIssuer) {
-      if (it_next >= 0) {  // the state buffer is free: the next item's first half
-        issue_s0(it_next, slot_next, 0);
-        s0_out = true;
-        s0_par = s0_ph;
+      if (it_next >= 0) {  // A^T and T read: the next item's second half
+        issue_s0(it_next, slot_next, 1);
+        s0b_out = true;
+        s0b_par = ph ^ 1u;
       }
       const uint32_t tb = tc::smem_u32(Tb);
 #pragma unroll
@@ -490,7 +500,8 @@ __global__ void __launch_bounds__(kD6Threads, 2)
     flag(p.dev_status, FLARE_DEV_WAIT_TIMEOUT);
   }
   if (tid == kIssuer && bad) {
-    if (s0_out) tc::mbar_wait(&sh.bar_s0, s0_par, nullptr, 100000000ull);
+    if (s0a_out) tc::mbar_wait(&sh.bar_s0a, s0a_par, nullptr, 100000000ull);
+    if (s0b_out) tc::mbar_wait(&sh.bar_s0b, s0b_par, nullptr, 100000000ull);
     if (kq_out) tc::mbar_wait(&sh.bar_kq, kq_par, nullptr, 100000000ull);
     if (v_out) tc::mbar_wait(&sh.bar_v, v_par, nullptr, 100000000ull);
     if (mma_out) tc::mbar_wait(&sh.bar_mma, ph_mma, nullptr, 100000000ull);
@@ -550,7 +561,7 @@ cudaError_t launch_gdr_denoise_chunk64(const GdrParams& p, cudaStream_t stream) 
       !d6_act_map(&maps.q, p.q, p.Hk, p.B, p.R, true) ||
       !d6_act_map(&maps.v, p.v, p.Hv, p.B, p.R, false))
     return cudaErrorInvalidValue;
-  const int smem = D6Cfg::kSmem + 1024;
+  const int smem = D6Cfg::kSmem;
   cudaError_t e = cudaFuncSetAttribute(gdr_denoise_chunk64_kernel,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
