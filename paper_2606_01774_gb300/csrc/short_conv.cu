@@ -7,25 +7,26 @@
 // clean stream) for lags that cross the block start; then bias and SiLU.
 //
 // The kernel is a pure stream (each input byte is used W times from on-chip
-// memory), so it is built to keep HBM busy: persistent CTAs, one per SM, walk
-// work items (request, 4 KiB channel slab, chunk of up to 8 block rows; small
-// items keep the last wave short).  A producer warp stages each item's rows --
-// the chunk plus the W - 1 rows before it, from the block or, for the first
-// chunk, from the conv state -- in shared memory: when the channels tile by
-// 512 bytes as one tensor-map box of (512 bytes x 8) x rows per item (the
+// memory), so it is built to keep HBM busy: persistent CTAs (two per SM for
+// bf16, one for fp32) walk work items (request, channel slab, chunk of up to 8
+// block rows).  A slab is 512 columns of a channel pair each: 2 KiB of bf16 or
+// 4 KiB of fp32 channels.  A producer warp stages each item's rows -- the
+// chunk plus the W - 1 rows before it, from the block or, for the first chunk,
+// from the conv state -- in shared memory: when the channels tile by 512 bytes
+// as one tensor-map box of (512 bytes x the slab's blocks) x rows per item (the
 // state rows of a first chunk as bulk copies), else one bulk copy per row;
 // completion counted on the stage's full barrier (a few large copies keep far
-// more bytes in flight per SM than a copy per 4 KiB row); four stages, so three
+// more bytes in flight per SM than a copy per row); four stages, so three
 // items' rows are in flight while 512 compute threads convolve the current
-// one, a thread per 8 bytes of channels (4 bf16 or 2 fp32) down the whole
-// chunk with its filter taps and a sliding window in registers, writing
-// 8-byte outputs coalesced across the slab; they release the stage on its
-// empty barrier.
+// one, a thread per channel pair down the whole chunk with its filter taps
+// and a sliding window in registers, writing its pair coalesced across the
+// slab; they release the stage on its empty barrier.  The producer also
+// leaves each stage's item coordinates in shared memory.
 // The arithmetic runs on fp32 pairs (packed f32x2 multiply-add); the SiLU's
-// exponentials run on the special-function unit, its reciprocals one per four
-// channels (the special-function unit is the busiest pipe here).  With a grid that
-// is a multiple of the slab count every CTA keeps one slab, so the filter taps
-// are loaded once, while the first rows are on their way.
+// exponentials run on the special-function unit, its reciprocals one per
+// channel pair.  With a grid that is a multiple of the slab count every CTA
+// keeps one slab, so the filter taps are loaded once, while the first rows are
+// on their way.
 // The state commit (last W - 1 rows of old state ++ accepted rows) is a bit
 // copy done by the threads of each slab's first chunk, the only ones that read
 // the old state of those channels, after their reads.
@@ -39,14 +40,21 @@
 namespace flare {
 
 namespace {
-constexpr int kConvThreads = 512;             // a thread per 8-byte column
-constexpr int kColBytes = 8;
-constexpr int kSlabBytes = kConvThreads * kColBytes;  // 4 KiB of channels per item
+constexpr int kConvThreads = 512;              // compute threads, a channel pair each
 constexpr int kChunkRows = 8;                  // block rows per item
 constexpr int kMaxStageRows = kChunkRows + 3;  // with the W - 1 <= 3 rows before the chunk
-constexpr int kStageBytes = kMaxStageRows * kSlabBytes;
 constexpr int kStages = 4;
-constexpr size_t kConvSmem = kStages * (size_t)kStageBytes;
+// A column of the slab is a channel pair: 4 bytes (bf16: 2 KiB slabs, 88 KiB
+// of stages, two CTAs per SM) or 8 bytes (fp32: 4 KiB slabs, 176 KiB, one)
+template <typename T>
+struct ConvCols {
+  static constexpr int kColBytes = 2 * (int)sizeof(T);
+  static constexpr int kSlabBytes = kConvThreads * kColBytes;
+  static constexpr int kBoxBlocks = kSlabBytes / 512;  // 512-byte tensor-map blocks per slab
+  static constexpr int kStageBytes = kMaxStageRows * kSlabBytes;
+  static constexpr int kSmem = kStages * kStageBytes;
+  static constexpr int kCtasPerSM = sizeof(T) == 2 ? 2 : 1;
+};
 
 struct ConvItem {
   int r, slab, chunk;
@@ -82,36 +90,33 @@ __device__ __forceinline__ float rcp_approx(float x) {
   return y;
 }
 
-// 8 bytes of T as V / 2 fp32 pairs (bf16 widens exactly: its bits are the
-// high half of the fp32 pattern)
-template <typename T>
-__device__ __forceinline__ void unpack8(const uint2& raw, uint64_t* f) {
-  if constexpr (sizeof(T) == 2) {
-    f[0] = f2(__uint_as_float(raw.x << 16), __uint_as_float(raw.x & 0xffff0000u));
-    f[1] = f2(__uint_as_float(raw.y << 16), __uint_as_float(raw.y & 0xffff0000u));
-  } else {
-    f[0] = f2(__uint_as_float(raw.x), __uint_as_float(raw.y));
-  }
+// A column (two channels) of T as an fp32 pair, and back; bf16 widens
+// exactly (its bits are the high half of the fp32 pattern)
+__device__ __forceinline__ uint64_t unpack_col(uint32_t raw) {
+  return f2(__uint_as_float(raw << 16), __uint_as_float(raw & 0xffff0000u));
 }
-
-template <typename T>
-__device__ __forceinline__ uint2 pack8(const uint64_t* f) {
-  if constexpr (sizeof(T) == 2) {
-    uint32_t u[2];
-#pragma unroll
-    for (int k = 0; k < 2; ++k) {
-      float lo, hi;
-      f2_split(f[k], lo, hi);
-      __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
-      u[k] = *reinterpret_cast<uint32_t*>(&h);
-    }
-    return make_uint2(u[0], u[1]);
-  } else {
-    float lo, hi;
-    f2_split(f[0], lo, hi);
-    return make_uint2(__float_as_uint(lo), __float_as_uint(hi));
-  }
+__device__ __forceinline__ uint64_t unpack_col(uint2 raw) {
+  return f2(__uint_as_float(raw.x), __uint_as_float(raw.y));
 }
+__device__ __forceinline__ void pack_col(uint64_t f, uint32_t& out) {
+  float lo, hi;
+  f2_split(f, lo, hi);
+  __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  out = *reinterpret_cast<uint32_t*>(&h);
+}
+__device__ __forceinline__ void pack_col(uint64_t f, uint2& out) {
+  float lo, hi;
+  f2_split(f, lo, hi);
+  out = make_uint2(__float_as_uint(lo), __float_as_uint(hi));
+}
+template <typename T>
+struct ColWord {
+  using type = uint32_t;
+};
+template <>
+struct ColWord<float> {
+  using type = uint2;
+};
 
 // A request is valid when its slot and (for a committing call) its accepted
 // length are in range; otherwise its items are skipped.
@@ -127,14 +132,19 @@ __device__ __forceinline__ int conv_check(const ConvParams& p, int r) {
 }  // namespace
 
 template <typename T, int W>
-__global__ void __launch_bounds__(kConvThreads + 32, 1)
+__global__ void __launch_bounds__(kConvThreads + 32, ConvCols<T>::kCtasPerSM)
     short_conv_kernel(const __grid_constant__ ConvMaps maps, ConvParams p) {
   constexpr int E = sizeof(T);
-  constexpr int V = kColBytes / E;  // channels per thread
-  constexpr int P = V / 2;          // fp32 pairs per thread
-  constexpr int H = W - 1;          // rows before a chunk
+  constexpr int kColBytes = ConvCols<T>::kColBytes;
+  constexpr int kSlabBytes = ConvCols<T>::kSlabBytes;
+  constexpr int kStageBytes = ConvCols<T>::kStageBytes;
+  constexpr int H = W - 1;  // rows before a chunk
+  using Col = typename ColWord<T>::type;
   extern __shared__ __align__(128) uint8_t conv_smem[];
   __shared__ uint64_t full[kStages], empty[kStages];
+  // per stage, written by the producer: the item's request, slab and chunk,
+  // the request's slot, accepted length and validity
+  __shared__ int st_r[kStages], st_slab[kStages], st_chunk[kStages];
   __shared__ int st_bad[kStages], st_slot[kStages], st_n[kStages];
   __shared__ int abort_flag, n_issued;
 
@@ -182,6 +192,9 @@ __global__ void __launch_bounds__(kConvThreads + 32, 1)
         const int rows = min(kChunkRows, p.B - l0);
         uint8_t* dst = conv_smem + (size_t)st * kStageBytes;
         const int bad = conv_check(p, it.r);
+        st_r[st] = it.r;
+        st_slab[st] = it.slab;
+        st_chunk[st] = it.chunk;
         st_bad[st] = bad;
         n_issued = k + 1;
         if (bad) {  // nothing to load; the stage completes empty
@@ -202,10 +215,11 @@ __global__ void __launch_bounds__(kConvThreads + 32, 1)
               tc::bulk_load(dst + (size_t)j * kSlabBytes,
                             sg + ((size_t)slot * H + j) * row_bytes + off, bytes, &full[st]);
             tc::tma_load_3d(dst + (size_t)H * kSlabBytes, &maps.x_first, &full[st], 0,
-                            it.slab * 8, row0);
+                            it.slab * ConvCols<T>::kBoxBlocks, row0);
           } else {
             tc::mbar_expect_tx(&full[st], (uint32_t)(kSlabBytes * (kChunkRows + H)));
-            tc::tma_load_3d(dst, &maps.x_halo, &full[st], 0, it.slab * 8, row0 - H);
+            tc::tma_load_3d(dst, &maps.x_halo, &full[st], 0, it.slab * ConvCols<T>::kBoxBlocks,
+                            row0 - H);
           }
         } else {
           tc::mbar_expect_tx(&full[st], bytes * (uint32_t)(H + rows));
@@ -220,41 +234,28 @@ __global__ void __launch_bounds__(kConvThreads + 32, 1)
     }
   } else {
     const int col = tid;
-    uint64_t w2[P][W], b2[P];
+    uint64_t w2[W], b2;  // this thread's two channels: taps and bias as fp32 pairs
     int cur_slab = -1;
-    // filter taps and bias of this thread's channels, paired (loaded while the
-    // first item's rows are on their way, and again only if the slab changes)
+    // filter taps and bias of this thread's channels (loaded while the first
+    // item's rows are on their way, and again only if the slab changes)
     auto load_taps = [&](int slab) {
       cur_slab = slab;
       const size_t off = (size_t)slab * kSlabBytes + (size_t)col * kColBytes;
       if (off >= row_bytes) return;
       const int c0 = (int)(off / E);
       const float2* w2p = reinterpret_cast<const float2*>(p.weight + (size_t)c0 * W);
-      float wf[V * W];
+      float wf[2 * W];
 #pragma unroll
-      for (int q = 0; q < V * W / 2; ++q) {
+      for (int q = 0; q < W; ++q) {
         const float2 v = __ldg(w2p + q);
         wf[2 * q] = v.x;
         wf[2 * q + 1] = v.y;
       }
-      float bf[V];
+      float2 bf = make_float2(0.f, 0.f);
+      if (p.bias) bf = __ldg(reinterpret_cast<const float2*>(p.bias + c0));
 #pragma unroll
-      for (int v = 0; v < V; ++v) bf[v] = 0.f;
-      if (p.bias) {
-        const float2* b2p = reinterpret_cast<const float2*>(p.bias + c0);
-#pragma unroll
-        for (int q = 0; q < V / 2; ++q) {
-          const float2 v = __ldg(b2p + q);
-          bf[2 * q] = v.x;
-          bf[2 * q + 1] = v.y;
-        }
-      }
-#pragma unroll
-      for (int q = 0; q < P; ++q) {
-#pragma unroll
-        for (int i = 0; i < W; ++i) w2[q][i] = f2(wf[2 * q * W + i], wf[(2 * q + 1) * W + i]);
-        b2[q] = f2(bf[2 * q], bf[2 * q + 1]);
-      }
+      for (int i = 0; i < W; ++i) w2[i] = f2(wf[i], wf[W + i]);
+      b2 = f2(bf.x, bf.y);
     };
     if ((int)blockIdx.x < n_items) load_taps(conv_item(blockIdx.x, n_slabs, n_chunks).slab);
     const uint64_t neg_log2e = f2(-1.4426950408889634f, -1.4426950408889634f);
@@ -267,66 +268,48 @@ __global__ void __launch_bounds__(kConvThreads + 32, 1)
         abort_flag = 1;
         break;
       }
-      const ConvItem it = conv_item(idx, n_slabs, n_chunks);
-      const size_t off = (size_t)it.slab * kSlabBytes + (size_t)col * kColBytes;
-      const int l0 = it.chunk * kChunkRows;
+      const int ir = st_r[st], islab = st_slab[st], ichunk = st_chunk[st];
+      const size_t off = (size_t)islab * kSlabBytes + (size_t)col * kColBytes;
+      const int l0 = ichunk * kChunkRows;
       const int rows = min(kChunkRows, p.B - l0);
       const int bad = st_bad[st];
       if (bad) {
-        if (tid == 0 && it.slab == 0 && it.chunk == 0) flag(p.dev_status, bad);
+        if (tid == 0 && islab == 0 && ichunk == 0) flag(p.dev_status, bad);
       } else {
-        if (it.slab != cur_slab) load_taps(it.slab);
+        if (islab != cur_slab) load_taps(islab);
         if (off < row_bytes) {
           const uint8_t* stage = conv_smem + (size_t)st * kStageBytes + (size_t)col * kColBytes;
           // sliding window: win[i] holds row l - i of the current output row l;
           // before the first row it holds the H rows before the chunk (stage rows H - 1 - i)
-          uint64_t win[W][P];
+          uint64_t win[W];
 #pragma unroll
           for (int i = 0; i < H; ++i)
-            unpack8<T>(*reinterpret_cast<const uint2*>(stage + (size_t)(H - 1 - i) * kSlabBytes),
-                       win[i]);
-          char* outg = static_cast<char*>(p.out) + ((size_t)it.r * p.B + l0) * row_bytes + off;
+            win[i] = unpack_col(*reinterpret_cast<const Col*>(stage + (size_t)(H - 1 - i) * kSlabBytes));
+          char* outg = static_cast<char*>(p.out) + ((size_t)ir * p.B + l0) * row_bytes + off;
           // one output row: shift the window, read row j, convolve, SiLU, store
           auto row_out = [&](int j) {
 #pragma unroll
-            for (int i = W - 1; i > 0; --i)
+            for (int i = W - 1; i > 0; --i) win[i] = win[i - 1];
+            win[0] = unpack_col(*reinterpret_cast<const Col*>(stage + (size_t)(H + j) * kSlabBytes));
+            uint64_t y = b2;
 #pragma unroll
-              for (int q = 0; q < P; ++q) win[i][q] = win[i - 1][q];
-            unpack8<T>(*reinterpret_cast<const uint2*>(stage + (size_t)(H + j) * kSlabBytes),
-                       win[0]);
-            uint64_t y[P];
-#pragma unroll
-            for (int q = 0; q < P; ++q) {
-              uint64_t acc = b2[q];
-#pragma unroll
-              for (int i = 0; i < W; ++i) acc = f2_fma(w2[q][i], win[i][q], acc);
-              y[q] = acc;
-            }
+            for (int i = 0; i < W; ++i) y = f2_fma(w2[i], win[i], y);
             if (p.silu) {
-              // SiLU u / d with d = 1 + 2^(-u log2 e), the channels of the
-              // thread sharing one reciprocal: 1/d_a = (prod_{b != a} d_b) / prod d.
-              // The exponent is capped at 30 so the product of four stays below
-              // 2^124; that changes only outputs below 2^-25 |u|.
-              float u[V], t[V], d[V];
-#pragma unroll
-              for (int q = 0; q < P; ++q) {
-                f2_split(y[q], u[2 * q], u[2 * q + 1]);
-                f2_split(f2_mul(y[q], neg_log2e), t[2 * q], t[2 * q + 1]);
-              }
-#pragma unroll
-              for (int e = 0; e < V; ++e) d[e] = 1.f + ex2_approx(fminf(t[e], 30.f));
-              if constexpr (V == 4) {
-                const float d01 = d[0] * d[1], d23 = d[2] * d[3];
-                const float r = rcp_approx(d01 * d23);
-                const float r01 = r * d23, r23 = r * d01;  // 1/(d0 d1), 1/(d2 d3)
-                y[0] = f2(u[0] * (r01 * d[1]), u[1] * (r01 * d[0]));
-                y[1] = f2(u[2] * (r23 * d[3]), u[3] * (r23 * d[2]));
-              } else {
-                const float r = rcp_approx(d[0] * d[1]);
-                y[0] = f2(u[0] * (r * d[1]), u[1] * (r * d[0]));
-              }
+              // SiLU u / d with d = 1 + 2^(-u log2 e), the two channels sharing
+              // one reciprocal: 1/d_a = d_b / (d_a d_b).  The exponent is capped
+              // at 60 so the product of two stays below 2^121; that changes only
+              // outputs below 2^-60 |u|.
+              float u0, u1, t0, t1;
+              f2_split(y, u0, u1);
+              f2_split(f2_mul(y, neg_log2e), t0, t1);
+              const float d0 = 1.f + ex2_approx(fminf(t0, 60.f));
+              const float d1 = 1.f + ex2_approx(fminf(t1, 60.f));
+              const float r = rcp_approx(d0 * d1);
+              y = f2_mul(y, f2_mul(f2_dup(r), f2(d1, d0)));
             }
-            *reinterpret_cast<uint2*>(outg + (size_t)j * row_bytes) = pack8<T>(y);
+            Col o;
+            pack_col(y, o);
+            *reinterpret_cast<Col*>(outg + (size_t)j * row_bytes) = o;
           };
           if (rows == kChunkRows) {
             // a whole chunk: no guards, so the window shifts are renamings
@@ -341,20 +324,20 @@ __global__ void __launch_bounds__(kConvThreads + 32, 1)
           // the old rows of the first chunk are still in the stage
           if constexpr (H > 0) {
             const int n = st_n[st];
-            if (n >= 0 && it.chunk == 0) {
+            if (n >= 0 && ichunk == 0) {
               const int slot = st_slot[st];
-              uint2 nw[H];
+              Col nw[H];
 #pragma unroll
               for (int j = 0; j < H; ++j) {
                 const int pos = n - H + j;
-                nw[j] = pos >= 0 ? __ldg(reinterpret_cast<const uint2*>(
-                                       xg + ((size_t)it.r * p.B + pos) * row_bytes + off))
-                                 : *reinterpret_cast<const uint2*>(
+                nw[j] = pos >= 0 ? *reinterpret_cast<const Col*>(
+                                       xg + ((size_t)ir * p.B + pos) * row_bytes + off)
+                                 : *reinterpret_cast<const Col*>(
                                        stage + (size_t)(H + pos) * kSlabBytes);
               }
 #pragma unroll
               for (int j = 0; j < H; ++j)
-                *reinterpret_cast<uint2*>(sg + ((size_t)slot * H + j) * row_bytes + off) = nw[j];
+                *reinterpret_cast<Col*>(sg + ((size_t)slot * H + j) * row_bytes + off) = nw[j];
             }
           }
         }
@@ -385,7 +368,8 @@ PFN_cuTensorMapEncodeTiled_v12000 sc_encode_fn() {
   return fn;
 }
 
-// x [R B, C] of T as (D0, C / D0, R B) with D0 = 512 / sizeof(T), box (D0, 8, rows)
+// x [R B, C] of T as (D0, C / D0, R B) with D0 = 512 / sizeof(T), box (D0, a
+// slab's blocks, rows)
 template <typename T>
 bool sc_map(CUtensorMap* m, const void* x, int C, long rows_total, int box_rows) {
   auto fn = sc_encode_fn();
@@ -393,7 +377,7 @@ bool sc_map(CUtensorMap* m, const void* x, int C, long rows_total, int box_rows)
   constexpr int D0 = 512 / (int)sizeof(T);
   cuuint64_t gd[3] = {(cuuint64_t)D0, (cuuint64_t)(C / D0), (cuuint64_t)rows_total};
   cuuint64_t gs[2] = {(cuuint64_t)512, (cuuint64_t)C * sizeof(T)};
-  cuuint32_t bx[3] = {(cuuint32_t)D0, 8, (cuuint32_t)box_rows};
+  cuuint32_t bx[3] = {(cuuint32_t)D0, (cuuint32_t)ConvCols<T>::kBoxBlocks, (cuuint32_t)box_rows};
   cuuint32_t es[3] = {1, 1, 1};
   return fn(m, sizeof(T) == 2 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32,
             3, const_cast<void*>(x), gd, gs, bx, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
@@ -405,7 +389,7 @@ template <typename T, int W>
 cudaError_t launch_conv_w(const ConvParams& p, int grid, cudaStream_t stream) {
   cudaError_t e = cudaFuncSetAttribute(short_conv_kernel<T, W>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)kConvSmem);
+                                       ConvCols<T>::kSmem);
   if (e != cudaSuccess) return e;
   ConvMaps maps;
   memset(&maps, 0, sizeof maps);
@@ -413,7 +397,7 @@ cudaError_t launch_conv_w(const ConvParams& p, int grid, cudaStream_t stream) {
   if (p.C % (512 / (int)sizeof(T)) == 0 && rows_total < (1l << 31))
     maps.use = sc_map<T>(&maps.x_halo, p.x, p.C, rows_total, kChunkRows + W - 1) &&
                sc_map<T>(&maps.x_first, p.x, p.C, rows_total, kChunkRows);
-  short_conv_kernel<T, W><<<grid, kConvThreads + 32, kConvSmem, stream>>>(maps, p);
+  short_conv_kernel<T, W><<<grid, kConvThreads + 32, ConvCols<T>::kSmem, stream>>>(maps, p);
   note_launches(1);
   return cudaGetLastError();
 }
@@ -421,12 +405,14 @@ cudaError_t launch_conv_w(const ConvParams& p, int grid, cudaStream_t stream) {
 template <typename T>
 cudaError_t launch_conv_t(const ConvParams& p, cudaStream_t stream) {
   const size_t row_bytes = (size_t)p.C * sizeof(T);
-  const long n_slabs = (long)((row_bytes + kSlabBytes - 1) / kSlabBytes);
+  constexpr int kSlab = ConvCols<T>::kSlabBytes;
+  const long n_slabs = (long)((row_bytes + kSlab - 1) / kSlab);
   const long items = (long)p.R * n_slabs * ((p.B + kChunkRows - 1) / kChunkRows);
   int dev = 0, sms = kNumSMs;
   if (cudaGetDevice(&dev) == cudaSuccess)
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  int grid = (int)(items < sms ? items : sms);
+  const long ctas = (long)ConvCols<T>::kCtasPerSM * sms;
+  int grid = (int)(items < ctas ? items : ctas);
   if (n_slabs <= grid) grid = grid / (int)n_slabs * (int)n_slabs;  // one slab per CTA
   switch (p.W) {
     case 1: return launch_conv_w<T, 1>(p, grid, stream);
