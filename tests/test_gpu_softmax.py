@@ -122,3 +122,31 @@ def test_nan_poisoned_pool_does_not_leak():
     for mode in (0, 1):
         out, lse = run_softmax(w, 0, mode)
         assert torch.isfinite(out.float()).all() and torch.isfinite(lse).all()
+
+
+def test_more_requests_than_the_prepass_holds_on_chip():
+    # 4100 requests: the validation pre-pass keeps the prefix lengths and the
+    # bad requests of at most 4096 in shared memory, so this call takes its
+    # global-memory path; one bad page on each side of that bound
+    spec = W["tiny_fp32"].replace(name="many_requests", act_dtype="bf16", num_requests=4100,
+                                  prefix_lo=1, prefix_hi=40, seed=45)
+    w = gen(spec)
+    bad = (5, 4099)
+    for r in bad:
+        w.page_table[r, 0] = w.k_pool.shape[0]
+    sb = w.softmax[0]
+    desc = softmax_desc(spec, w)
+    nb = flare.flare_softmax_workspace_size(desc)
+    ws = torch.empty(max(nb, 1), dtype=torch.uint8, device="cuda")
+    out = torch.full_like(sb.q, 5.0)
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    flare.check(flare.flare_block_softmax_attn(desc, sb.q, sb.k_blk, sb.v_blk, w.k_pool,
+                                               w.v_pool, w.page_table, w.prefix_len, out, None,
+                                               ws, nb, st))
+    rc, bits = flare.flare_read_status(st)
+    assert rc == flare.FLARE_ERR_DEVICE_STATUS and bits == flare.FLARE_DEV_BAD_PAGE
+    for r in bad:
+        assert (out[r] == 5.0).all()
+    sample = [0, 6, 4095, 4096, 4098]
+    ref, _ = oracle_softmax(w, 0, requests=sample)
+    assert_out_close(out[sample], ref, spec.act_dtype, "many requests")
