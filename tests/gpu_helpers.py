@@ -10,8 +10,9 @@ import torch
 import oracle
 from paper_2606_01774_gb300 import flare, workloads
 
-# Tolerances (spec: max-abs 2e-2 on bf16 outputs, relative Frobenius 1e-3 on
-# fp32 committed states).  The tighter relative bounds on outputs follow from the
+# Tolerances (the accuracy the serving path must keep: max-abs 2e-2 on bf16
+# outputs, relative Frobenius 1e-3 on fp32 committed states).  The tighter
+# relative bounds on outputs follow from the
 # arithmetic: bf16 output rounding is 2^-9 relative, bf16 tensor-core operands
 # add a few 2^-9 more; fp32 paths carry ~1e-6.
 OUT_MAX_ABS = 2e-2
