@@ -63,7 +63,7 @@ extern "C" {
 typedef enum flare_status {
   FLARE_OK = 0,
   FLARE_ERR_INVALID_ARGUMENT = 1, /* null pointer, inconsistent sizes */
-  FLARE_ERR_UNSUPPORTED = 2,      /* sizes or dtypes this build does not implement */
+  FLARE_ERR_UNSUPPORTED = 2,      /* sizes or dtypes the library does not implement */
   FLARE_ERR_CUDA = 3,             /* a CUDA runtime call failed (launch, attribute) */
   FLARE_ERR_DEVICE_STATUS = 4     /* flare_read_status found device error bits */
 } flare_status;
