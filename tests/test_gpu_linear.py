@@ -81,6 +81,23 @@ def test_denoise_full_size_every_request(name):
     assert_out_close(out, ref, spec.act_dtype, name)
 
 
+@pytest.mark.parametrize("name", ["serving_batch64_r3", "small_model_batch256_r4",
+                                  "multistep_batch128_r3", "d64_bf16"])
+def test_denoise_strong_decay(name):
+    """Log-gates of -3 per token on every other value head: the block's running
+    decay falls below the fp32 range inside the block (Gam_{B-1} is 0 in fp32 at
+    B = 64) and the masked exponentials of A and M2 overflow; half the heads
+    keep the ordinary gates.  Same oracle, same tolerances."""
+    spec = CASES[name]
+    w = gen(spec)
+    w.denoise[0].log_decay[:, :, ::2] = -3.0
+    install_states(w)
+    out = run_linear(w, 0)
+    ref = oracle_linear(w, 0)
+    assert torch.isfinite(out.float()).all()
+    assert_out_close(out, ref, spec.act_dtype, f"{name} strong decay")
+
+
 def test_denoise_is_bidirectional_readout():
     """All block rows read the block-end state: equal queries give equal rows."""
     spec = CASES["serving_batch64_r3"]
