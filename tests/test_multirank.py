@@ -37,7 +37,9 @@ def _worker(rank, world, port, out):
 
 def test_max_over_ranks_with_gloo():
     world = 2
-    mgr = mp.Manager()
+    # the manager's server process is spawned too: forking a process whose
+    # earlier tests started torch's CPU threads can deadlock the child
+    mgr = mp.get_context("spawn").Manager()
     out = mgr.dict()
     mp.spawn(_worker, args=(world, _free_port(), out), nprocs=world, join=True)
     assert dict(out) == {0: 2.5, 1: 2.5}
